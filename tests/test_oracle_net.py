@@ -1,0 +1,189 @@
+"""Pins of the oracle's scoring network (Sec. 3.2; App. A; Table "hparams").
+
+The network's values are parity unpinned against any paper number (no weights or
+worked example are published). What is pinned: the architecture, by the
+parameter counts the paper prints; each component, by an independent library
+implementation (torch RMSNorm, multi-head attention, SiLU); and structural
+properties the paper states (shared hidden term per slot, bidirectional
+attention, unit-norm out/in vectors, cosine range)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as Fn
+
+import oracle
+import workloads
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def test_param_count_matches_paper():
+    g = json.load(open(os.path.join(GOLD, "param_counts.json")))
+    for c in g["cases"]:
+        n = oracle.param_count(c["H"], c["D"], c["d"], c["F"], c["n_heads"], c["L"], c["K"],
+                               c["n_layers"])
+        assert round(n / 1e6, 2) == c["millions"], n
+
+
+def test_alternative_readings_miss_the_paper_count():
+    # a gated FFN, concatenated target layers or bias-free linears all miss 36.76M
+    base = oracle.param_count(4096, 1024, 1024, 2048, 8, 15, 8)
+    gated = base + 2 * (1024 * 2048 + 2048)
+    concat5 = base + 4 * 4096 * 1024 + 4 * 4096
+    n_lin_bias = 4 + 2 + 2 * 6 + 1 + 3
+    assert round(base / 1e6, 2) == 36.76
+    for alt in (gated, concat5):
+        assert round(alt / 1e6, 2) != 36.76
+    assert round((base - n_lin_bias * 1024 - 2 * 1024) / 1e6, 2) != 36.76
+
+
+def test_generator_shapes_follow_oracle_architecture():
+    for name in workloads.WORKLOAD_ORDER:
+        wl = workloads.WORKLOADS[name]
+        gen = dict(workloads.head_param_shapes(wl.H, wl.D, wl.d, wl.F, wl.n_heads, wl.L, wl.K))
+        want = oracle.param_shapes(wl.H, wl.D, wl.d, wl.F, wl.n_heads, wl.L, wl.K)
+        assert gen == want
+
+
+def test_confidence_features_golden():
+    g = json.load(open(os.path.join(GOLD, "conf_features.json")))
+    f = oracle.confidence_features(np.array(g["logp"]))
+    assert np.allclose(f, np.array(g["features"]), atol=1e-15)
+    f1 = oracle.confidence_features(np.array([-0.7]))
+    assert np.allclose(f1, [[-0.7, np.exp(-0.7), 0.0, 0.0, 1.0]])
+
+
+def test_rms_norm_matches_torch():
+    rng = np.random.default_rng(0)
+    x = rng.standard_normal((9, 64)) * 3
+    g = 1 + 0.1 * rng.standard_normal(64)
+    want = Fn.rms_norm(torch.from_numpy(x), (64,), weight=torch.from_numpy(g), eps=1e-6)
+    assert np.allclose(oracle.rms_norm(x, g), want.numpy(), atol=1e-13)
+
+
+def test_silu_matches_torch():
+    z = np.linspace(-30, 30, 1001)
+    assert np.allclose(oracle.silu(z), Fn.silu(torch.from_numpy(z)).numpy(), atol=1e-14)
+
+
+def _rand_layer(rng, D, nh, L, scale=0.3):
+    W = {}
+    for n in ("wq", "wk", "wv", "wo"):
+        W["l0." + n] = rng.standard_normal((D, D)) * scale
+    for n in ("bq", "bk", "bv", "bo"):
+        W["l0." + n] = rng.standard_normal(D) * scale
+    W["l0.dist"] = rng.standard_normal((nh, 2 * L - 1))
+    W["l0.same"] = rng.standard_normal(nh)
+    return W
+
+
+def test_attention_matches_torch_multi_head_attention():
+    rng = np.random.default_rng(1)
+    L, K, D, nh = 5, 3, 32, 8
+    N = L * K
+    W = _rand_layer(rng, D, nh, L)
+    x = rng.standard_normal((N, D))
+    got = oracle.attention(x, W, "l0.", L, K, nh)
+    slot = np.arange(N) // K
+    mask = np.zeros((nh, N, N))
+    for h in range(nh):
+        for i in range(N):
+            for j in range(N):
+                mask[h, i, j] = W["l0.dist"][h, slot[j] - slot[i] + L - 1] + \
+                    (W["l0.same"][h] if slot[i] == slot[j] else 0.0)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a))
+    xq = t(x)[:, None, :]
+    want, _ = Fn.multi_head_attention_forward(
+        xq, xq, xq, D, nh,
+        in_proj_weight=t(np.concatenate([W["l0.wq"], W["l0.wk"], W["l0.wv"]])),
+        in_proj_bias=t(np.concatenate([W["l0.bq"], W["l0.bk"], W["l0.bv"]])),
+        bias_k=None, bias_v=None, add_zero_attn=False, dropout_p=0.0,
+        out_proj_weight=t(W["l0.wo"]), out_proj_bias=t(W["l0.bo"]),
+        training=False, need_weights=False, attn_mask=t(mask))
+    assert np.allclose(got, want[:, 0, :].numpy(), atol=1e-11)
+
+
+def test_attention_is_bidirectional_and_bias_sensitive():
+    rng = np.random.default_rng(2)
+    L, K, D, nh = 4, 2, 16, 8
+    W = _rand_layer(rng, D, nh, L)
+    x = rng.standard_normal((L * K, D))
+    y = oracle.attention(x, W, "l0.", L, K, nh)
+    x2 = x.copy()
+    x2[-1] += 1.0                                  # last node of the last slot
+    y2 = oracle.attention(x2, W, "l0.", L, K, nh)
+    assert not np.allclose(y[0], y2[0])            # first node sees it: no causal mask
+    W2 = dict(W)
+    W2["l0.dist"] = W["l0.dist"].copy()
+    W2["l0.dist"][:, L - 1 + 2] += 1.0             # only pairs with s_j - s_i = +2
+    y3 = oracle.attention(x, W2, "l0.", L, K, nh)
+    assert not np.allclose(y[0], y3[0])            # slot 0 has a slot 2 to its right
+    assert np.allclose(y[-1], y3[-1])              # last slot has no slot at +2
+
+
+def _tiny():
+    wl = workloads.WORKLOADS["tiny_f32"]
+    W = workloads.head_weights(wl)
+    inp = workloads.sequence_inputs(wl, wl.seeds()[0])
+    emb = lambda ids: workloads.embed_rows(wl.V, wl.H, wl.dtype, ids)
+    return wl, W, inp, emb
+
+
+def test_hidden_term_is_shared_by_the_slot():
+    wl, W, inp, emb = _tiny()
+    L, K = 3, wl.K
+    ids = np.tile(np.arange(K), (L, 1))
+    logp = np.tile(-np.arange(K, dtype=float), (L, 1))
+    E = emb(ids.reshape(-1)).reshape(L, K, -1)
+    Wd = {k: v.astype(np.float64) for k, v in W.items()}
+    h = inp["hidden"][:L].astype(np.float64)
+    n1 = oracle.nodes(ids, logp, h, E, Wd).reshape(L, K, -1)
+    n2 = oracle.nodes(ids, logp, h + 1.0, E, Wd).reshape(L, K, -1)
+    diff = n2 - n1
+    assert np.allclose(diff, diff[:, :1, :])                     # same shift for all K
+    assert np.allclose(diff[0, 0], Wd["hid_w"].sum(axis=1))      # = W_h applied to ones
+
+
+def test_tiny_workload_end_to_end_properties():
+    wl, W, inp, emb = _tiny()
+    r = oracle.select_sequence(inp["logits"], inp["hidden"], inp["target"], emb, W, wl.K)
+    assert r["tokens"].shape == (wl.L,)
+    for s in range(wl.L):
+        assert r["tokens"][s] == r["ids"][s, r["choice"][s]]
+    assert np.allclose(np.linalg.norm(r["out"], axis=-1), 1)
+    assert np.allclose(np.linalg.norm(r["in"], axis=-1), 1)
+    assert abs(np.linalg.norm(r["anchor"]) - 1) < 1e-12
+    assert np.all(np.abs(r["P"]) <= 1) and np.all(np.abs(r["A"]) <= 1)
+    # brute force over all K^L = 4^8 paths: greedy = lexicographic maximiser, Viterbi = max
+    A, P = r["A"], r["P"]
+    best_vec, best_path = None, None
+    gmax = -np.inf
+    import itertools
+    for c in itertools.product(range(wl.K), repeat=wl.L):
+        vec = [A[c[0]]] + [P[s - 1, c[s - 1], c[s]] for s in range(1, wl.L)]
+        if best_vec is None or vec > best_vec:
+            best_vec, best_path = vec, c
+        gmax = max(gmax, oracle.SIGMA * sum(vec))
+    assert tuple(r["choice"]) == best_path
+    _, gv = oracle.viterbi(A, P)
+    assert abs(gv - gmax) < 1e-9
+
+
+def test_fusion_with_zero_target_reduces_to_first_block():
+    rng = np.random.default_rng(3)
+    D, d, L, K = 8, 6, 2, 2
+    W = {"fuse_w": rng.standard_normal((D, 3 * D)), "fuse_b": rng.standard_normal(D),
+         "out_w": rng.standard_normal((d, D)), "out_b": rng.standard_normal(d),
+         "in_w": rng.standard_normal((d, D)), "in_b": rng.standard_normal(d),
+         "anc_w": rng.standard_normal((d, D)), "anc_b": rng.standard_normal(d)}
+    x = rng.standard_normal((L * K, D))
+    out, inn, anc = oracle.fuse_and_heads(x, np.zeros(D), W, L, K)
+    u = Fn.silu(Fn.linear(torch.from_numpy(x), torch.from_numpy(W["fuse_w"][:, :D]),
+                          torch.from_numpy(W["fuse_b"]))).numpy()
+    o = u @ W["out_w"].T + W["out_b"]
+    assert np.allclose(out.reshape(L * K, d), o / np.linalg.norm(o, axis=1, keepdims=True))
+    a = W["anc_b"] / np.linalg.norm(W["anc_b"])
+    assert np.allclose(anc, a)
