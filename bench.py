@@ -1,0 +1,405 @@
+#!/usr/bin/env python
+"""Benchmark of the LiLiCorr per-block draft-selection path (one process per GPU).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Default workload: single requests (batch 1, L = 16 slots, V = 151936 bf16 logits,
+K = 8, d = 256, H = 4096), 1000 distinct blocks drawn from seeds 1..1000 and
+resident in HBM (4.9 GB of logits, larger than L2, so no L2 flush is needed).
+One step selects all 1000 blocks one after another, each a complete batch-1
+call of lilicorr_select_block replayed from its own CUDA graph. Batched
+workloads (``--workload serving_b32`` etc.) time one call over the batch per step.
+
+Prints one JSON line (rank 0): device-timed throughput (``value``), the same
+metric end to end through pinned host buffers (``e2e``), the top-K kernel's
+roofline measured live with CUDA events, SM clocks sampled during the timed
+region, and the CPU oracle timed on a bounded sample (``cpu_baseline``).
+``--impl reference`` times the CPU oracle itself as the reference arm.
+"""
+from __future__ import annotations
+
+import os
+
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")          # the oracle baseline runs on one core
+
+import argparse
+import json
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "draft blocks selected/sec at 1 GB300"
+UNIT = "blocks/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--workload", default="single_request", choices=workloads.WORKLOAD_ORDER)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--blocks", type=int, default=None, help="blocks per step (batch-1 workload)")
+    p.add_argument("--e2e-host-blocks", type=int, default=64)
+    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+# --------------------------------------------------------------------------- distributed
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(world, x: float) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of this GPU's SM clock and throttle reasons, every 200 ms."""
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self):
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.uuid = str(torch.cuda.get_device_properties(torch.cuda.current_device()).uuid)
+        except Exception:
+            self.uuid = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        self.out.flush()
+        rows = []
+        for line in open(self.out.name):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            if self.uuid and self.uuid not in f[0] and f[0] not in self.uuid:
+                continue
+            rows.append(f)
+        os.unlink(self.out.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def peaks():
+    try:
+        return json.load(open(PEAKS_FILE)), "measured"
+    except Exception:
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+# --------------------------------------------------------------------------- CPU oracle leg
+def oracle_blocks_per_s(wl, W, seeds, seconds: float):
+    """The oracle, as it stands, selecting whole blocks one after another on the host."""
+    import oracle
+    emb = lambda ids: workloads.embed_rows(wl.V, wl.H, wl.dtype, ids)
+    done, t0 = 0, time.perf_counter()
+    for seed in seeds:
+        inp = workloads.sequence_inputs(wl, seed)
+        oracle.select_sequence(inp["logits"], inp["hidden"], inp["target"], emb, W, wl.K)
+        done += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return done / dt, done, dt
+
+
+def run_reference(args, world, rank):
+    """Reference arm: the CPU oracle on the host cores, one block per step."""
+    if rank != 0:
+        return
+    wl = workloads.WORKLOADS[args.workload]
+    W = workloads.head_weights(wl)
+    seeds = wl.block_seeds() if wl.blocks > 1 else wl.seeds()
+    workloads.embed_table(wl.V, wl.H, wl.dtype)          # generate once, outside the timing
+    for i in range(args.warmup):
+        oracle_blocks_per_s(wl, W, [seeds[i % len(seeds)]], 0.0)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle_blocks_per_s(wl, W, [seeds[(args.warmup + i) % len(seeds)]], 0.0)
+    dt = time.perf_counter() - t0
+    v = args.steps / dt
+    sample = f"{args.steps} sequences of the {wl.name} workload, one per step"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": wl.name, "B": 1, "L": wl.L, "V": wl.V,
+                                        "K": wl.K, "d": wl.d, "H": wl.H},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# --------------------------------------------------------------------------- GPU arm
+def upload(a: np.ndarray, dtype: str, dev) -> torch.Tensor:
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    return (t.to(torch.bfloat16) if dtype == "bf16" else t).to(dev)
+
+
+def gen_blocks(wl, seeds, dev, chunk=50):
+    """Batch-1 blocks [n, 1, L, V] etc., generated in chunks straight into device memory."""
+    n = len(seeds)
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    logits = torch.empty((n, 1, wl.L, wl.V), dtype=tdt, device=dev)
+    hidden = torch.empty((n, 1, wl.L, wl.H), dtype=tdt, device=dev)
+    target = torch.empty((n, 1, wl.n_tgt, wl.H), dtype=tdt, device=dev)
+    for i in range(0, n, chunk):
+        inp = workloads.batch_inputs(wl, seeds[i:i + chunk])
+        m = inp["logits"].shape[0]
+        logits[i:i + m, 0] = upload(inp["logits"], wl.dtype, dev)
+        hidden[i:i + m, 0] = upload(inp["hidden"], wl.dtype, dev)
+        target[i:i + m, 0] = upload(inp["target"], wl.dtype, dev)
+    return logits, hidden, target
+
+
+def run_ours(args, world, rank, local):
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_20530_gb300 as ll
+
+    dev = torch.device("cuda", torch.cuda.current_device())
+    wl = workloads.WORKLOADS[args.workload]
+    es = 2 if wl.dtype == "bf16" else 4
+    W = workloads.head_weights(wl)
+    E = workloads.embed_table(wl.V, wl.H, wl.dtype)
+    head = ll.Head.from_workload(wl, W, E)
+    stream = torch.cuda.current_stream()
+
+    batch1 = wl.blocks > 1
+    if batch1:
+        nblk = args.blocks or wl.blocks
+        seeds = [s + rank * nblk for s in wl.block_seeds()[:nblk]] if nblk <= wl.blocks else \
+            [wl.seed_base + i + rank * nblk for i in range(nblk)]
+        logits, hidden, target = gen_blocks(wl, seeds, dev)
+        B = 1
+    else:
+        nblk = 1
+        inp = workloads.batch_inputs(wl, [s + rank * 100000 for s in wl.seeds()])
+        logits = upload(inp["logits"], wl.dtype, dev)[None]
+        hidden = upload(inp["hidden"], wl.dtype, dev)[None]
+        target = upload(inp["target"], wl.dtype, dev)[None]
+        B = wl.B
+        del inp
+    ws = head.workspace(B)
+    tokens = torch.empty((nblk, B, wl.L), dtype=torch.int32, device=dev)
+
+    # one call outside capture (configures kernels, counts launches per call)
+    n0 = ll.launch_count()
+    ll.select_block(head, logits[0], hidden[0], target[0], ws=ws, tokens=tokens[0])
+    launches_per_call = ll.launch_count() - n0
+    torch.cuda.synchronize()
+    if ws.status() != 0:
+        raise RuntimeError("device status set on the first call")
+
+    graphs = []
+    for i in range(nblk):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            ll.select_block(head, logits[i], hidden[i], target[i], ws=ws, tokens=tokens[i])
+        graphs.append(g)
+    torch.cuda.synchronize()
+
+    def step():
+        for g in graphs:
+            g.replay()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    clocks = ClockSampler()
+    clocks.start()
+    time.sleep(0.25)
+    barrier(world)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_stop = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        step()
+    t_stop.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    ms = t_start.elapsed_time(t_stop)
+    ms = max_over_ranks(world, ms)
+    units = nblk * B * args.steps * world
+    value = units / (ms / 1e3) if not batch1 else nblk * args.steps * world / (ms / 1e3)
+    ms_per_step = ms / args.steps
+    if ws.status() != 0:
+        raise RuntimeError("device status set during the timed region")
+
+    # ---- end to end: pinned host inputs -> device -> select -> tokens back to pinned host
+    nh = min(args.e2e_host_blocks, nblk)
+    h_logits = torch.empty((nh,) + tuple(logits.shape[1:]), dtype=logits.dtype).pin_memory()
+    h_hidden = torch.empty((nh,) + tuple(hidden.shape[1:]), dtype=hidden.dtype).pin_memory()
+    h_target = torch.empty((nh,) + tuple(target.shape[1:]), dtype=target.dtype).pin_memory()
+    h_logits.copy_(logits[:nh].cpu())
+    h_hidden.copy_(hidden[:nh].cpu())
+    h_target.copy_(target[:nh].cpu())
+    h_tokens = torch.empty((nh, B, wl.L), dtype=torch.int32).pin_memory()
+    d_logits = torch.empty_like(logits[0])
+    d_hidden = torch.empty_like(hidden[0])
+    d_target = torch.empty_like(target[0])
+    d_tokens = torch.empty((B, wl.L), dtype=torch.int32, device=dev)
+    e2e_graphs = []
+    for i in range(nh):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            d_logits.copy_(h_logits[i], non_blocking=True)
+            d_hidden.copy_(h_hidden[i], non_blocking=True)
+            d_target.copy_(h_target[i], non_blocking=True)
+            ll.select_block(head, d_logits, d_hidden, d_target, ws=ws, tokens=d_tokens)
+            h_tokens[i].copy_(d_tokens, non_blocking=True)
+        e2e_graphs.append(g)
+    e2e_calls = nblk
+
+    def e2e_step():
+        for i in range(e2e_calls):
+            e2e_graphs[i % nh].replay()
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = max_over_ranks(world, e0.elapsed_time(e1))
+    e2e_value = e2e_calls * B * args.steps * world / (e2e_ms / 1e3) if not batch1 else \
+        e2e_calls * args.steps * world / (e2e_ms / 1e3)
+    h2d = (d_logits.numel() * d_logits.element_size() + d_hidden.numel() * d_hidden.element_size()
+           + d_target.numel() * d_target.element_size()) * e2e_calls
+    d2h = d_tokens.numel() * 4 * e2e_calls
+
+    # ---- roofline of the top-K pass: each launch bracketed by CUDA events on its stream
+    rows = B * wl.L
+    tk_ws = ll.Workspace(ll.lib().lilicorr_topk_lse_workspace_bytes(rows, wl.V, wl.K))
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(nblk)]
+    flat = logits.view(nblk, rows, wl.V)
+    for i in range(min(nblk, 8)):
+        ll.topk_lse(flat[i], wl.K, ws=tk_ws)
+    torch.cuda.synchronize()
+    for i in range(nblk):
+        ev[i][0].record(stream)
+        ll.topk_lse(flat[i], wl.K, ws=tk_ws)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    tk_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    alg_bytes = rows * wl.V * es
+    pk, pk_kind = peaks()
+    hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
+    achieved = alg_bytes / (tk_ms / 1e3) / 1e9
+    roofline = {"kernel": "topk_lse_kernel", "bound": "hbm", "achieved": round(achieved, 1),
+                "peak": hbm, "peak_kind": pk_kind, "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                "traffic": None, "alg_bytes_per_launch": alg_bytes,
+                "us_per_launch": round(tk_ms * 1e3, 3)}
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "B": B, "L": wl.L, "V": wl.V, "K": wl.K, "d": wl.d,
+                   "D": wl.D, "H": wl.H, "blocks_per_step": nblk,
+                   "l2": ("inputs larger than L2: %d distinct resident blocks, %.2f GB of logits"
+                          % (nblk, logits.numel() * es / 1e9)) if batch1 else
+                         ("inputs larger than L2: %.2f GB of logits" % (logits.numel() * es / 1e9)),
+                   "graphs": "one CUDA graph per call, replayed", "parallelism": f"dp{world}"},
+        "us_per_block": ms_per_step * 1e3 / (nblk if batch1 else 1),
+        "clocks": clk,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h,
+                "note": f"pinned host blocks cycled ({nh} distinct), copies captured with the call"},
+        "gpu_launches": launches_per_call * (nblk if batch1 else 1) * args.steps,
+        "roofline": roofline,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        seeds_cpu = wl.block_seeds() if batch1 else wl.seeds()
+        v, n, dt = oracle_blocks_per_s(wl, W, seeds_cpu, args.cpu_seconds)
+        per = 1 if batch1 else 1
+        result["cpu_baseline"] = {
+            "value": v * per, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{n} sequences of the {wl.name} workload in {dt:.1f} s (fp64 NumPy, 1 thread)"}
+    if rank == 0:
+        print(json.dumps(result))
+    head.close()
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,330 @@
+"""Python binding of the LiLiCorr per-block draft-selection library (sm_103a).
+
+Argument marshalling only: every step of the path runs in the CUDA library
+``lib/liblilicorr.so`` through its C ABI (``include/lilicorr.h``). PyTorch
+supplies device memory and the current stream. There is no CPU fallback: if the
+library is missing, every call raises.
+
+Names follow the C ABI: ``topk_lse``, ``embed_in_out``, ``pair_scores``,
+``greedy_walk``, ``select_block``, plus ``Head`` (an uploaded scoring head) and
+``Workspace`` (caller-owned scratch).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Mapping, Optional, Sequence, Tuple
+
+import numpy as np
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "lib", "liblilicorr.so")
+
+F32, BF16 = 0, 1
+STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported or inconsistent shape",
+          3: "unsupported dtype", 4: "CUDA error", 5: "non-finite logit row",
+          6: "device wait timed out", 7: "workspace too small"}
+ERR_NONFINITE = 5
+MAX_K = 32
+
+
+class LilicorrError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {STATUS.get(status, status)} (status {status})")
+        self.status = status
+
+
+class HeadDesc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int) for n in
+                ("H", "D", "d", "n_heads", "ffn", "n_layers", "L", "K", "V", "n_tgt")] + \
+               [("dtype", ctypes.c_int)]
+
+
+_LIB: Optional[ctypes.CDLL] = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_S = ctypes.c_size_t
+
+_SIGS = {
+    "lilicorr_status_str": (ctypes.c_char_p, [_I]),
+    "lilicorr_version": (_I, []),
+    "lilicorr_head_param_count": (_S, [ctypes.POINTER(HeadDesc)]),
+    "lilicorr_head_create": (_I, [ctypes.POINTER(HeadDesc), _P, _P, ctypes.POINTER(_P)]),
+    "lilicorr_head_destroy": (_I, [_P]),
+    "lilicorr_workspace_init": (_I, [_P, _S, _P]),
+    "lilicorr_topk_lse_workspace_bytes": (_S, [_I, _I, _I]),
+    "lilicorr_topk_lse": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P, _S, _P]),
+    "lilicorr_workspace_bytes": (_S, [_P, _I]),
+    "lilicorr_embed_in_out": (_I, [_P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _S, _P]),
+    "lilicorr_pair_scores": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "lilicorr_greedy_walk": (_I, [_I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
+    "lilicorr_select_block": (_I, [_P, _I, _P, _P, _P, _P, _P, _S, _P]),
+    "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
+    "lilicorr_get_device_status": (_I, [_P, _P]),
+    "lilicorr_launch_count": (ctypes.c_uint64, []),
+}
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded CUDA library (raises if it has not been built)."""
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"CUDA library not built ({LIB_PATH}); run __graft_entry__.build()")
+        so = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            f = getattr(so, name)
+            f.restype = res
+            f.argtypes = args
+        _LIB = so
+    return _LIB
+
+
+def _check(status: int, where: str) -> None:
+    if status != 0:
+        raise LilicorrError(status, where)
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _dev(t: torch.Tensor, name: str) -> torch.Tensor:
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def launch_count() -> int:
+    """Kernel launches the library has enqueued in this process (graph replays excluded)."""
+    return int(lib().lilicorr_launch_count())
+
+
+# --------------------------------------------------------------------------- workspace
+class Workspace:
+    """Caller-owned device scratch, zero-filled once (the library's counters start at 0)."""
+
+    def __init__(self, nbytes: int, device=None):
+        self.nbytes = int(max(nbytes, 256))
+        self.buf = torch.zeros(self.nbytes, dtype=torch.uint8, device=device or "cuda")
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+    def status(self) -> int:
+        """Read and clear the device status word (synchronises the current stream)."""
+        return int(lib().lilicorr_get_device_status(self.ptr, _stream()))
+
+
+# --------------------------------------------------------------------------- head
+def blob_order(H: int, D: int, d: int, F: int, n_heads: int, L: int, K: int,
+               n_layers: int) -> Sequence[Tuple[str, Tuple[int, ...]]]:
+    """Tensor names and shapes in the weight-blob order of ``lilicorr.h``."""
+    s = [("emb_w", (D, H)), ("emb_b", (D,)), ("hid_w", (D, H)), ("hid_b", (D,)),
+         ("conf1_w", (D, 5)), ("conf1_b", (D,)), ("conf2_w", (D, D)), ("conf2_b", (D,)),
+         ("slot", (L, D)), ("rank", (K, D)), ("tgt_norm", (H,)), ("tgt_w", (D, H)),
+         ("tgt_b", (D,))]
+    for i in range(n_layers):
+        p = f"l{i}."
+        s += [(p + "an", (D,)), (p + "wq", (D, D)), (p + "bq", (D,)), (p + "wk", (D, D)),
+              (p + "bk", (D,)), (p + "wv", (D, D)), (p + "bv", (D,)), (p + "wo", (D, D)),
+              (p + "bo", (D,)), (p + "dist", (n_heads, 2 * L - 1)), (p + "same", (n_heads,)),
+              (p + "fn", (D,)), (p + "w1", (F, D)), (p + "b1", (F,)), (p + "w2", (D, F)),
+              (p + "b2", (D,))]
+    s += [("final_norm", (D,)), ("fuse_w", (D, 3 * D)), ("fuse_b", (D,)), ("out_w", (d, D)),
+          ("out_b", (d,)), ("in_w", (d, D)), ("in_b", (d,)), ("anc_w", (d, D)), ("anc_b", (d,))]
+    return s
+
+
+def _as_storage(a: np.ndarray, dtype: int) -> np.ndarray:
+    """float32 values -> contiguous storage of the head dtype (bf16 as uint16 bits,
+    round to nearest even; exact for values already representable in bf16)."""
+    if dtype == F32:
+        return np.ascontiguousarray(a, dtype=np.float32)
+    if a.dtype == np.uint16:
+        return np.ascontiguousarray(a)
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+class Head:
+    """A scoring head uploaded to the current CUDA device (lilicorr_head_create)."""
+
+    def __init__(self, *, H: int, D: int, d: int, n_heads: int, ffn: int, n_layers: int, L: int,
+                 K: int, V: int, n_tgt: int, dtype: str, weights: Mapping[str, np.ndarray],
+                 embed_table: np.ndarray):
+        self.dtype_code = BF16 if dtype == "bf16" else F32
+        self.desc = HeadDesc(H, D, d, n_heads, ffn, n_layers, L, K, V, n_tgt, self.dtype_code)
+        self.L, self.K, self.V, self.H, self.d, self.D, self.n_tgt = L, K, V, H, d, D, n_tgt
+        order = blob_order(H, D, d, ffn, n_heads, L, K, n_layers)
+        parts = []
+        for name, shape in order:
+            w = np.asarray(weights[name])
+            if tuple(w.shape) != tuple(shape):
+                raise ValueError(f"{name}: shape {w.shape}, expected {shape}")
+            parts.append(_as_storage(w, self.dtype_code).reshape(-1))
+        blob = np.concatenate(parts)
+        n = lib().lilicorr_head_param_count(ctypes.byref(self.desc))
+        if n == 0 or n != blob.size:
+            raise LilicorrError(2, f"head_param_count ({n} vs blob {blob.size})")
+        emb = _as_storage(embed_table, self.dtype_code)
+        if emb.shape != (V, H):
+            raise ValueError(f"embed_table shape {emb.shape}, expected {(V, H)}")
+        h = _P()
+        _check(lib().lilicorr_head_create(ctypes.byref(self.desc), blob.ctypes.data,
+                                          emb.ctypes.data, ctypes.byref(h)), "head_create")
+        self._h = h
+        self.torch_dtype = torch.bfloat16 if self.dtype_code == BF16 else torch.float32
+
+    @classmethod
+    def from_workload(cls, wl, weights, embed_table) -> "Head":
+        return cls(H=wl.H, D=wl.D, d=wl.d, n_heads=wl.n_heads, ffn=wl.F, n_layers=wl.n_layers,
+                   L=wl.L, K=wl.K, V=wl.V, n_tgt=wl.n_tgt, dtype=wl.dtype, weights=weights,
+                   embed_table=embed_table)
+
+    @property
+    def handle(self) -> int:
+        return self._h.value
+
+    def workspace_bytes(self, B: int) -> int:
+        return int(lib().lilicorr_workspace_bytes(self._h, B))
+
+    def workspace(self, B: int) -> Workspace:
+        return Workspace(self.workspace_bytes(B))
+
+    def close(self) -> None:
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(lib().lilicorr_head_destroy(self._h), "head_destroy")
+            self._h = _P()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+# --------------------------------------------------------------------------- calls
+def topk_lse(logits: torch.Tensor, K: int, ws: Optional[Workspace] = None):
+    """Top-K ids [rows, K] int32, log-probs [rows, K] fp32 and log-normaliser [rows] fp32
+    of logit rows [..., V] (fp32 or bf16)."""
+    _dev(logits, "logits")
+    V = logits.shape[-1]
+    rows = logits.numel() // V if V else 0
+    need = int(lib().lilicorr_topk_lse_workspace_bytes(rows, V, K))
+    if ws is None:
+        ws = Workspace(need, logits.device)
+    lead = tuple(logits.shape[:-1])
+    ids = torch.empty(lead + (K,), dtype=torch.int32, device=logits.device)
+    logp = torch.empty(lead + (K,), dtype=torch.float32, device=logits.device)
+    lse = torch.empty(lead, dtype=torch.float32, device=logits.device)
+    _check(lib().lilicorr_topk_lse(logits.data_ptr(), _dtype_code(logits), rows, V, K,
+                                   ids.data_ptr(), logp.data_ptr(), lse.data_ptr(), ws.ptr,
+                                   ws.nbytes, _stream()), "topk_lse")
+    return ids, logp, lse
+
+
+def embed_in_out(head: Head, ids: torch.Tensor, logp: torch.Tensor, hidden: torch.Tensor,
+                 target: torch.Tensor, ws: Optional[Workspace] = None):
+    """Unit out/in vectors [B, L, K, d] and anchor out vectors [B, d] (fp32)."""
+    B = ids.shape[0]
+    for t, n in ((ids, "ids"), (logp, "logp"), (hidden, "hidden"), (target, "target")):
+        _dev(t, n)
+    if hidden.dtype != head.torch_dtype or target.dtype != head.torch_dtype:
+        raise ValueError("hidden/target dtype must match the head dtype")
+    ws = ws or head.workspace(B)
+    dev = ids.device
+    out = torch.empty((B, head.L, head.K, head.d), dtype=torch.float32, device=dev)
+    inn = torch.empty_like(out)
+    anc = torch.empty((B, head.d), dtype=torch.float32, device=dev)
+    _check(lib().lilicorr_embed_in_out(head._h, B, ids.data_ptr(), logp.data_ptr(),
+                                       hidden.data_ptr(), target.data_ptr(), out.data_ptr(),
+                                       inn.data_ptr(), anc.data_ptr(), ws.ptr, ws.nbytes,
+                                       _stream()), "embed_in_out")
+    return out, inn, anc
+
+
+def pair_scores(out_vec: torch.Tensor, in_vec: torch.Tensor, anchor_out: torch.Tensor):
+    """Anchor row [B, K] and pair matrices [B, L-1, K, K] of cosines (no sigma)."""
+    B, L, K, d = out_vec.shape
+    for t, n in ((out_vec, "out_vec"), (in_vec, "in_vec"), (anchor_out, "anchor_out")):
+        _dev(t, n)
+    A = torch.empty((B, K), dtype=torch.float32, device=out_vec.device)
+    P = torch.empty((B, max(L - 1, 0), K, K), dtype=torch.float32, device=out_vec.device)
+    _check(lib().lilicorr_pair_scores(B, L, K, d, out_vec.data_ptr(), in_vec.data_ptr(),
+                                      anchor_out.data_ptr(), A.data_ptr(),
+                                      P.data_ptr() if P.numel() else None, _stream()),
+           "pair_scores")
+    return A, P
+
+
+def greedy_walk(A: torch.Tensor, P: torch.Tensor, ids: torch.Tensor):
+    """Greedy walk: choice [B, L], tokens [B, L] (int32) and margins [B, L] (fp32)."""
+    B, K = A.shape
+    L = P.shape[1] + 1
+    for t, n in ((A, "anchor_scores"), (P, "pair_scores"), (ids, "ids")):
+        _dev(t, n)
+    choice = torch.empty((B, L), dtype=torch.int32, device=A.device)
+    tokens = torch.empty_like(choice)
+    margin = torch.empty((B, L), dtype=torch.float32, device=A.device)
+    _check(lib().lilicorr_greedy_walk(B, L, K, A.data_ptr(), P.data_ptr() if P.numel() else None,
+                                      ids.data_ptr(), choice.data_ptr(), tokens.data_ptr(),
+                                      margin.data_ptr(), _stream()), "greedy_walk")
+    return choice, tokens, margin
+
+
+def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target: torch.Tensor,
+                 ws: Optional[Workspace] = None, tokens: Optional[torch.Tensor] = None):
+    """The fused path: logits [B, L, V], hidden [B, L, H], target [B, n_tgt, H] (head dtype,
+    on the device) -> chosen token ids [B, L] int32."""
+    B = logits.shape[0]
+    for t, n in ((logits, "logits"), (hidden, "hidden"), (target, "target")):
+        _dev(t, n)
+        if t.dtype != head.torch_dtype:
+            raise ValueError(f"{n} dtype must match the head dtype")
+    ws = ws or head.workspace(B)
+    if tokens is None:
+        tokens = torch.empty((B, head.L), dtype=torch.int32, device=logits.device)
+    _check(lib().lilicorr_select_block(head._h, B, logits.data_ptr(), hidden.data_ptr(),
+                                       target.data_ptr(), tokens.data_ptr(), ws.ptr, ws.nbytes,
+                                       _stream()), "select_block")
+    return tokens
+
+
+def select_block_intermediates(head: Head, B: int, ws: Workspace) -> Dict[str, torch.Tensor]:
+    """Views of the last select_block call's intermediates inside ``ws``."""
+    ptrs = [_P() for _ in range(6)]
+    _check(lib().lilicorr_select_block_intermediates(head._h, B, ws.ptr, ws.nbytes,
+                                                     *[ctypes.byref(p) for p in ptrs]),
+           "select_block_intermediates")
+    base = ws.buf.data_ptr()
+    L, K = head.L, head.K
+
+    def view(p, shape, dtype):
+        n = int(np.prod(shape))
+        off = p.value - base
+        es = 4
+        return ws.buf[off: off + n * es].view(dtype).reshape(shape)
+
+    return {"ids": view(ptrs[0], (B, L, K), torch.int32),
+            "logp": view(ptrs[1], (B, L, K), torch.float32),
+            "lse": view(ptrs[2], (B, L), torch.float32),
+            "A": view(ptrs[3], (B, K), torch.float32),
+            "P": view(ptrs[4], (B, max(L - 1, 0), K, K), torch.float32),
+            "choice": view(ptrs[5], (B, L), torch.int32)}

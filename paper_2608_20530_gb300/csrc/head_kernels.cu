@@ -1,0 +1,366 @@
+// Step (2): the scoring network's fp32 CUDA-core kernels (Sec. 3.2; App. A "Architecture").
+//
+// Node construction, RMSNorm, target state, bidirectional attention with the two
+// learned bias tables, the fusion input and row normalisation, plus a tiled
+// fp32 linear layer with fused bias / per-sequence bias / SiLU / residual
+// epilogue. The fp32 head runs every matrix product here; the bf16 head runs its
+// large products on the tensor cores (gemm_tc.cu) and the rest here.
+#include "internal.cuh"
+
+namespace lilicorr {
+
+namespace {
+
+constexpr float RMS_EPS = 1e-6f;
+constexpr float UNIT_EPS = 1e-12f;
+
+// ----------------------------------------------------------------------------- linear
+constexpr int GB_M = 64, GB_N = 64, GB_K = 16, G_THREADS = 256;
+
+template <typename TA, typename TW, typename TC>
+__global__ void __launch_bounds__(G_THREADS) gemm_simt_kernel(GemmArgs g) {
+  __shared__ float As[GB_K][GB_M + 4];
+  __shared__ __align__(16) float Ws[GB_K][GB_N + 4];
+  const TA* A = static_cast<const TA*>(g.A);
+  const TW* W = static_cast<const TW*>(g.W);
+  const int tid = threadIdx.x;
+  const int m0 = blockIdx.y * GB_M, n0 = blockIdx.x * GB_N;
+  const int tx = tid & 15, ty = tid >> 4;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+  for (int k0 = 0; k0 < g.Kd; k0 += GB_K) {
+#pragma unroll
+    for (int i = tid; i < GB_M * GB_K; i += G_THREADS) {
+      const int r = i / GB_K, c = i % GB_K;
+      const int gm = m0 + r, gk = k0 + c;
+      As[c][r] = (gm < g.M && gk < g.Kd) ? ld_elem(A, (size_t)gm * g.lda + gk) : 0.f;
+      const int gn = n0 + r;
+      Ws[c][r] = (gn < g.N && gk < g.Kd) ? ld_elem(W, (size_t)gn * g.ldw + gk) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GB_K; ++kk) {
+      float a[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+      const float4 b = *reinterpret_cast<const float4*>(&Ws[kk][tx * 4]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        acc[i][0] = fmaf(a[i], b.x, acc[i][0]);
+        acc[i][1] = fmaf(a[i], b.y, acc[i][1]);
+        acc[i][2] = fmaf(a[i], b.z, acc[i][2]);
+        acc[i][3] = fmaf(a[i], b.w, acc[i][3]);
+      }
+    }
+    __syncthreads();
+  }
+  TC* C = static_cast<TC*>(g.C);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int m = m0 + ty * 4 + i;
+    if (m >= g.M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = n0 + tx * 4 + j;
+      if (n >= g.N) continue;
+      float v = acc[i][j];
+      if (g.bias) v += g.bias[n];
+      if (g.bias_rows) v += g.bias_rows[(size_t)(m / g.rows_per_bias) * g.N + n];
+      if (g.act == ACT_SILU) v = silu_f(v);
+      if (g.residual) v += g.residual[(size_t)m * g.ldr + n];
+      st_elem(C, (size_t)m * g.ldc + n, v);
+    }
+  }
+}
+
+template <typename TA, typename TW>
+lilicorr_status_t gemm_dispatch_c(const GemmArgs& g, dim3 grid, cudaStream_t st) {
+  if (g.c_dt == LILICORR_F32) gemm_simt_kernel<TA, TW, float><<<grid, G_THREADS, 0, st>>>(g);
+  else gemm_simt_kernel<TA, TW, __nv_bfloat16><<<grid, G_THREADS, 0, st>>>(g);
+  return last_launch();
+}
+template <typename TA>
+lilicorr_status_t gemm_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st) {
+  if (g.w_dt == LILICORR_F32) return gemm_dispatch_c<TA, float>(g, grid, st);
+  return gemm_dispatch_c<TA, __nv_bfloat16>(g, grid, st);
+}
+
+// ----------------------------------------------------------------------------- target state
+// tn[b] = RMSNorm_H(mean over the n_tgt captured layers of T[b]) * gain (App. A).
+template <typename T>
+__global__ void target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H,
+                                   const float* __restrict__ gain, float* __restrict__ tn) {
+  __shared__ float red[32];
+  const int b = blockIdx.x;
+  const T* tb = Tin + (size_t)b * n_tgt * H;
+  float ss = 0.f;
+  for (int h = threadIdx.x; h < H; h += blockDim.x) {
+    float acc = 0.f;
+    for (int l = 0; l < n_tgt; ++l) acc += ld_elem(tb, (size_t)l * H + h);
+    acc /= (float)n_tgt;
+    tn[(size_t)b * H + h] = acc;
+    ss += acc * acc;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float r = rsqrtf(red[0] / (float)H + RMS_EPS);
+  for (int h = threadIdx.x; h < H; h += blockDim.x)
+    tn[(size_t)b * H + h] = tn[(size_t)b * H + h] * r * gain[h];
+}
+
+// ----------------------------------------------------------------------------- nodes
+// One CTA per slot row r = b*L + s. For candidate k (Sec. 3.2; App. A):
+//   c1 = SiLU(W_c1 f_k + b_c1)   (first layer of the confidence network; the second
+//                                 layer is a linear launch that adds into x)
+//   x  = fold[id_k] + hproj[r] + slot[s] + rank[k]
+// with f_k = [logp_k, exp(logp_k), logp_0 - logp_k, k / (K-1), 1{k = 0}].
+__global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __restrict__ ids,
+                                  const float* __restrict__ logp, const float* __restrict__ fold,
+                                  const float* __restrict__ hproj, const float* __restrict__ slot,
+                                  const float* __restrict__ rank, const float* __restrict__ w1,
+                                  const float* __restrict__ b1, float* __restrict__ c1,
+                                  float* __restrict__ x, uint32_t* status) {
+  __shared__ float f[LILICORR_MAX_K][LILICORR_N_CONF];
+  __shared__ int sid[LILICORR_MAX_K];
+  const int r = blockIdx.x;
+  const int s = r % L;
+  if (threadIdx.x < K) {
+    const int k = threadIdx.x;
+    const float lp = logp[(size_t)r * K + k];
+    const float lp0 = logp[(size_t)r * K];
+    f[k][0] = lp;
+    f[k][1] = expf(lp);
+    f[k][2] = lp0 - lp;
+    f[k][3] = K > 1 ? (float)k / (float)(K - 1) : 0.f;
+    f[k][4] = k == 0 ? 1.f : 0.f;
+    int id = ids[(size_t)r * K + k];
+    if (id < 0 || id >= V) {          // an id outside the vocabulary: flag it, read row 0
+      set_status(status, LILICORR_ERR_ARG);
+      id = 0;
+    }
+    sid[k] = id;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < K * D; i += blockDim.x) {
+    const int k = i / D, n = i % D;
+    float z = b1[n];
+#pragma unroll
+    for (int j = 0; j < LILICORR_N_CONF; ++j) z = fmaf(w1[n * LILICORR_N_CONF + j], f[k][j], z);
+    const size_t node = (size_t)r * K + k;
+    c1[node * D + n] = silu_f(z);
+    x[node * D + n] = fold[(size_t)sid[k] * D + n] + hproj[(size_t)r * D + n] +
+                      slot[(size_t)s * D + n] + rank[(size_t)k * D + n];
+  }
+}
+
+// ----------------------------------------------------------------------------- RMSNorm
+template <typename TY>
+__global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int D,
+                               const float* __restrict__ gain, TY* __restrict__ y) {
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const float* xr = x + (size_t)row * D;
+  float ss = 0.f;
+  for (int i = lane; i < D; i += 32) ss += xr[i] * xr[i];
+  ss = warp_sum(ss);
+  const float r = rsqrtf(ss / (float)D + RMS_EPS);
+  for (int i = lane; i < D; i += 32) st_elem(y, (size_t)row * D + i, xr[i] * r * gain[i]);
+}
+
+// fin[row] = [xf, xf * t_b] with xf = RMSNorm(x[row]) * gain: the x and x*t blocks of
+// the fusion layer's input [x; t; x*t] (App. A); the t block is a per-sequence bias.
+template <typename TY>
+__global__ void fusion_input_kernel(const float* __restrict__ x, int M, int LK, int D,
+                                    const float* __restrict__ gain, const float* __restrict__ t,
+                                    TY* __restrict__ fin) {
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= M) return;
+  const float* xr = x + (size_t)row * D;
+  const float* tb = t + (size_t)(row / LK) * D;
+  float ss = 0.f;
+  for (int i = lane; i < D; i += 32) ss += xr[i] * xr[i];
+  ss = warp_sum(ss);
+  const float r = rsqrtf(ss / (float)D + RMS_EPS);
+  for (int i = lane; i < D; i += 32) {
+    const float xf = xr[i] * r * gain[i];
+    st_elem(fin, (size_t)row * 2 * D + i, xf);
+    st_elem(fin, (size_t)row * 2 * D + D + i, xf * tb[i]);
+  }
+}
+
+// dst[row] = src[row] / max(||src[row]||, 1e-12), rows of n floats.
+__global__ void unit_rows_kernel(const float* __restrict__ src, int rows, int n, int ld_src,
+                                 float* __restrict__ dst, int ld_dst) {
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const float* s = src + (size_t)row * ld_src;
+  float ss = 0.f;
+  for (int i = lane; i < n; i += 32) ss += s[i] * s[i];
+  ss = warp_sum(ss);
+  const float inv = 1.0f / fmaxf(sqrtf(ss), UNIT_EPS);
+  for (int i = lane; i < n; i += 32) dst[(size_t)row * ld_dst + i] = s[i] * inv;
+}
+
+// ----------------------------------------------------------------------------- attention
+// One CTA per (sequence, head): all L*K nodes attend to all L*K nodes (no mask),
+// logits q.k / sqrt(hd) + dist[h, s_j - s_i + L - 1] + same[h] * 1{s_i == s_j}.
+// qkv rows hold [q | k | v], each D wide, head h in columns [h*hd, (h+1)*hd).
+__global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, int D, int n_heads,
+                                 const float* __restrict__ dist, const float* __restrict__ same,
+                                 float* __restrict__ out) {
+  extern __shared__ float sm[];
+  const int LK = L * K, hd = D / n_heads;
+  const int b = blockIdx.x / n_heads, h = blockIdx.x % n_heads;
+  const int nw = blockDim.x >> 5, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float* Ks = sm;                       // [LK][hd + 1]
+  float* Vs = Ks + (size_t)LK * (hd + 1);   // [LK][hd]
+  float* Qw = Vs + (size_t)LK * hd;     // [nw][hd]
+  float* Pw = Qw + (size_t)nw * hd;     // [nw][LK]
+  const size_t ld = 3 * (size_t)D;
+  const float* base = qkv + (size_t)b * LK * ld;
+  for (int i = threadIdx.x; i < LK * hd; i += blockDim.x) {
+    const int j = i / hd, c = i % hd;
+    Ks[j * (hd + 1) + c] = base[j * ld + D + h * hd + c];
+    Vs[j * hd + c] = base[j * ld + 2 * D + h * hd + c];
+  }
+  __syncthreads();
+  const float scale = rsqrtf((float)hd);
+  const float* dh = dist + (size_t)h * (2 * L - 1);
+  const float sh = same[h];
+  float* q = Qw + warp * hd;
+  float* p = Pw + (size_t)warp * LK;
+  for (int i = warp; i < LK; i += nw) {
+    for (int c = lane; c < hd; c += 32) q[c] = base[(size_t)i * ld + h * hd + c];
+    __syncwarp();
+    const int si = i / K;
+    float mx = -INFINITY;
+    for (int j = lane; j < LK; j += 32) {
+      const float* kj = Ks + j * (hd + 1);
+      float acc = 0.f;
+      for (int c = 0; c < hd; ++c) acc = fmaf(q[c], kj[c], acc);
+      const int sj = j / K;
+      const float v = acc * scale + dh[sj - si + L - 1] + (si == sj ? sh : 0.f);
+      p[j] = v;
+      mx = fmaxf(mx, v);
+    }
+    mx = warp_max(mx);
+    float sum = 0.f;
+    for (int j = lane; j < LK; j += 32) {
+      const float e = __expf(p[j] - mx);
+      p[j] = e;
+      sum += e;
+    }
+    sum = warp_sum(sum);
+    __syncwarp();
+    const float inv = 1.0f / sum;
+    for (int c = lane; c < hd; c += 32) {
+      float acc = 0.f;
+      for (int j = 0; j < LK; ++j) acc = fmaf(p[j], Vs[j * hd + c], acc);
+      out[((size_t)b * LK + i) * D + h * hd + c] = acc * inv;
+    }
+    __syncwarp();
+  }
+}
+
+}  // namespace
+
+size_t attention_smem_bytes(int LK, int hd, int warps) {
+  return sizeof(float) * ((size_t)LK * (hd + 1) + (size_t)LK * hd + (size_t)warps * hd +
+                          (size_t)warps * LK);
+}
+
+lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st) {
+  if (g.M == 0 || g.N == 0) return LILICORR_OK;
+  dim3 grid(ceil_div(g.N, GB_N), ceil_div(g.M, GB_M));
+  if (g.a_dt == LILICORR_F32) return gemm_dispatch_w<float>(g, grid, st);
+  return gemm_dispatch_w<__nv_bfloat16>(g, grid, st);
+}
+
+lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
+                                     const float* gain, float* tn, cudaStream_t st) {
+  if (B == 0) return LILICORR_OK;
+  if (dt == LILICORR_F32)
+    target_norm_kernel<float><<<B, 256, 0, st>>>(static_cast<const float*>(T), n_tgt, H, gain, tn);
+  else
+    target_norm_kernel<__nv_bfloat16><<<B, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(T),
+                                                         n_tgt, H, gain, tn);
+  return last_launch();
+}
+
+lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
+                                    const float* logp, const float* hproj, float* c1, float* x,
+                                    uint32_t* status, cudaStream_t st) {
+  const lilicorr_head_desc& d = h->desc;
+  if (B == 0) return LILICORR_OK;
+  node_build_kernel<<<B * d.L, 256, 0, st>>>(d.L, d.K, d.D, d.V, ids, logp,
+                                             static_cast<const float*>(h->fold), hproj, h->slot,
+                                             h->rank, h->conf1_w, h->conf1_b, c1, x, status);
+  return last_launch();
+}
+
+lilicorr_status_t launch_rmsnorm(const float* x, int M, int D, const float* gain, void* y,
+                                 lilicorr_dtype_t y_dt, cudaStream_t st) {
+  if (M == 0) return LILICORR_OK;
+  const int grid = ceil_div(M, 8);
+  if (y_dt == LILICORR_F32)
+    rmsnorm_kernel<float><<<grid, 256, 0, st>>>(x, M, D, gain, static_cast<float*>(y));
+  else
+    rmsnorm_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, M, D, gain,
+                                                        static_cast<__nv_bfloat16*>(y));
+  return last_launch();
+}
+
+lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, const float* gain,
+                                      const float* t, void* fin, lilicorr_dtype_t dt,
+                                      cudaStream_t st) {
+  const int M = B * LK;
+  if (M == 0) return LILICORR_OK;
+  const int grid = ceil_div(M, 8);
+  if (dt == LILICORR_F32)
+    fusion_input_kernel<float><<<grid, 256, 0, st>>>(x, M, LK, D, gain, t, static_cast<float*>(fin));
+  else
+    fusion_input_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, M, LK, D, gain, t,
+                                                             static_cast<__nv_bfloat16*>(fin));
+  return last_launch();
+}
+
+lilicorr_status_t launch_unit_rows(const float* src, int rows, int n, int ld_src, float* dst,
+                                   int ld_dst, cudaStream_t st) {
+  if (rows == 0) return LILICORR_OK;
+  unit_rows_kernel<<<ceil_div(rows, 8), 256, 0, st>>>(src, rows, n, ld_src, dst, ld_dst);
+  return last_launch();
+}
+
+lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D, int n_heads,
+                                   const float* dist, const float* same, float* out,
+                                   cudaStream_t st) {
+  if (B == 0) return LILICORR_OK;
+  const int warps = 8;
+  const size_t smem = attention_smem_bytes(L * K, D / n_heads, warps);
+  static bool configured[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 64 && !configured[dev]) {
+    LL_CUDA_TRY(cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     227 * 1024));
+    configured[dev] = true;
+  }
+  attention_kernel<<<B * n_heads, warps * 32, smem, st>>>(qkv, L, K, D, n_heads, dist, same, out);
+  return last_launch();
+}
+
+}  // namespace lilicorr

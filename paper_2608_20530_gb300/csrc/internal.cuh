@@ -1,0 +1,183 @@
+// Internal declarations of the LiLiCorr selection library (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "lilicorr.h"
+
+namespace lilicorr {
+
+// ----------------------------------------------------------------------------- host helpers
+#define LL_CUDA_TRY(expr)                                   \
+  do {                                                      \
+    cudaError_t _e = (expr);                                \
+    if (_e != cudaSuccess) return LILICORR_ERR_CUDA;        \
+  } while (0)
+
+#define LL_TRY(expr)                                        \
+  do {                                                      \
+    lilicorr_status_t _s = (expr);                          \
+    if (_s != LILICORR_OK) return _s;                       \
+  } while (0)
+
+void count_launch();   // host-side launch counter (lilicorr_launch_count)
+
+// Call right after each kernel launch: counts it and reports a launch error.
+inline lilicorr_status_t last_launch() {
+  count_launch();
+  return cudaGetLastError() == cudaSuccess ? LILICORR_OK : LILICORR_ERR_CUDA;
+}
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline int ceil_div(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+int num_sms();   // of the current device, cached per device
+
+// ----------------------------------------------------------------------------- device helpers
+__device__ __forceinline__ float bf16_to_f32(uint16_t b) {
+  return __uint_as_float(((uint32_t)b) << 16);
+}
+__device__ __forceinline__ float ld_elem(const float* p, size_t i) { return p[i]; }
+__device__ __forceinline__ float ld_elem(const __nv_bfloat16* p, size_t i) {
+  return __bfloat162float(p[i]);
+}
+__device__ __forceinline__ void st_elem(float* p, size_t i, float v) { p[i] = v; }
+__device__ __forceinline__ void st_elem(__nv_bfloat16* p, size_t i, float v) {
+  p[i] = __float2bfloat16_rn(v);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float silu_f(float z) { return z / (1.0f + __expf(-z)); }
+
+// Record the first device-detected error in the workspace status word.
+__device__ __forceinline__ void set_status(uint32_t* status, uint32_t code) {
+  if (status) atomicCAS(status, 0u, code);
+}
+
+// ----------------------------------------------------------------------------- head
+struct HeadW {          // device pointers of one Transformer layer
+  const void* wqkv;     // [3D, D] (q rows, then k, then v)
+  const float* bqkv;    // [3D]
+  const void* wo;       // [D, D]
+  const float* bo;
+  const void* w1;       // [F, D]
+  const float* b1;
+  const void* w2;       // [D, F]
+  const float* b2;
+  const float* an;      // [D] attention RMSNorm gain
+  const float* fn;      // [D] FFN RMSNorm gain
+  const float* dist;    // [n_heads, 2L-1]
+  const float* same;    // [n_heads]
+};
+
+}  // namespace lilicorr
+
+struct lilicorr_head {
+  lilicorr_head_desc desc;
+  int device;
+  void* pool;                 // one device allocation holding everything below
+  size_t pool_bytes;
+  // matrices in head dtype; vectors and tables in fp32
+  const void* fold;           // [V, D] folded embedding table E W_e^T + b_e (head dtype)
+  const void* hid_w;  const float* hid_b;
+  const float* conf1_w; const float* conf1_b;     // [D, 5], [D] (fp32)
+  const void* conf2_w; const float* conf2_b;
+  const float* slot; const float* rank;           // [L, D], [K, D]
+  const float* tgt_norm;                          // [H]
+  const void* tgt_w; const float* tgt_b;
+  lilicorr::HeadW layer[8];
+  const float* final_norm;
+  const void* fuse_x;         // [D, 2D]: columns of W_f acting on x and on x*t
+  const void* fuse_t;         // [D, D]:  columns of W_f acting on t
+  const float* fuse_b;
+  const void* woi;            // [2d, D]: out_w rows then in_w rows
+  const float* boi;           // [2d]
+  const void* anc_w; const float* anc_b;
+};
+
+namespace lilicorr {
+
+// ----------------------------------------------------------------------------- workspace
+struct TopkPlan {
+  int splits;          // CTAs per row
+  int chunk_vecs;      // 16-byte vectors per split
+  size_t rec_bytes;    // bytes of one partial record
+};
+TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt);
+
+struct WsLayout {
+  size_t status, counters, partials;
+  size_t ids, logp, lse;
+  size_t hproj, tn, t, anc, cb;
+  size_t x, c1, xn, qkv, att, hf, u, oi;
+  size_t A, P, choice;
+  size_t total;
+};
+WsLayout ws_layout(const lilicorr_head_desc& d, int B);
+size_t topk_ws_bytes(int rows, int V, int K, lilicorr_dtype_t dt);
+
+// ----------------------------------------------------------------------------- launchers
+// (1) top-K + log-normaliser. ws: status word at offset 0, then counters, partials.
+lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int rows, int V, int K,
+                                  int32_t* ids, float* logp, float* lse, uint32_t* status,
+                                  uint32_t* counters, void* partials, cudaStream_t st);
+
+// Generic linear layer C = act(A W^T + bias [+ bias_rows[m / rows_per_bias]]) [+ residual].
+enum { ACT_NONE = 0, ACT_SILU = 1 };
+struct GemmArgs {
+  const void* A; lilicorr_dtype_t a_dt; int lda;
+  const void* W; lilicorr_dtype_t w_dt; int ldw;
+  void* C; lilicorr_dtype_t c_dt; int ldc;
+  const float* bias;
+  const float* bias_rows; int rows_per_bias;
+  const float* residual; int ldr;
+  int act;
+  int M, N, Kd;
+};
+lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
+
+// scoring-network helpers (head_kernels.cu)
+lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
+                                     const float* gain, float* tn, cudaStream_t st);
+lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
+                                    const float* logp, const float* hproj, float* c1, float* x,
+                                    uint32_t* status, cudaStream_t st);
+lilicorr_status_t launch_rmsnorm(const float* x, int M, int D, const float* gain, void* y,
+                                 lilicorr_dtype_t y_dt, cudaStream_t st);
+lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D, int n_heads,
+                                   const float* dist, const float* same, float* out,
+                                   cudaStream_t st);
+lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, const float* gain,
+                                      const float* t, void* fin, lilicorr_dtype_t dt,
+                                      cudaStream_t st);
+lilicorr_status_t launch_unit_rows(const float* src, int rows, int n, int ld_src, float* dst,
+                                   int ld_dst, cudaStream_t st);
+
+// (3)+(4) pair scores and greedy walk (pair_walk.cu)
+struct PairWalkArgs {
+  int B, L, K, d;
+  const float* out; const float* in; int ld_vec;  // node rows, row stride in floats
+  const float* anchor;                            // [B, d]
+  float* A; float* P;                             // outputs (pair mode) or inputs (walk-only)
+  const int32_t* ids;                             // [B, L, K] (walk)
+  int32_t* choice; int32_t* tokens; float* margin;
+  bool do_pairs, do_walk;
+  bool scores_in_smem;                            // set by the launcher
+};
+lilicorr_status_t launch_pair_walk(const PairWalkArgs& a, cudaStream_t st);
+
+}  // namespace lilicorr

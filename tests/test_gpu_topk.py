@@ -1,0 +1,128 @@
+"""GPU parity of step (1), top-K + log-normaliser (Sec. 3.2; App. A "Serving"), against
+the oracle: ids bit-exact, log-probs and log-normaliser within 1e-3."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from _helpers import TOL_LOGP, to_dev, workload_data
+
+pytestmark = pytest.mark.gpu
+
+
+def _ll():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_20530_gb300 as ll
+    return ll
+
+
+def _close(a, b, tol):
+    """Equal infinities at the same places, finite entries within tol."""
+    a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+    inf = np.isinf(b)
+    return np.array_equal(np.isinf(a), inf) and np.all(a[inf] == b[inf]) and \
+        (not np.any(~inf) or np.abs(a[~inf] - b[~inf]).max() <= tol)
+
+
+def _check_rows(x: np.ndarray, K: int, ids, logp, lse, rows):
+    for r in rows:
+        oid, olp, olse = oracle.topk_lse(x[r], K)
+        assert np.array_equal(ids[r], oid), f"row {r}: {ids[r]} vs {oid}"
+        assert abs(lse[r] - olse) <= TOL_LOGP, (r, lse[r], olse)
+        assert _close(logp[r], olp, TOL_LOGP), (r, logp[r], olp)
+
+
+def _run(x: np.ndarray, K: int, dtype: str):
+    ll = _ll()
+    t = to_dev(x, dtype)
+    ws = ll.Workspace(ll.lib().lilicorr_topk_lse_workspace_bytes(x.shape[0], x.shape[1], K))
+    ids, logp, lse = ll.topk_lse(t, K, ws=ws)
+    torch.cuda.synchronize()
+    return ids.cpu().numpy(), logp.cpu().numpy(), lse.cpu().numpy(), ws.status()
+
+
+def test_tiny_workload_all_rows():
+    wl, _, inp = workload_data("tiny_f32")
+    x = inp["logits"].reshape(-1, wl.V)
+    ids, logp, lse, st = _run(x, wl.K, wl.dtype)
+    assert st == 0
+    _check_rows(x, wl.K, ids, logp, lse, range(x.shape[0]))
+
+
+@pytest.mark.parametrize("name,tier", [("single_request", 0), ("serving_b32", 0),
+                                       ("entropy_tiers_b64", 0), ("entropy_tiers_b64", 1),
+                                       ("entropy_tiers_b64", 2), ("ties_b256", 0)])
+def test_full_size_workloads_sampled_rows(name, tier):
+    wl, _, inp = workload_data(name, tier)
+    x = inp["logits"].reshape(-1, wl.V)
+    ids, logp, lse, st = _run(x, wl.K, wl.dtype)
+    assert st == 0
+    rng = np.random.default_rng(17)
+    rows = sorted(set([0, x.shape[0] - 1] + list(rng.integers(0, x.shape[0], 6))))
+    _check_rows(x, wl.K, ids, logp, lse, rows)
+    # every row: ids sorted by (logit desc, id asc) and logp consistent with lse
+    xv = np.take_along_axis(x, ids.astype(np.int64), axis=1)
+    assert np.all(np.diff(xv, axis=1) <= 0)
+    assert np.allclose(logp, xv - lse[:, None], atol=1e-5)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("rows,V,K", [(1, 1, 1), (3, 7, 7), (37, 1001, 5), (5, 9, 8),
+                                      (2, 151936, 32), (1, 151936, 1), (300, 4096, 16),
+                                      (64, 33, 32)])
+def test_shapes_and_ragged_rows(dtype, rows, V, K):
+    rng = np.random.default_rng(rows * 1000 + V + K)
+    x = rng.standard_normal((rows, V)).astype(np.float32) * 3
+    if dtype == "bf16":
+        x = workloads.round_to_bf16(x)
+    ids, logp, lse, st = _run(x, K, dtype)
+    assert st == 0
+    _check_rows(x, K, ids, logp, lse, range(rows))
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_ties_zero_signs_and_minus_inf(dtype):
+    V = 5000
+    x = np.zeros((6, V), dtype=np.float32)
+    x[0] = 1.5                                            # all equal: ids 0..K-1
+    x[1] = np.where(np.arange(V) % 2 == 0, -0.0, 0.0)     # -0 == +0
+    x[1, 4321] = -1.0
+    x[2] = np.round(np.random.default_rng(1).standard_normal(V) * 2) * 0.25
+    x[3] = -np.inf
+    x[3, [17, 4000, 2]] = [3.0, 3.0, -2.0]                 # mostly -inf, a tie at the top
+    x[4] = np.random.default_rng(2).standard_normal(V)
+    x[4, 100:200] = -np.inf
+    x[5] = 0.5
+    x[5, 4999] = 0.75                                      # maximum in the very last element
+    ids, logp, lse, st = _run(x, 16, dtype)
+    assert st == 0
+    _check_rows(x, 16, ids, logp, lse, range(6))
+
+
+@pytest.mark.parametrize("bad", ["nan", "all_minus_inf", "plus_inf"])
+def test_nonfinite_rows_set_device_status(bad):
+    x = np.random.default_rng(0).standard_normal((4, 3000)).astype(np.float32)
+    if bad == "nan":
+        x[2, 5] = np.nan
+    elif bad == "all_minus_inf":
+        x[1] = -np.inf
+    else:
+        x[3, 7] = np.inf
+    _, _, _, st = _run(x, 4, "f32")
+    assert st == 5
+    ids, logp, lse, st2 = _run(np.zeros((2, 10), np.float32), 3, "f32")
+    assert st2 == 0
+
+
+def test_workspace_reuse_and_split_path_repeatable():
+    ll = _ll()
+    rng = np.random.default_rng(9)
+    x = to_dev(workloads.round_to_bf16(rng.standard_normal((16, 151936)).astype(np.float32)), "bf16")
+    ws = ll.Workspace(ll.lib().lilicorr_topk_lse_workspace_bytes(16, 151936, 8))
+    outs = [ll.topk_lse(x, 8, ws=ws) for _ in range(5)]
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        assert torch.equal(o[0], outs[0][0]) and torch.equal(o[2], outs[0][2])
+    assert ws.status() == 0
