@@ -1,0 +1,32 @@
+/*
+ * lilicorr_testing.h - test hooks of the LiLiCorr library. Not part of the
+ * selection path; they expose internal building blocks so tests can check them
+ * one at a time.
+ */
+#ifndef LILICORR_TESTING_H_
+#define LILICORR_TESTING_H_
+
+#include "lilicorr.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* One linear layer as the scoring network runs it:
+ *   C[M, N] = act(A[M, Kd] W[N, Kd]^T + bias[N]) + residual[M, N]
+ * A, W, C row-major device arrays with leading dimensions lda, ldw, ldc (elements);
+ * bias and residual (fp32, residual with leading dimension ldc) may be NULL;
+ * act 0 = none, 1 = SiLU. path selects the kernel: 0 = the network's own choice,
+ * 1 = tiled CUDA-core kernel, 2 = few-row (split-N) CUDA-core kernel,
+ * 3 = tensor cores (bf16 A and W only; LILICORR_ERR_DTYPE otherwise).
+ * status: a device uint32 word that receives bounded-wait timeouts (may be NULL). */
+lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W,
+                                       lilicorr_dtype_t w_dt, int ldw, void* C,
+                                       lilicorr_dtype_t c_dt, int ldc, int M, int N, int Kd,
+                                       const float* bias, const float* residual, int act, int path,
+                                       uint32_t* status, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LILICORR_TESTING_H_ */

@@ -63,6 +63,8 @@ _SIGS = {
     "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
+    "lilicorr_test_linear": (_I, [_P, _I, _I, _P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I,
+                                  _P, _P]),
 }
 
 
@@ -305,6 +307,20 @@ def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target:
                                        target.data_ptr(), tokens.data_ptr(), ws.ptr, ws.nbytes,
                                        _stream()), "select_block")
     return tokens
+
+
+def test_linear(A: torch.Tensor, W: torch.Tensor, out_dtype=torch.float32, bias=None,
+                residual=None, act: int = 0, path: int = 0, status: Optional[torch.Tensor] = None):
+    """Test hook: one linear layer C = act(A W^T + bias) + residual through kernel `path`
+    (0 auto, 1 tiled CUDA cores, 2 few-row CUDA cores, 3 tensor cores)."""
+    M, Kd = A.shape
+    N = W.shape[0]
+    C = torch.empty((M, N), dtype=out_dtype, device=A.device)
+    _check(lib().lilicorr_test_linear(A.data_ptr(), _dtype_code(A), A.stride(0), W.data_ptr(),
+                                      _dtype_code(W), W.stride(0), C.data_ptr(), _dtype_code(C),
+                                      C.stride(0), M, N, Kd, _ptr(bias), _ptr(residual), act,
+                                      path, _ptr(status), _stream()), "test_linear")
+    return C
 
 
 def select_block_intermediates(head: Head, B: int, ws: Workspace) -> Dict[str, torch.Tensor]:

@@ -9,13 +9,12 @@
 #include <vector>
 
 #include "internal.cuh"
+#include "lilicorr_testing.h"
 
 namespace lilicorr {
 
 size_t attention_smem_bytes(int LK, int hd, int warps);
 size_t pair_walk_smem_bytes(int L, int K, int d);
-bool gemm_tc_supported(const GemmArgs& g);
-lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
 
 static std::atomic<uint64_t> g_launches{0};
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -42,11 +41,12 @@ bool desc_ok(const lilicorr_head_desc* d) {
   if (d->n_layers <= 0 || d->n_layers > 8 || d->n_tgt <= 0) return false;
   if (d->L <= 0 || d->L > LILICORR_MAX_L || d->K <= 0 || d->K > LILICORR_MAX_K) return false;
   if (d->K > d->V || d->L * d->K > LILICORR_MAX_NODES) return false;
-  if (d->D % d->n_heads != 0 || d->D / d->n_heads > 128) return false;
+  if (d->D % d->n_heads != 0 || d->D / d->n_heads > 128 || (d->D / d->n_heads) % 4 != 0)
+    return false;
   // every row handed to a linear layer or a TMA copy stays 16-byte aligned
   if (d->H % 8 != 0 || d->D % 8 != 0 || d->d % 8 != 0 || d->ffn % 8 != 0) return false;
-  if (attention_smem_bytes(d->L * d->K, d->D / d->n_heads, 8) > 227 * 1024) return false;
-  if (pair_walk_smem_bytes(d->L, d->K, d->d) > 227 * 1024) return false;
+  if (attention_smem_bytes(d->L * d->K, d->D / d->n_heads, 8) > 200 * 1024) return false;
+  if (pair_walk_smem_bytes(d->L, d->K, d->d) > 200 * 1024) return false;
   return true;
 }
 
@@ -167,6 +167,7 @@ WsLayout ws_layout(const lilicorr_head_desc& d, int B) {
   w.A = take((size_t)B * d.K * 4);
   w.P = take((size_t)B * (d.L > 1 ? d.L - 1 : 0) * d.K * d.K * 4);
   w.choice = take(R * 4);
+  w.pw_counters = take((size_t)B * 4);
   w.total = o;
   return w;
 }
@@ -193,7 +194,10 @@ GemmArgs gemm(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, lili
   return g;
 }
 
+// Few rows: split-N CUDA-core kernel. bf16 operands: tensor cores. Otherwise the
+// tiled fp32 CUDA-core kernel (the fp32 head keeps fp32 arithmetic throughout).
 lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
+  if (g.M <= 64) return launch_gemm_skinny(g, st);
   if (gemm_tc_supported(g)) return launch_gemm_tc(g, st);
   return launch_gemm_simt(g, st);
 }
@@ -205,81 +209,96 @@ lilicorr_status_t run_head(const lilicorr_head* h, int B, const int32_t* ids, co
                            cudaStream_t st) {
   const lilicorr_head_desc& d = h->desc;
   const lilicorr_dtype_t wdt = d.dtype;
+  const lilicorr_dtype_t adt = d.dtype;     // matrix-product operands: bf16 on the bf16 head
   const lilicorr_dtype_t F32 = LILICORR_F32;
   const int R = B * d.L, N = R * d.K, LK = d.L * d.K;
   const int D = d.D, F = d.ffn;
+  uint32_t* status = at<uint32_t>(ws, w.status);
   float* hproj = at<float>(ws, w.hproj);
   float* tn = at<float>(ws, w.tn);
   float* t = at<float>(ws, w.t);
   float* anc = at<float>(ws, w.anc);
   float* cb = at<float>(ws, w.cb);
   float* x = at<float>(ws, w.x);
-  float* c1 = at<float>(ws, w.c1);
-  float* xn = at<float>(ws, w.xn);
-  float* qkv = at<float>(ws, w.qkv);
-  float* att = at<float>(ws, w.att);
-  float* hf = at<float>(ws, w.hf);
-  float* u = at<float>(ws, w.u);
+  void* c1 = at<void>(ws, w.c1);
+  void* xn = at<void>(ws, w.xn);
+  void* qkv = at<void>(ws, w.qkv);
+  const int hd = D / d.n_heads;
+  const bool tc_attn = wdt == LILICORR_BF16 && attention_tc_supported(hd) &&
+                       attention_tc_smem_bytes(LK, hd, d.L) <= 200 * 1024;
+  const lilicorr_dtype_t qkv_dt = tc_attn ? LILICORR_BF16 : F32;
+  void* att = at<void>(ws, w.att);
+  void* hf = at<void>(ws, w.hf);
+  void* u = at<void>(ws, w.u);
   float* oi = at<float>(ws, w.oi);
+  auto G = [&](const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, int ldw, void* C,
+               lilicorr_dtype_t c_dt, int ldc, int M, int Nn, int Kd) {
+    GemmArgs g = gemm(A, a_dt, lda, W, wdt, ldw, C, c_dt, ldc, M, Nn, Kd);
+    g.status = status;
+    return g;
+  };
 
   // drafter state projection W_h h_s + b_h, one row per slot (shared by its K candidates)
-  GemmArgs g = gemm(hidden, wdt, d.H, h->hid_w, wdt, d.H, hproj, F32, D, R, D, d.H);
+  GemmArgs g = G(hidden, wdt, d.H, h->hid_w, d.H, hproj, F32, D, R, D, d.H);
   g.bias = h->hid_b;
   LL_TRY(run_gemm(g, st));
   // target state t = W_t RMSNorm(mean of the captured layers) + b_t
   LL_TRY(launch_target_norm(target, wdt, B, d.n_tgt, d.H, h->tgt_norm, tn, st));
-  g = gemm(tn, F32, d.H, h->tgt_w, wdt, d.H, t, F32, D, B, D, d.H);
+  g = G(tn, F32, d.H, h->tgt_w, d.H, t, F32, D, B, D, d.H);
   g.bias = h->tgt_b;
   LL_TRY(run_gemm(g, st));
   // anchor out vector o_0 = unit(W_a t + b_a)
-  g = gemm(t, F32, D, h->anc_w, wdt, D, anc, F32, d.d, B, d.d, D);
+  g = G(t, F32, D, h->anc_w, D, anc, F32, d.d, B, d.d, D);
   g.bias = h->anc_b;
   LL_TRY(run_gemm(g, st));
   LL_TRY(launch_unit_rows(anc, B, d.d, d.d, anc, d.d, st));
   // the t block of the fusion layer is constant per sequence: cb = W_f[:, t] t + b_f
-  g = gemm(t, F32, D, h->fuse_t, wdt, D, cb, F32, D, B, D, D);
+  g = G(t, F32, D, h->fuse_t, D, cb, F32, D, B, D, D);
   g.bias = h->fuse_b;
   LL_TRY(run_gemm(g, st));
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
-  LL_TRY(launch_node_build(h, B, ids, logp, hproj, c1, x, at<uint32_t>(ws, w.status), st));
-  g = gemm(c1, F32, D, h->conf2_w, wdt, D, x, F32, D, N, D, D);
+  LL_TRY(launch_node_build(h, B, ids, logp, hproj, c1, adt, x, status, st));
+  g = G(c1, adt, D, h->conf2_w, D, x, F32, D, N, D, D);
   g.bias = h->conf2_b;
   g.residual = x; g.ldr = D;
   LL_TRY(run_gemm(g, st));
   // Transformer layers
   for (int i = 0; i < d.n_layers; ++i) {
     const HeadW& l = h->layer[i];
-    LL_TRY(launch_rmsnorm(x, N, D, l.an, xn, F32, st));
-    g = gemm(xn, F32, D, l.wqkv, wdt, D, qkv, F32, 3 * D, N, 3 * D, D);
+    LL_TRY(launch_rmsnorm(x, N, D, l.an, xn, adt, st));
+    g = G(xn, adt, D, l.wqkv, D, qkv, qkv_dt, 3 * D, N, 3 * D, D);
     g.bias = l.bqkv;
     LL_TRY(run_gemm(g, st));
-    LL_TRY(launch_attention(qkv, B, d.L, d.K, D, d.n_heads, l.dist, l.same, att, st));
-    g = gemm(att, F32, D, l.wo, wdt, D, x, F32, D, N, D, D);
+    if (tc_attn)
+      LL_TRY(launch_attention_tc(qkv, B, d.L, d.K, D, d.n_heads, l.dist, l.same, att, st));
+    else
+      LL_TRY(launch_attention(static_cast<const float*>(qkv), B, d.L, d.K, D, d.n_heads, l.dist,
+                              l.same, att, adt, st));
+    g = G(att, adt, D, l.wo, D, x, F32, D, N, D, D);
     g.bias = l.bo;
     g.residual = x; g.ldr = D;
     LL_TRY(run_gemm(g, st));
-    LL_TRY(launch_rmsnorm(x, N, D, l.fn, xn, F32, st));
-    g = gemm(xn, F32, D, l.w1, wdt, D, hf, F32, F, N, F, D);
+    LL_TRY(launch_rmsnorm(x, N, D, l.fn, xn, adt, st));
+    g = G(xn, adt, D, l.w1, D, hf, adt, F, N, F, D);
     g.bias = l.b1;
     g.act = ACT_SILU;
     LL_TRY(run_gemm(g, st));
-    g = gemm(hf, F32, F, l.w2, wdt, F, x, F32, D, N, D, F);
+    g = G(hf, adt, F, l.w2, F, x, F32, D, N, D, F);
     g.bias = l.b2;
     g.residual = x; g.ldr = D;
     LL_TRY(run_gemm(g, st));
   }
   // fusion u = SiLU(W_f [x; t; x*t] + b_f) with x the final-normed state
-  LL_TRY(launch_fusion_input(x, B, LK, D, h->final_norm, t, xn, F32, st));
-  g = gemm(xn, F32, 2 * D, h->fuse_x, wdt, 2 * D, u, F32, D, N, D, 2 * D);
+  LL_TRY(launch_fusion_input(x, B, LK, D, h->final_norm, t, xn, adt, st));
+  g = G(xn, adt, 2 * D, h->fuse_x, 2 * D, u, adt, D, N, D, 2 * D);
   g.bias_rows = cb;
   g.rows_per_bias = LK;
   g.act = ACT_SILU;
   LL_TRY(run_gemm(g, st));
   // out and in heads in one product: oi = [W_o u + b_o | W_i u + b_i]
-  g = gemm(u, F32, D, h->woi, wdt, D, oi, F32, 2 * d.d, N, 2 * d.d, D);
+  g = G(u, adt, D, h->woi, D, oi, F32, 2 * d.d, N, 2 * d.d, D);
   g.bias = h->boi;
   LL_TRY(run_gemm(g, st));
-  (void)ids;
   return LILICORR_OK;
 }
 
@@ -510,7 +529,7 @@ lilicorr_status_t lilicorr_pair_scores(int B, int L, int K, int d, const float* 
   if (B == 0) return LILICORR_OK;
   if (!out_vec || !in_vec || !anchor_out || !anchor_scores || (L > 1 && !pair_scores))
     return LILICORR_ERR_ARG;
-  if (pair_walk_smem_bytes(L, K, d) > 227 * 1024) return LILICORR_ERR_SHAPE;
+  if (pair_walk_smem_bytes(L, K, d) > 200 * 1024) return LILICORR_ERR_SHAPE;
   PairWalkArgs a;
   memset(&a, 0, sizeof(a));
   a.B = B; a.L = L; a.K = K; a.d = d;
@@ -529,7 +548,7 @@ lilicorr_status_t lilicorr_greedy_walk(int B, int L, int K, const float* anchor_
   if (B == 0) return LILICORR_OK;
   if (!anchor_scores || (L > 1 && !pair_scores) || !ids || !choice || !tokens)
     return LILICORR_ERR_ARG;
-  if (pair_walk_smem_bytes(L, K, 0) > 227 * 1024) return LILICORR_ERR_SHAPE;
+  if (pair_walk_smem_bytes(L, K, 0) > 200 * 1024) return LILICORR_ERR_SHAPE;
   PairWalkArgs a;
   memset(&a, 0, sizeof(a));
   a.B = B; a.L = L; a.K = K; a.d = 0;
@@ -568,6 +587,7 @@ lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const 
   a.A = at<float>(ws, w.A); a.P = at<float>(ws, w.P);
   a.ids = ids; a.choice = at<int32_t>(ws, w.choice); a.tokens = tokens; a.margin = nullptr;
   a.do_pairs = true; a.do_walk = true;
+  a.counters = at<uint32_t>(ws, w.pw_counters);
   return launch_pair_walk(a, stream);
 }
 
@@ -585,6 +605,27 @@ lilicorr_status_t lilicorr_select_block_intermediates(const lilicorr_head* head,
   if (pair_scores) *pair_scores = at<float>(ws, w.P);
   if (choice) *choice = at<int32_t>(ws, w.choice);
   return LILICORR_OK;
+}
+
+lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W,
+                                       lilicorr_dtype_t w_dt, int ldw, void* C,
+                                       lilicorr_dtype_t c_dt, int ldc, int M, int N, int Kd,
+                                       const float* bias, const float* residual, int act, int path,
+                                       uint32_t* status, cudaStream_t stream) {
+  if (!A || !W || !C || M < 0 || N < 0 || Kd <= 0) return LILICORR_ERR_ARG;
+  GemmArgs g = gemm(A, a_dt, lda, W, w_dt, ldw, C, c_dt, ldc, M, N, Kd);
+  g.bias = bias;
+  g.residual = residual;
+  g.ldr = ldc;
+  g.act = act;
+  g.status = status;
+  switch (path) {
+    case 0: return run_gemm(g, stream);
+    case 1: return launch_gemm_simt(g, stream);
+    case 2: return launch_gemm_skinny(g, stream);
+    case 3: return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_DTYPE;
+  }
+  return LILICORR_ERR_ARG;
 }
 
 uint64_t lilicorr_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }

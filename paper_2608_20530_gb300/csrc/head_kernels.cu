@@ -89,34 +89,171 @@ lilicorr_status_t gemm_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st)
   return gemm_dispatch_c<TA, __nv_bfloat16>(g, grid, st);
 }
 
+// ----------------------------------------------------------------------------- skinny linear
+// Few rows (M <= 64: one row per slot or per sequence) against long rows (Kd up to H).
+// CTA (column block of SK_NB, row block of SK_MB): its 256 threads split Kd in
+// 8-element vectors, each accumulating SK_MB x SK_NB partial dot products, reduced by
+// warp shuffles and shared memory. Many CTAs stream disjoint weight rows.
+constexpr int SK_NB = 4, SK_MB = 16, SK_THREADS = 256;
+
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
+  const uint4 a = *reinterpret_cast<const uint4*>(p);
+  const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    v[2 * i] = __uint_as_float(w[i] << 16);
+    v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+template <typename TA, typename TW, typename TC>
+__global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
+  __shared__ float red[SK_THREADS / 32][SK_MB * SK_NB];
+  const TA* A = static_cast<const TA*>(g.A);
+  const TW* W = static_cast<const TW*>(g.W);
+  const int n0 = blockIdx.x * SK_NB, m0 = blockIdx.y * SK_MB;
+  const int nb = min(SK_NB, g.N - n0), mb = min(SK_MB, g.M - m0);
+  float acc[SK_MB][SK_NB];
+#pragma unroll
+  for (int i = 0; i < SK_MB; ++i)
+#pragma unroll
+    for (int j = 0; j < SK_NB; ++j) acc[i][j] = 0.f;
+  for (int k = threadIdx.x * 8; k < g.Kd; k += SK_THREADS * 8) {
+    float w[SK_NB][8];
+#pragma unroll
+    for (int j = 0; j < SK_NB; ++j) {
+      if (j < nb) load8(W + (size_t)(n0 + j) * g.ldw + k, w[j]);
+      else
+#pragma unroll
+        for (int e = 0; e < 8; ++e) w[j][e] = 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < SK_MB; ++i) {
+      if (i >= mb) break;
+      float a[8];
+      load8(A + (size_t)(m0 + i) * g.lda + k, a);
+#pragma unroll
+      for (int j = 0; j < SK_NB; ++j)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[i][j] = fmaf(a[e], w[j][e], acc[i][j]);
+    }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < SK_MB; ++i)
+#pragma unroll
+    for (int j = 0; j < SK_NB; ++j) {
+      const float v = warp_sum(acc[i][j]);
+      if (lane == 0) red[warp][i * SK_NB + j] = v;
+    }
+  __syncthreads();
+  if (threadIdx.x < SK_MB * SK_NB) {
+    const int i = threadIdx.x / SK_NB, j = threadIdx.x % SK_NB;
+    if (i < mb && j < nb) {
+      float v = 0.f;
+#pragma unroll
+      for (int w = 0; w < SK_THREADS / 32; ++w) v += red[w][threadIdx.x];
+      const int m = m0 + i, n = n0 + j;
+      if (g.bias) v += g.bias[n];
+      if (g.bias_rows) v += g.bias_rows[(size_t)(m / g.rows_per_bias) * g.N + n];
+      if (g.act == ACT_SILU) v = silu_f(v);
+      if (g.residual) v += g.residual[(size_t)m * g.ldr + n];
+      st_elem(static_cast<TC*>(g.C), (size_t)m * g.ldc + n, v);
+    }
+  }
+}
+
+template <typename TA, typename TW>
+lilicorr_status_t skinny_dispatch_c(const GemmArgs& g, dim3 grid, cudaStream_t st) {
+  if (g.c_dt == LILICORR_F32) gemm_skinny_kernel<TA, TW, float><<<grid, SK_THREADS, 0, st>>>(g);
+  else gemm_skinny_kernel<TA, TW, __nv_bfloat16><<<grid, SK_THREADS, 0, st>>>(g);
+  return last_launch();
+}
+template <typename TA>
+lilicorr_status_t skinny_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st) {
+  if (g.w_dt == LILICORR_F32) return skinny_dispatch_c<TA, float>(g, grid, st);
+  return skinny_dispatch_c<TA, __nv_bfloat16>(g, grid, st);
+}
+
 // ----------------------------------------------------------------------------- target state
 // tn[b] = RMSNorm_H(mean over the n_tgt captured layers of T[b]) * gain (App. A).
+// One CTA per sequence; each thread owns 8-element vectors of the row (H % 8 == 0),
+// keeps its means in registers between the two passes (up to TN_VPT vectors).
+constexpr int TN_THREADS = 512, TN_VPT = 4;
+
 template <typename T>
-__global__ void target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H,
-                                   const float* __restrict__ gain, float* __restrict__ tn) {
-  __shared__ float red[32];
+__global__ void __launch_bounds__(TN_THREADS)
+target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H, const float* __restrict__ gain,
+                   float* __restrict__ tn) {
+  __shared__ float red[TN_THREADS / 32];
+  __shared__ float s_total;
   const int b = blockIdx.x;
   const T* tb = Tin + (size_t)b * n_tgt * H;
+  const int nv = H / 8;
+  float mean[TN_VPT][8];
   float ss = 0.f;
-  for (int h = threadIdx.x; h < H; h += blockDim.x) {
-    float acc = 0.f;
-    for (int l = 0; l < n_tgt; ++l) acc += ld_elem(tb, (size_t)l * H + h);
-    acc /= (float)n_tgt;
-    tn[(size_t)b * H + h] = acc;
-    ss += acc * acc;
+  const float inv_p = 1.0f / (float)n_tgt;
+#pragma unroll
+  for (int q = 0; q < TN_VPT; ++q) {
+    const int v = threadIdx.x + q * TN_THREADS;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) mean[q][e] = 0.f;
+    if (v >= nv) continue;
+    for (int l = 0; l < n_tgt; ++l) {
+      float x[8];
+      load8(tb + (size_t)l * H + v * 8, x);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mean[q][e] += x[e];
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      mean[q][e] *= inv_p;
+      ss += mean[q][e] * mean[q][e];
+    }
+  }
+  // rows longer than TN_VPT * TN_THREADS * 8 are handled by a second strided pass
+  for (int v = threadIdx.x + TN_VPT * TN_THREADS; v < nv; v += TN_THREADS) {
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    for (int l = 0; l < n_tgt; ++l) {
+      float x[8];
+      load8(tb + (size_t)l * H + v * 8, x);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] += x[e];
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      acc[e] *= inv_p;
+      ss += acc[e] * acc[e];
+      tn[(size_t)b * H + v * 8 + e] = acc[e];
+    }
   }
   ss = warp_sum(ss);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
   __syncthreads();
   if (threadIdx.x < 32) {
-    float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+    float v = threadIdx.x < TN_THREADS / 32 ? red[threadIdx.x] : 0.f;
     v = warp_sum(v);
-    if (threadIdx.x == 0) red[0] = v;
+    if (threadIdx.x == 0) s_total = v;
   }
   __syncthreads();
-  const float r = rsqrtf(red[0] / (float)H + RMS_EPS);
-  for (int h = threadIdx.x; h < H; h += blockDim.x)
-    tn[(size_t)b * H + h] = tn[(size_t)b * H + h] * r * gain[h];
+  const float r = rsqrtf(s_total / (float)H + RMS_EPS);
+#pragma unroll
+  for (int q = 0; q < TN_VPT; ++q) {
+    const int v = threadIdx.x + q * TN_THREADS;
+    if (v >= nv) continue;
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      tn[(size_t)b * H + v * 8 + e] = mean[q][e] * r * gain[v * 8 + e];
+  }
+  for (int v = threadIdx.x + TN_VPT * TN_THREADS; v < nv; v += TN_THREADS)
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      tn[(size_t)b * H + v * 8 + e] = tn[(size_t)b * H + v * 8 + e] * r * gain[v * 8 + e];
 }
 
 // ----------------------------------------------------------------------------- nodes
@@ -125,11 +262,12 @@ __global__ void target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H,
 //                                 layer is a linear launch that adds into x)
 //   x  = fold[id_k] + hproj[r] + slot[s] + rank[k]
 // with f_k = [logp_k, exp(logp_k), logp_0 - logp_k, k / (K-1), 1{k = 0}].
+template <typename TC1>
 __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __restrict__ ids,
                                   const float* __restrict__ logp, const float* __restrict__ fold,
                                   const float* __restrict__ hproj, const float* __restrict__ slot,
                                   const float* __restrict__ rank, const float* __restrict__ w1,
-                                  const float* __restrict__ b1, float* __restrict__ c1,
+                                  const float* __restrict__ b1, TC1* __restrict__ c1,
                                   float* __restrict__ x, uint32_t* status) {
   __shared__ float f[LILICORR_MAX_K][LILICORR_N_CONF];
   __shared__ int sid[LILICORR_MAX_K];
@@ -152,15 +290,29 @@ __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __r
     sid[k] = id;
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < K * D; i += blockDim.x) {
-    const int k = i / D, n = i % D;
-    float z = b1[n];
-#pragma unroll
-    for (int j = 0; j < LILICORR_N_CONF; ++j) z = fmaf(w1[n * LILICORR_N_CONF + j], f[k][j], z);
+  const int D4 = D / 4;
+#pragma unroll 2
+  for (int i = threadIdx.x; i < K * D4; i += blockDim.x) {
+    const int k = i / D4, n = (i % D4) * 4;
     const size_t node = (size_t)r * K + k;
-    c1[node * D + n] = silu_f(z);
-    x[node * D + n] = fold[(size_t)sid[k] * D + n] + hproj[(size_t)r * D + n] +
-                      slot[(size_t)s * D + n] + rank[(size_t)k * D + n];
+    const float4 fo = *reinterpret_cast<const float4*>(fold + (size_t)sid[k] * D + n);
+    const float4 hp = *reinterpret_cast<const float4*>(hproj + (size_t)r * D + n);
+    const float4 sl = *reinterpret_cast<const float4*>(slot + (size_t)s * D + n);
+    const float4 rk = *reinterpret_cast<const float4*>(rank + (size_t)k * D + n);
+    float4 o;
+    o.x = fo.x + hp.x + sl.x + rk.x;
+    o.y = fo.y + hp.y + sl.y + rk.y;
+    o.z = fo.z + hp.z + sl.z + rk.z;
+    o.w = fo.w + hp.w + sl.w + rk.w;
+    *reinterpret_cast<float4*>(x + node * D + n) = o;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float z = b1[n + q];
+#pragma unroll
+      for (int j = 0; j < LILICORR_N_CONF; ++j)
+        z = fmaf(w1[(n + q) * LILICORR_N_CONF + j], f[k][j], z);
+      st_elem(c1, node * D + n + q, silu_f(z));
+    }
   }
 }
 
@@ -219,12 +371,14 @@ __global__ void unit_rows_kernel(const float* __restrict__ src, int rows, int n,
 // One CTA per (sequence, head): all L*K nodes attend to all L*K nodes (no mask),
 // logits q.k / sqrt(hd) + dist[h, s_j - s_i + L - 1] + same[h] * 1{s_i == s_j}.
 // qkv rows hold [q | k | v], each D wide, head h in columns [h*hd, (h+1)*hd).
+template <typename TO>
 __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, int D, int n_heads,
-                                 const float* __restrict__ dist, const float* __restrict__ same,
-                                 float* __restrict__ out) {
+                                 int q_per_cta, const float* __restrict__ dist,
+                                 const float* __restrict__ same, TO* __restrict__ out) {
   extern __shared__ float sm[];
   const int LK = L * K, hd = D / n_heads;
   const int b = blockIdx.x / n_heads, h = blockIdx.x % n_heads;
+  const int q0 = blockIdx.y * q_per_cta, q1 = min(LK, q0 + q_per_cta);
   const int nw = blockDim.x >> 5, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* Ks = sm;                       // [LK][hd + 1]
   float* Vs = Ks + (size_t)LK * (hd + 1);   // [LK][hd]
@@ -232,10 +386,15 @@ __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, in
   float* Pw = Qw + (size_t)nw * hd;     // [nw][LK]
   const size_t ld = 3 * (size_t)D;
   const float* base = qkv + (size_t)b * LK * ld;
-  for (int i = threadIdx.x; i < LK * hd; i += blockDim.x) {
-    const int j = i / hd, c = i % hd;
-    Ks[j * (hd + 1) + c] = base[j * ld + D + h * hd + c];
-    Vs[j * hd + c] = base[j * ld + 2 * D + h * hd + c];
+  const int hv = hd / 4;                       // 16-byte vectors per head row
+#pragma unroll 4
+  for (int i = threadIdx.x; i < LK * hv; i += blockDim.x) {
+    const int j = i / hv, c = (i % hv) * 4;
+    const float4 kv = *reinterpret_cast<const float4*>(base + j * ld + D + h * hd + c);
+    const float4 vv = *reinterpret_cast<const float4*>(base + j * ld + 2 * D + h * hd + c);
+    float* kd = Ks + j * (hd + 1) + c;
+    kd[0] = kv.x; kd[1] = kv.y; kd[2] = kv.z; kd[3] = kv.w;
+    *reinterpret_cast<float4*>(Vs + j * hd + c) = vv;
   }
   __syncthreads();
   const float scale = rsqrtf((float)hd);
@@ -243,7 +402,7 @@ __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, in
   const float sh = same[h];
   float* q = Qw + warp * hd;
   float* p = Pw + (size_t)warp * LK;
-  for (int i = warp; i < LK; i += nw) {
+  for (int i = q0 + warp; i < q1; i += nw) {
     for (int c = lane; c < hd; c += 32) q[c] = base[(size_t)i * ld + h * hd + c];
     __syncwarp();
     const int si = i / K;
@@ -270,7 +429,7 @@ __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, in
     for (int c = lane; c < hd; c += 32) {
       float acc = 0.f;
       for (int j = 0; j < LK; ++j) acc = fmaf(p[j], Vs[j * hd + c], acc);
-      out[((size_t)b * LK + i) * D + h * hd + c] = acc * inv;
+      st_elem(out, ((size_t)b * LK + i) * D + h * hd + c, acc * inv);
     }
     __syncwarp();
   }
@@ -281,6 +440,14 @@ __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, in
 size_t attention_smem_bytes(int LK, int hd, int warps) {
   return sizeof(float) * ((size_t)LK * (hd + 1) + (size_t)LK * hd + (size_t)warps * hd +
                           (size_t)warps * LK);
+}
+
+lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st) {
+  if (g.M == 0 || g.N == 0) return LILICORR_OK;
+  if ((g.Kd % 8) || (g.lda % 8) || (g.ldw % 8)) return launch_gemm_simt(g, st);
+  dim3 grid(ceil_div(g.N, SK_NB), ceil_div(g.M, SK_MB));
+  if (g.a_dt == LILICORR_F32) return skinny_dispatch_w<float>(g, grid, st);
+  return skinny_dispatch_w<__nv_bfloat16>(g, grid, st);
 }
 
 lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st) {
@@ -294,21 +461,29 @@ lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, 
                                      const float* gain, float* tn, cudaStream_t st) {
   if (B == 0) return LILICORR_OK;
   if (dt == LILICORR_F32)
-    target_norm_kernel<float><<<B, 256, 0, st>>>(static_cast<const float*>(T), n_tgt, H, gain, tn);
+    target_norm_kernel<float><<<B, TN_THREADS, 0, st>>>(static_cast<const float*>(T), n_tgt, H, gain,
+                                                        tn);
   else
-    target_norm_kernel<__nv_bfloat16><<<B, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(T),
-                                                         n_tgt, H, gain, tn);
+    target_norm_kernel<__nv_bfloat16><<<B, TN_THREADS, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, tn);
   return last_launch();
 }
 
 lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
-                                    const float* logp, const float* hproj, float* c1, float* x,
-                                    uint32_t* status, cudaStream_t st) {
+                                    const float* logp, const float* hproj, void* c1,
+                                    lilicorr_dtype_t c1_dt, float* x, uint32_t* status,
+                                    cudaStream_t st) {
   const lilicorr_head_desc& d = h->desc;
   if (B == 0) return LILICORR_OK;
-  node_build_kernel<<<B * d.L, 256, 0, st>>>(d.L, d.K, d.D, d.V, ids, logp,
-                                             static_cast<const float*>(h->fold), hproj, h->slot,
-                                             h->rank, h->conf1_w, h->conf1_b, c1, x, status);
+  const float* fold = static_cast<const float*>(h->fold);
+  if (c1_dt == LILICORR_F32)
+    node_build_kernel<float><<<B * d.L, 256, 0, st>>>(d.L, d.K, d.D, d.V, ids, logp, fold, hproj,
+                                                      h->slot, h->rank, h->conf1_w, h->conf1_b,
+                                                      static_cast<float*>(c1), x, status);
+  else
+    node_build_kernel<__nv_bfloat16><<<B * d.L, 256, 0, st>>>(
+        d.L, d.K, d.D, d.V, ids, logp, fold, hproj, h->slot, h->rank, h->conf1_w, h->conf1_b,
+        static_cast<__nv_bfloat16*>(c1), x, status);
   return last_launch();
 }
 
@@ -346,20 +521,27 @@ lilicorr_status_t launch_unit_rows(const float* src, int rows, int n, int ld_src
 }
 
 lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D, int n_heads,
-                                   const float* dist, const float* same, float* out,
-                                   cudaStream_t st) {
+                                   const float* dist, const float* same, void* out,
+                                   lilicorr_dtype_t out_dt, cudaStream_t st) {
   if (B == 0) return LILICORR_OK;
   const int warps = 8;
-  const size_t smem = attention_smem_bytes(L * K, D / n_heads, warps);
-  static bool configured[64] = {false};
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 64 && !configured[dev]) {
-    LL_CUDA_TRY(cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     227 * 1024));
-    configured[dev] = true;
-  }
-  attention_kernel<<<B * n_heads, warps * 32, smem, st>>>(qkv, L, K, D, n_heads, dist, same, out);
+  const int LK = L * K;
+  const size_t smem = attention_smem_bytes(LK, D / n_heads, warps);
+  static bool cfg_f32[64] = {false}, cfg_bf16[64] = {false};
+  LL_TRY(allow_max_dynamic_smem(attention_kernel<float>, cfg_f32));
+  LL_TRY(allow_max_dynamic_smem(attention_kernel<__nv_bfloat16>, cfg_bf16));
+  // split the queries of a (sequence, head) over CTAs until the grid covers the GPU
+  int qblocks = ceil_div(2 * num_sms(), B * n_heads);
+  qblocks = max(1, min(qblocks, ceil_div(LK, 2 * warps)));
+  const int q_per_cta = ceil_div(LK, qblocks);
+  qblocks = ceil_div(LK, q_per_cta);
+  dim3 grid(B * n_heads, qblocks);
+  if (out_dt == LILICORR_F32)
+    attention_kernel<float><<<grid, warps * 32, smem, st>>>(qkv, L, K, D, n_heads, q_per_cta, dist,
+                                                            same, static_cast<float*>(out));
+  else
+    attention_kernel<__nv_bfloat16><<<grid, warps * 32, smem, st>>>(
+        qkv, L, K, D, n_heads, q_per_cta, dist, same, static_cast<__nv_bfloat16*>(out));
   return last_launch();
 }
 

@@ -14,7 +14,10 @@ namespace lilicorr {
 #define LL_CUDA_TRY(expr)                                   \
   do {                                                      \
     cudaError_t _e = (expr);                                \
-    if (_e != cudaSuccess) return LILICORR_ERR_CUDA;        \
+    if (_e != cudaSuccess) {                                \
+      (void)cudaGetLastError(); /* do not leak into later calls */ \
+      return LILICORR_ERR_CUDA;                             \
+    }                                                       \
   } while (0)
 
 #define LL_TRY(expr)                                        \
@@ -32,6 +35,29 @@ inline lilicorr_status_t last_launch() {
 }
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+constexpr int SMEM_PER_BLOCK_MAX = 227 * 1024;   // opt-in shared memory per block (sm_103a)
+
+// Raise a kernel's dynamic shared-memory cap to what is left beside its static shared
+// memory, once per device.
+template <typename F>
+lilicorr_status_t allow_max_dynamic_smem(F* func, bool (&done)[64]) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) { (void)cudaGetLastError(); return LILICORR_ERR_CUDA; }
+  if (dev < 0 || dev >= 64 || done[dev]) return LILICORR_OK;
+  cudaFuncAttributes attr;
+  if (cudaFuncGetAttributes(&attr, func) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return LILICORR_ERR_CUDA;
+  }
+  const int dyn = SMEM_PER_BLOCK_MAX - (int)attr.sharedSizeBytes;
+  if (cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return LILICORR_ERR_CUDA;
+  }
+  done[dev] = true;
+  return LILICORR_OK;
+}
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline int ceil_div(long long a, long long b) { return (int)((a + b - 1) / b); }
 
@@ -124,7 +150,7 @@ struct WsLayout {
   size_t ids, logp, lse;
   size_t hproj, tn, t, anc, cb;
   size_t x, c1, xn, qkv, att, hf, u, oi;
-  size_t A, P, choice;
+  size_t A, P, choice, pw_counters;
   size_t total;
 };
 WsLayout ws_layout(const lilicorr_head_desc& d, int B);
@@ -147,20 +173,31 @@ struct GemmArgs {
   const float* residual; int ldr;
   int act;
   int M, N, Kd;
+  uint32_t* status;        // device status word (bounded-wait timeouts), may be null
 };
 lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
+lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st);   // M <= 64
+bool gemm_tc_supported(const GemmArgs& g);
+lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
 
 // scoring-network helpers (head_kernels.cu)
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
                                      const float* gain, float* tn, cudaStream_t st);
 lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
-                                    const float* logp, const float* hproj, float* c1, float* x,
-                                    uint32_t* status, cudaStream_t st);
+                                    const float* logp, const float* hproj, void* c1,
+                                    lilicorr_dtype_t c1_dt, float* x, uint32_t* status,
+                                    cudaStream_t st);
 lilicorr_status_t launch_rmsnorm(const float* x, int M, int D, const float* gain, void* y,
                                  lilicorr_dtype_t y_dt, cudaStream_t st);
 lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D, int n_heads,
-                                   const float* dist, const float* same, float* out,
-                                   cudaStream_t st);
+                                   const float* dist, const float* same, void* out,
+                                   lilicorr_dtype_t out_dt, cudaStream_t st);
+// bf16 attention core on warp-level tensor-core instructions (attention_tc.cu)
+bool attention_tc_supported(int hd);
+size_t attention_tc_smem_bytes(int LK, int hd, int L);
+lilicorr_status_t launch_attention_tc(const void* qkv, int B, int L, int K, int D, int n_heads,
+                                      const float* dist, const float* same, void* out,
+                                      cudaStream_t st);
 lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, const float* gain,
                                       const float* t, void* fin, lilicorr_dtype_t dt,
                                       cudaStream_t st);
@@ -176,6 +213,7 @@ struct PairWalkArgs {
   const int32_t* ids;                             // [B, L, K] (walk)
   int32_t* choice; int32_t* tokens; float* margin;
   bool do_pairs, do_walk;
+  uint32_t* counters;                             // [B] zeroed tickets (pairs + walk fused)
   bool scores_in_smem;                            // set by the launcher
 };
 lilicorr_status_t launch_pair_walk(const PairWalkArgs& a, cudaStream_t st);

@@ -4,14 +4,20 @@
 // extraction with vocabulary-wide logit normalisation. Here every logit is read
 // from HBM exactly once:
 //   * grid = (splits, rows): each CTA streams one contiguous chunk of one row with
-//     16-byte loads, 4 in flight per thread;
+//     16-byte loads, a batch of 4 per thread in flight;
 //   * every thread keeps an online (max, sum exp) pair, merged by warp shuffles;
-//   * every warp keeps its top-K as order-preserving 64-bit keys
-//     (value, then lower id first) in shared memory, filtering with a warp-uniform
-//     threshold; candidates that pass are appended through a ballot and merged
-//     into the list when the buffer fills (rare after the first few vectors);
-//   * the last CTA of a row to finish (atomic ticket, no waiting) merges the
-//     splits' partial (max, sum, top-K) records and writes ids, logp, lse.
+//   * candidates are kept as order-preserving 64-bit keys (value, then lower id
+//     first). The hot loop costs one compare per batch: a warp looks at a batch
+//     only if some lane's batch maximum reaches the threshold, the larger of the
+//     warp's own K-th value and the CTA's (shared memory; every warp's K-th value
+//     bounds the CTA's K-th from below). On such a batch the warp first raises the
+//     threshold to the K-th largest lane maximum (each lane maximum is a distinct
+//     element, so at least K elements reach it), then appends the elements that
+//     pass to a per-warp buffer, one ballot round per hot element of the busiest
+//     lane. A full buffer is merged into the warp's list by rank counting;
+//   * the CTA merges its warps' lists by rank counting; with several splits per
+//     row the last CTA to finish (atomic ticket, no waiting) merges the splits'
+//     partial (max, sum, top-K) records and writes ids, logp and lse.
 #include "internal.cuh"
 
 namespace lilicorr {
@@ -20,9 +26,10 @@ namespace {
 
 constexpr int TK_THREADS = 256;
 constexpr int TK_WARPS = TK_THREADS / 32;
-constexpr int TK_CAP = 96;             // candidate buffer per warp
-constexpr int TK_UNROLL = 4;           // 16-byte loads in flight per thread
+constexpr int TK_CAP = 64;             // candidate buffer per warp
+constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch
 constexpr int TK_MAX_SPLITS = 64;
+constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr unsigned FULL = 0xffffffffu;
 
@@ -40,6 +47,14 @@ __device__ __forceinline__ float key_value(uint64_t k) {
 __device__ __forceinline__ int32_t key_id(uint64_t k) {
   return (int32_t)(0xFFFFFFFFu - (uint32_t)k);
 }
+// order-preserving 32-bit image of a float (for atomicMax on a threshold)
+__device__ __forceinline__ uint32_t ord32(float v) {
+  const uint32_t b = __float_as_uint(v);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float unord32(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -47,84 +62,32 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const uint64_t w = __shfl_xor_sync(FULL, v, o);
-    v = w > v ? w : v;
-  }
-  return v;
-}
-
-// K largest keys of keys[0..n) (distinct except zeros = empty), by K rounds of
-// "largest key below the previous one". Lane r returns the r-th key (0 if none).
-__device__ uint64_t warp_select(const uint64_t* keys, int n, int K, int lane) {
-  uint64_t prev = ~0ull, mine = 0ull;
-  for (int r = 0; r < K; ++r) {
-    uint64_t best = 0ull;
-    for (int i = lane; i < n; i += 32) {
-      const uint64_t k = keys[i];
-      if (k < prev && k > best) best = k;
-    }
-    best = warp_max_u64(best);
-    if (lane == r) mine = best;
-    prev = best;
-    if (best == 0ull) break;
-  }
-  return mine;
-}
-
-struct WarpState {
-  uint64_t* list;    // [LILICORR_MAX_K] sorted descending; 0 = empty
-  uint64_t* buf;     // [TK_CAP]; list and buf are contiguous: list first
-  int nbuf;
-  uint64_t thr;      // K-th key of the list (0 while the list is not full)
-  float thr_val;     // its value (-inf while not full)
-};
-
-// Merge buffer and list into the list. The candidate set is list[0..K) followed by
-// buf[0..nbuf) in one contiguous array, so a single selection pass covers both.
-__device__ __forceinline__ void warp_flush(WarpState& w, int K, int lane) {
-  __syncwarp();
-  const uint64_t mine = warp_select(w.list, LILICORR_MAX_K + w.nbuf, K, lane);
-  __syncwarp();
-  if (lane < K) w.list[lane] = mine;
-  w.thr = __shfl_sync(FULL, mine, K - 1);
-  w.thr_val = w.thr ? key_value(w.thr) : -INFINITY;
-  w.nbuf = 0;
-  __syncwarp();
-}
-
-// Offer n values (ids id0 + j) of this lane to the warp list. Warp-collective.
-template <int N>
-__device__ __forceinline__ void warp_offer(WarpState& w, const float (&x)[N], uint32_t id0,
-                                           bool hot, int K, int lane) {
-#pragma unroll
-  for (int j = 0; j < N; ++j) {
-    const uint64_t key = make_key(x[j], id0 + (uint32_t)j);
-    unsigned m = __ballot_sync(FULL, hot && key > w.thr);
-    if (m == 0u) continue;
-    if (w.nbuf + __popc(m) > TK_CAP) {
-      warp_flush(w, K, lane);
-      m = __ballot_sync(FULL, hot && key > w.thr);
-      if (m == 0u) continue;
-    }
-    if ((m >> lane) & 1u) w.buf[w.nbuf + __popc(m & ((1u << lane) - 1u))] = key;
-    w.nbuf += __popc(m);
+// Rank counting: each key of keys[0..n) (distinct apart from zeros, which mean "empty")
+// counts the keys larger than itself and, if that rank is below K, lands in out[rank].
+// Run by `nthreads` threads with indices t; out[0..K) must be zeroed beforehand and
+// must not alias keys; the caller synchronises before and after.
+__device__ __forceinline__ void rank_place(const uint64_t* keys, int n, int K, uint64_t* out,
+                                           int t, int nthreads) {
+  for (int i = t; i < n; i += nthreads) {
+    const uint64_t c = keys[i];
+    if (c == 0ull) continue;
+    int rank = 0;
+    for (int j = 0; j < n; ++j) rank += keys[j] > c ? 1 : 0;
+    if (rank < K) out[rank] = c;
   }
 }
 
 template <int N>
-__device__ __forceinline__ void lse_update(float& m, float& s, const float (&x)[N], bool valid) {
-  if (!valid) return;
+__device__ __forceinline__ float lse_update(float& m, float& s, const float (&x)[N], bool valid) {
   float vmax = x[0];
 #pragma unroll
   for (int j = 1; j < N; ++j) vmax = fmaxf(vmax, x[j]);
+  if (!valid) return -INFINITY;
   if (vmax > m) {
     s *= ex2((m - vmax) * LOG2E);
     m = vmax;
   }
-  if (m == -INFINITY) return;
+  if (m == -INFINITY) return vmax;
   const float ml = m * LOG2E;
   float acc[N];
 #pragma unroll
@@ -134,6 +97,7 @@ __device__ __forceinline__ void lse_update(float& m, float& s, const float (&x)[
 #pragma unroll
     for (int j = 0; j + w < N; j += 2 * w) acc[j] += acc[j + w];
   s += acc[0];
+  return vmax;
 }
 
 template <typename T> struct Vec;
@@ -158,6 +122,83 @@ template <> struct Vec<float> {
   __device__ static float scalar(const float* p, size_t i) { return p[i]; }
 };
 
+// K-th largest (K <= 32) of one value per lane, by a bitonic sort across the warp.
+__device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const float o = __shfl_xor_sync(FULL, v, stride);
+      const bool lower = (lane & stride) == 0, desc = (lane & size) == 0;
+      v = (lower == desc) ? fmaxf(v, o) : fminf(v, o);
+    }
+  return __shfl_sync(FULL, v, K - 1);
+}
+
+struct WarpTopK {
+  uint64_t* list;      // [LILICORR_MAX_K] descending, 0 = empty
+  uint64_t* buf;       // [TK_CAP]; list and buf contiguous (list first)
+  uint64_t* tmp;       // [LILICORR_MAX_K] scratch of the merge
+  uint32_t* cta_thr;   // CTA-wide threshold (order image), shared by the warps
+  int nbuf;
+  uint64_t thr;        // K-th key of the list (0 while not full)
+  float thr_val;       // value threshold of this warp (never decreases)
+};
+
+// Merge the buffer into the list (rank counting over list + buffer) and raise the
+// thresholds. Warp-collective.
+__device__ __forceinline__ void warp_flush(WarpTopK& w, int K, int lane) {
+  __syncwarp();
+  const int n = LILICORR_MAX_K + w.nbuf;
+  if (lane < K) w.tmp[lane] = 0ull;
+  __syncwarp();
+  rank_place(w.list, n, K, w.tmp, lane, 32);
+  __syncwarp();
+  uint64_t mine = lane < K ? w.tmp[lane] : 0ull;
+  if (lane < LILICORR_MAX_K) w.list[lane] = mine;
+  w.thr = __shfl_sync(FULL, mine, K - 1);
+  if (w.thr) {
+    w.thr_val = fmaxf(w.thr_val, key_value(w.thr));
+    if (lane == 0) atomicMax(w.cta_thr, ord32(w.thr_val));
+  }
+  w.nbuf = 0;
+  __syncwarp();
+}
+
+// Append x (id) to the warp buffer if `c`; warp-collective. Flushes when full.
+__device__ __forceinline__ void warp_append(WarpTopK& w, float x, uint32_t id, bool c, int K,
+                                            int lane) {
+  uint64_t key = make_key(x, id);
+  unsigned m = __ballot_sync(FULL, c && key > w.thr);
+  if (m == 0u) return;
+  if (w.nbuf + __popc(m) > TK_CAP) {
+    warp_flush(w, K, lane);
+    m = __ballot_sync(FULL, c && x >= w.thr_val && key > w.thr);
+    if (m == 0u) return;
+  }
+  if ((m >> lane) & 1u) w.buf[w.nbuf + __popc(m & ((1u << lane) - 1u))] = key;
+  w.nbuf += __popc(m);
+}
+
+// Offer the elements of one vector that reach thr: one ballot round per hot element
+// of the busiest lane. Warp-collective.
+template <int N>
+__device__ __forceinline__ void warp_offer(WarpTopK& w, const float (&x)[N], uint32_t id0,
+                                           bool valid, float thr, int K, int lane) {
+  uint32_t hm = 0u;
+#pragma unroll
+  for (int j = 0; j < N; ++j) hm |= (valid && x[j] >= thr) ? (1u << j) : 0u;
+  while (__any_sync(FULL, hm != 0u)) {
+    const bool has = hm != 0u;
+    const int j = has ? __ffs(hm) - 1 : 0;
+    hm &= hm - 1u;
+    float xv = x[0];
+#pragma unroll
+    for (int t = 1; t < N; ++t) xv = (j == t) ? x[t] : xv;
+    warp_append(w, xv, id0 + (uint32_t)j, has, K, lane);
+  }
+}
+
 struct Rec {            // partial record of one (row, split)
   float m, s;
   uint64_t keys[1];     // [K]
@@ -171,8 +212,11 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
                 unsigned char* partials) {
   constexpr int VEC = Vec<T>::N;
   __shared__ uint64_t s_keys[TK_WARPS][LILICORR_MAX_K + TK_CAP];
-  __shared__ uint64_t s_merge[TK_MAX_SPLITS * LILICORR_MAX_K];
+  __shared__ uint64_t s_tmp[TK_WARPS][LILICORR_MAX_K];
+  __shared__ uint64_t s_merge[TK_MERGE_MAX];
+  __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ float s_m[TK_WARPS], s_s[TK_WARPS];
+  __shared__ uint32_t s_cta_thr;
   __shared__ int s_last;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -187,14 +231,17 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   const int v_begin = min(split * chunk_vecs, nvec);
   const int v_end = min(v_begin + chunk_vecs, nvec);
 
-  WarpState w;
+  WarpTopK w;
   w.list = s_keys[warp];
   w.buf = s_keys[warp] + LILICORR_MAX_K;
+  w.tmp = s_tmp[warp];
+  w.cta_thr = &s_cta_thr;
   w.nbuf = 0;
   w.thr = 0ull;
   w.thr_val = -INFINITY;
   w.list[lane] = 0ull;
-  __syncwarp();
+  if (tid == 0) s_cta_thr = ord32(-INFINITY);
+  __syncthreads();
 
   float m = -INFINITY, s = 0.f;
 
@@ -208,34 +255,39 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       const int e = valid ? (i < e0 ? i : tail0 + (i - e0)) : 0;
       float x[1] = {valid ? Vec<T>::scalar(rp, e) : -INFINITY};
       lse_update<1>(m, s, x, valid);
-      const bool hot = valid && x[0] >= w.thr_val;
-      if (__any_sync(FULL, hot)) warp_offer<1>(w, x, (uint32_t)e, hot, K, lane);
+      warp_offer<1>(w, x, (uint32_t)e, valid, w.thr_val, K, lane);
     }
   }
 
-  // main stream: 16-byte vectors, TK_UNROLL loads in flight per thread
+  // main stream: batches of TK_UNROLL 16-byte vectors per thread
   const uint4* vp = reinterpret_cast<const uint4*>(rp + e0);
   for (int it = v_begin; it < v_end; it += TK_UNROLL * TK_THREADS) {
     uint4 raw[TK_UNROLL];
 #pragma unroll
     for (int u = 0; u < TK_UNROLL; ++u) {
       const int v = it + u * TK_THREADS + tid;
-      if (v < v_end) raw[u] = __ldcs(vp + v);
-      else raw[u] = make_uint4(0, 0, 0, 0);
+      raw[u] = v < v_end ? __ldcs(vp + v) : make_uint4(0, 0, 0, 0);
     }
+    float bmax = -INFINITY;
 #pragma unroll
     for (int u = 0; u < TK_UNROLL; ++u) {
-      const int v = it + u * TK_THREADS + tid;
-      const bool valid = v < v_end;
       float x[VEC];
       Vec<T>::unpack(raw[u], x);
-      lse_update<VEC>(m, s, x, valid);
-      float vmax = x[0];
+      bmax = fmaxf(bmax, lse_update<VEC>(m, s, x, it + u * TK_THREADS + tid < v_end));
+    }
+    float thr = fmaxf(w.thr_val, unord32(*(volatile uint32_t*)&s_cta_thr));
+    if (__any_sync(FULL, bmax >= thr)) {
+      // raise the bound to the K-th largest lane maximum of this batch
+      thr = fmaxf(thr, warp_kth_largest(bmax, K, lane));
+      w.thr_val = thr;
 #pragma unroll
-      for (int j = 1; j < VEC; ++j) vmax = fmaxf(vmax, x[j]);
-      const bool hot = valid && vmax >= w.thr_val;
-      if (__any_sync(FULL, hot))
-        warp_offer<VEC>(w, x, (uint32_t)(e0 + v * VEC), hot, K, lane);
+      for (int u = 0; u < TK_UNROLL; ++u) {
+        const int v = it + u * TK_THREADS + tid;
+        float x[VEC];
+        Vec<T>::unpack(raw[u], x);
+        warp_offer<VEC>(w, x, (uint32_t)(e0 + v * VEC), v < v_end, w.thr_val, K, lane);
+      }
+      if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr_val));
     }
   }
   warp_flush(w, K, lane);
@@ -245,6 +297,12 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   float ws = (m == -INFINITY) ? 0.f : s * ex2((m - wm) * LOG2E);
   ws = warp_sum(ws);
   if (lane == 0) { s_m[warp] = wm; s_s[warp] = ws; }
+  // CTA top-K over the warps' lists: gather them, rank-count with all threads
+  for (int i = tid; i < TK_WARPS * LILICORR_MAX_K; i += TK_THREADS)
+    s_merge[i] = s_keys[i / LILICORR_MAX_K][i % LILICORR_MAX_K];
+  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
+  __syncthreads();
+  rank_place(s_merge, TK_WARPS * LILICORR_MAX_K, K, s_top, tid, TK_THREADS);
   __syncthreads();
 
   float cm = -INFINITY, cs = 0.f;
@@ -254,27 +312,18 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
     cm = warp_max(pm);
     cs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - cm) * LOG2E));
   }
-  // CTA top-K over the warps' lists (list entries >= K are zero)
-  uint64_t mine = 0ull;
-  if (warp == 0) {
-    // gather the warp lists into s_merge so the selection reads only list entries
-    for (int i = lane; i < TK_WARPS * LILICORR_MAX_K; i += 32)
-      s_merge[i] = s_keys[i / LILICORR_MAX_K][i % LILICORR_MAX_K];
-    __syncwarp();
-    mine = warp_select(s_merge, TK_WARPS * LILICORR_MAX_K, K, lane);
-  }
 
   if (splits == 1) {
     if (warp == 0) {
       const float l = cm + logf(cs);
-      const bool bad = !(isfinite(l));
       if (lane == 0) {
         lse[row] = l;
-        if (bad) set_status(status, LILICORR_ERR_NONFINITE);
+        if (!isfinite(l)) set_status(status, LILICORR_ERR_NONFINITE);
       }
       if (lane < K) {
-        ids[(size_t)row * K + lane] = key_id(mine);
-        logp[(size_t)row * K + lane] = key_value(mine) - l;
+        const uint64_t k = s_top[lane];
+        ids[(size_t)row * K + lane] = key_id(k);
+        logp[(size_t)row * K + lane] = key_value(k) - l;
       }
     }
     return;
@@ -284,7 +333,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   Rec* rec = reinterpret_cast<Rec*>(partials + ((size_t)row * splits + split) * rec_bytes);
   if (warp == 0) {
     if (lane == 0) { rec->m = cm; rec->s = cs; }
-    if (lane < K) rec->keys[lane] = mine;
+    if (lane < K) rec->keys[lane] = s_top[lane];
     __threadfence();
   }
   __syncthreads();
@@ -297,10 +346,14 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   __threadfence();
 
   // last CTA of the row: merge all splits
-  for (int i = tid; i < splits * K; i += TK_THREADS) {
+  const int n = splits * K;
+  for (int i = tid; i < n; i += TK_THREADS) {
     const Rec* r = reinterpret_cast<const Rec*>(partials + ((size_t)row * splits + i / K) * rec_bytes);
     s_merge[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
   }
+  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
+  __syncthreads();
+  rank_place(s_merge, n, K, s_top, tid, TK_THREADS);
   __syncthreads();
   if (warp == 0) {
     float pm = -INFINITY, ps = 0.f;
@@ -313,7 +366,6 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
     }
     const float gm = warp_max(pm);
     const float gs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - gm) * LOG2E));
-    const uint64_t top = warp_select(s_merge, splits * K, K, lane);
     const float l = gm + logf(gs);
     if (lane == 0) {
       lse[row] = l;
@@ -321,8 +373,9 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       counters[row] = 0u;             // leave the workspace reusable
     }
     if (lane < K) {
-      ids[(size_t)row * K + lane] = key_id(top);
-      logp[(size_t)row * K + lane] = key_value(top) - l;
+      const uint64_t k = s_top[lane];
+      ids[(size_t)row * K + lane] = key_id(k);
+      logp[(size_t)row * K + lane] = key_value(k) - l;
     }
   }
 }
@@ -332,11 +385,13 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
 TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   const int vec = dt == LILICORR_BF16 ? 8 : 4;
   const int nvec = V / vec;
-  const int target_ctas = num_sms() * 4;
-  const int min_chunk = 512;                 // vectors (8 KB) per CTA at least
+  // about two waves of resident CTAs (4 per SM) when rows are many, one when few
+  const int slots = num_sms() * 4;
+  const int target_ctas = rows >= slots ? 2 * slots : slots;
+  const int min_chunk = 256;                 // vectors (4 KB) per CTA at least
   int splits = ceil_div(target_ctas, rows);
   splits = max(1, min(splits, ceil_div(max(nvec, 1), min_chunk)));
-  splits = min(splits, TK_MAX_SPLITS);
+  splits = min(splits, min(TK_MAX_SPLITS, TK_MERGE_MAX / K));
   TopkPlan p;
   p.splits = splits;
   p.chunk_vecs = ceil_div(max(nvec, 1), splits);

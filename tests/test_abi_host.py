@@ -10,7 +10,7 @@ import pytest
 import oracle
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADER = os.path.join(ROOT, "include", "lilicorr.h")
+HEADERS = [os.path.join(ROOT, "include", h) for h in ("lilicorr.h", "lilicorr_testing.h")]
 
 
 @pytest.fixture(scope="module")
@@ -22,7 +22,7 @@ def lib():
 
 
 def declared_functions():
-    src = open(HEADER).read()
+    src = "".join(open(h).read() for h in HEADERS)
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     return sorted(set(re.findall(r"\b(lilicorr_[a-z_0-9]+)\s*\(", src)))
 

@@ -1,0 +1,66 @@
+"""GPU check of the scoring network's linear-layer kernels (building blocks of step 2)
+against a plain PyTorch fp32 matmul of the same bf16/fp32 operands: the tensor-core
+(tcgen05) kernel, the tiled and the few-row CUDA-core kernels, with bias, SiLU,
+residual, bf16 output, ragged M/N and long Kd."""
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+def _ll():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2608_20530_gb300 as ll
+    return ll
+
+
+def _ref(A, W, bias, residual, act):
+    y = A.float() @ W.float().T
+    if bias is not None:
+        y = y + bias
+    if act == 1:
+        y = torch.nn.functional.silu(y)
+    if residual is not None:
+        y = y + residual
+    return y
+
+
+CASES = [  # M, N, Kd
+    (128, 256, 256), (128, 64, 64), (300, 768, 256), (129, 64, 4096), (512, 512, 4096),
+    (256, 1536, 512), (1000, 200, 512), (4096, 512, 512), (16, 256, 4096), (1, 256, 256),
+    (64, 1024, 2048),
+]
+
+
+@pytest.mark.parametrize("M,N,Kd", CASES)
+@pytest.mark.parametrize("path", [0, 1, 2, 3])
+def test_linear_paths(M, N, Kd, path):
+    ll = _ll()
+    if path == 2 and M > 64:
+        pytest.skip("few-row kernel serves M <= 64")
+    g = torch.Generator(device="cuda").manual_seed(M * 7 + N + Kd)
+    A = torch.randn((M, Kd), generator=g, device="cuda").to(torch.bfloat16)
+    W = (0.02 * torch.randn((N, Kd), generator=g, device="cuda")).to(torch.bfloat16)
+    bias = 0.1 * torch.randn(N, generator=g, device="cuda")
+    res = torch.randn((M, N), generator=g, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for act, b, r, odt in [(0, None, None, torch.float32), (1, bias, None, torch.float32),
+                           (0, bias, res, torch.float32), (1, bias, None, torch.bfloat16)]:
+        C = ll.test_linear(A, W, odt, bias=b, residual=r, act=act, path=path, status=status)
+        torch.cuda.synchronize()
+        want = _ref(A, W, b, r, act)
+        tol = 2e-2 if odt == torch.bfloat16 else 2e-4 * max(1.0, (Kd / 256) ** 0.5)
+        err = (C.float() - want).abs().max().item()
+        assert err <= tol * max(1.0, want.abs().max().item()), (path, act, odt, err)
+    assert int(status.item()) == 0
+
+
+def test_linear_fp32_operands_use_cuda_cores():
+    ll = _ll()
+    A = torch.randn((200, 96), device="cuda")
+    W = torch.randn((72, 96), device="cuda")
+    with pytest.raises(ll.LilicorrError):
+        ll.test_linear(A, W, path=3)
+    C = ll.test_linear(A, W, path=0)
+    assert (C - A @ W.T).abs().max().item() < 1e-4

