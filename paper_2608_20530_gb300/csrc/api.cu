@@ -202,104 +202,141 @@ lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
   return launch_gemm_simt(g, st);
 }
 
-// The scoring network (Sec. 3.2; App. A) over B sequences: writes oi = [W_o u + b_o |
-// W_i u + b_i] (not yet normalised) at ws.oi and the unit anchor vector at ws.anc.
-lilicorr_status_t run_head(const lilicorr_head* h, int B, const int32_t* ids, const float* logp,
-                           const void* hidden, const void* target, void* ws, const WsLayout& w,
-                           cudaStream_t st) {
-  const lilicorr_head_desc& d = h->desc;
-  const lilicorr_dtype_t wdt = d.dtype;
-  const lilicorr_dtype_t adt = d.dtype;     // matrix-product operands: bf16 on the bf16 head
-  const lilicorr_dtype_t F32 = LILICORR_F32;
-  const int R = B * d.L, N = R * d.K, LK = d.L * d.K;
-  const int D = d.D, F = d.ffn;
-  uint32_t* status = at<uint32_t>(ws, w.status);
-  float* hproj = at<float>(ws, w.hproj);
-  float* tn = at<float>(ws, w.tn);
-  float* t = at<float>(ws, w.t);
-  float* anc = at<float>(ws, w.anc);
-  float* cb = at<float>(ws, w.cb);
-  float* x = at<float>(ws, w.x);
-  void* c1 = at<void>(ws, w.c1);
-  void* xn = at<void>(ws, w.xn);
-  void* qkv = at<void>(ws, w.qkv);
-  const int hd = D / d.n_heads;
-  const bool tc_attn = wdt == LILICORR_BF16 && attention_tc_supported(hd) &&
-                       attention_tc_smem_bytes(LK, hd, d.L) <= 200 * 1024;
-  const lilicorr_dtype_t qkv_dt = tc_attn ? LILICORR_BF16 : F32;
-  void* att = at<void>(ws, w.att);
-  void* hf = at<void>(ws, w.hf);
-  void* u = at<void>(ws, w.u);
-  float* oi = at<float>(ws, w.oi);
-  auto G = [&](const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, int ldw, void* C,
-               lilicorr_dtype_t c_dt, int ldc, int M, int Nn, int Kd) {
+// Views of one call's workspace buffers and the per-call kernel choices.
+struct HeadCall {
+  const lilicorr_head* h;
+  const lilicorr_head_desc& d;
+  int B, R, N, LK, D, F;
+  lilicorr_dtype_t wdt, adt, qkv_dt;     // weights; matrix-product operands; q|k|v buffer
+  bool tc_attn;                          // tensor-core attention core
+  uint32_t* status;
+  float *hproj, *tn, *t, *anc, *cb, *x, *oi;
+  void *c1, *xn, *qkv, *att, *hf, *u;
+
+  HeadCall(const lilicorr_head* head, int b, void* ws, const WsLayout& w)
+      : h(head), d(head->desc), B(b) {
+    R = B * d.L;
+    N = R * d.K;
+    LK = d.L * d.K;
+    D = d.D;
+    F = d.ffn;
+    wdt = d.dtype;
+    adt = d.dtype;                       // bf16 operands on the bf16 head
+    const int hd = D / d.n_heads;
+    tc_attn = wdt == LILICORR_BF16 && attention_tc_supported(hd) &&
+              attention_tc_smem_bytes(LK, hd, d.L) <= 200 * 1024;
+    qkv_dt = tc_attn ? LILICORR_BF16 : LILICORR_F32;
+    status = at<uint32_t>(ws, w.status);
+    hproj = at<float>(ws, w.hproj);
+    tn = at<float>(ws, w.tn);
+    t = at<float>(ws, w.t);
+    anc = at<float>(ws, w.anc);
+    cb = at<float>(ws, w.cb);
+    x = at<float>(ws, w.x);
+    oi = at<float>(ws, w.oi);
+    c1 = at<void>(ws, w.c1);
+    xn = at<void>(ws, w.xn);
+    qkv = at<void>(ws, w.qkv);
+    att = at<void>(ws, w.att);
+    hf = at<void>(ws, w.hf);
+    u = at<void>(ws, w.u);
+  }
+  GemmArgs G(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, int ldw, void* C,
+             lilicorr_dtype_t c_dt, int ldc, int M, int Nn, int Kd) const {
     GemmArgs g = gemm(A, a_dt, lda, W, wdt, ldw, C, c_dt, ldc, M, Nn, Kd);
     g.status = status;
     return g;
-  };
+  }
+};
 
+// Candidate-independent part of the scoring network (Sec. 3.2; App. A): the drafter
+// state projection, the target state, the anchor out vector and the fusion layer's t block.
+lilicorr_status_t run_prologue(const HeadCall& c, const void* hidden, const void* target,
+                               cudaStream_t st) {
+  const lilicorr_head* h = c.h;
+  const lilicorr_head_desc& d = c.d;
+  const lilicorr_dtype_t F32 = LILICORR_F32;
+  const int D = c.D;
   // drafter state projection W_h h_s + b_h, one row per slot (shared by its K candidates)
-  GemmArgs g = G(hidden, wdt, d.H, h->hid_w, d.H, hproj, F32, D, R, D, d.H);
+  GemmArgs g = c.G(hidden, c.wdt, d.H, h->hid_w, d.H, c.hproj, F32, D, c.R, D, d.H);
   g.bias = h->hid_b;
   LL_TRY(run_gemm(g, st));
   // target state t = W_t RMSNorm(mean of the captured layers) + b_t
-  LL_TRY(launch_target_norm(target, wdt, B, d.n_tgt, d.H, h->tgt_norm, tn, st));
-  g = G(tn, F32, d.H, h->tgt_w, d.H, t, F32, D, B, D, d.H);
+  LL_TRY(launch_target_norm(target, c.wdt, c.B, d.n_tgt, d.H, h->tgt_norm, c.tn, st));
+  g = c.G(c.tn, F32, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
   g.bias = h->tgt_b;
   LL_TRY(run_gemm(g, st));
   // anchor out vector o_0 = unit(W_a t + b_a)
-  g = G(t, F32, D, h->anc_w, D, anc, F32, d.d, B, d.d, D);
+  g = c.G(c.t, F32, D, h->anc_w, D, c.anc, F32, d.d, c.B, d.d, D);
   g.bias = h->anc_b;
   LL_TRY(run_gemm(g, st));
-  LL_TRY(launch_unit_rows(anc, B, d.d, d.d, anc, d.d, st));
+  LL_TRY(launch_unit_rows(c.anc, c.B, d.d, d.d, c.anc, d.d, st));
   // the t block of the fusion layer is constant per sequence: cb = W_f[:, t] t + b_f
-  g = G(t, F32, D, h->fuse_t, D, cb, F32, D, B, D, D);
+  g = c.G(c.t, F32, D, h->fuse_t, D, c.cb, F32, D, c.B, D, D);
   g.bias = h->fuse_b;
-  LL_TRY(run_gemm(g, st));
+  return run_gemm(g, st);
+}
+
+// Candidate-dependent part, after run_prologue: nodes, the Transformer, fusion and the
+// out/in heads. Writes oi = [W_o u + b_o | W_i u + b_i] (not yet normalised).
+lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* logp,
+                           cudaStream_t st) {
+  const lilicorr_head* h = c.h;
+  const lilicorr_head_desc& d = c.d;
+  const lilicorr_dtype_t F32 = LILICORR_F32, adt = c.adt;
+  const int D = c.D, F = c.F, N = c.N;
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
-  LL_TRY(launch_node_build(h, B, ids, logp, hproj, c1, adt, x, status, st));
-  g = G(c1, adt, D, h->conf2_w, D, x, F32, D, N, D, D);
+  LL_TRY(launch_node_build(h, c.B, ids, logp, c.hproj, c.c1, adt, c.x, c.status, st));
+  GemmArgs g = c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D);
   g.bias = h->conf2_b;
-  g.residual = x; g.ldr = D;
+  g.residual = c.x; g.ldr = D;
   LL_TRY(run_gemm(g, st));
   // Transformer layers
   for (int i = 0; i < d.n_layers; ++i) {
     const HeadW& l = h->layer[i];
-    LL_TRY(launch_rmsnorm(x, N, D, l.an, xn, adt, st));
-    g = G(xn, adt, D, l.wqkv, D, qkv, qkv_dt, 3 * D, N, 3 * D, D);
+    LL_TRY(launch_rmsnorm(c.x, N, D, l.an, c.xn, adt, st));
+    g = c.G(c.xn, adt, D, l.wqkv, D, c.qkv, c.qkv_dt, 3 * D, N, 3 * D, D);
     g.bias = l.bqkv;
     LL_TRY(run_gemm(g, st));
-    if (tc_attn)
-      LL_TRY(launch_attention_tc(qkv, B, d.L, d.K, D, d.n_heads, l.dist, l.same, att, st));
+    if (c.tc_attn)
+      LL_TRY(launch_attention_tc(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att, st));
     else
-      LL_TRY(launch_attention(static_cast<const float*>(qkv), B, d.L, d.K, D, d.n_heads, l.dist,
-                              l.same, att, adt, st));
-    g = G(att, adt, D, l.wo, D, x, F32, D, N, D, D);
+      LL_TRY(launch_attention(static_cast<const float*>(c.qkv), c.B, d.L, d.K, D, d.n_heads,
+                              l.dist, l.same, c.att, adt, st));
+    g = c.G(c.att, adt, D, l.wo, D, c.x, F32, D, N, D, D);
     g.bias = l.bo;
-    g.residual = x; g.ldr = D;
+    g.residual = c.x; g.ldr = D;
     LL_TRY(run_gemm(g, st));
-    LL_TRY(launch_rmsnorm(x, N, D, l.fn, xn, adt, st));
-    g = G(xn, adt, D, l.w1, D, hf, adt, F, N, F, D);
+    LL_TRY(launch_rmsnorm(c.x, N, D, l.fn, c.xn, adt, st));
+    g = c.G(c.xn, adt, D, l.w1, D, c.hf, adt, F, N, F, D);
     g.bias = l.b1;
     g.act = ACT_SILU;
     LL_TRY(run_gemm(g, st));
-    g = G(hf, adt, F, l.w2, F, x, F32, D, N, D, F);
+    g = c.G(c.hf, adt, F, l.w2, F, c.x, F32, D, N, D, F);
     g.bias = l.b2;
-    g.residual = x; g.ldr = D;
+    g.residual = c.x; g.ldr = D;
     LL_TRY(run_gemm(g, st));
   }
   // fusion u = SiLU(W_f [x; t; x*t] + b_f) with x the final-normed state
-  LL_TRY(launch_fusion_input(x, B, LK, D, h->final_norm, t, xn, adt, st));
-  g = G(xn, adt, 2 * D, h->fuse_x, 2 * D, u, adt, D, N, D, 2 * D);
-  g.bias_rows = cb;
-  g.rows_per_bias = LK;
+  LL_TRY(launch_fusion_input(c.x, c.B, c.LK, D, h->final_norm, c.t, c.xn, adt, st));
+  g = c.G(c.xn, adt, 2 * D, h->fuse_x, 2 * D, c.u, adt, D, N, D, 2 * D);
+  g.bias_rows = c.cb;
+  g.rows_per_bias = c.LK;
   g.act = ACT_SILU;
   LL_TRY(run_gemm(g, st));
   // out and in heads in one product: oi = [W_o u + b_o | W_i u + b_i]
-  g = G(u, adt, D, h->woi, D, oi, F32, 2 * d.d, N, 2 * d.d, D);
+  g = c.G(c.u, adt, D, h->woi, D, c.oi, F32, 2 * d.d, N, 2 * d.d, D);
   g.bias = h->boi;
-  LL_TRY(run_gemm(g, st));
-  return LILICORR_OK;
+  return run_gemm(g, st);
+}
+
+// The whole scoring network on one stream.
+lilicorr_status_t run_head(const lilicorr_head* h, int B, const int32_t* ids, const float* logp,
+                           const void* hidden, const void* target, void* ws, const WsLayout& w,
+                           cudaStream_t st) {
+  const HeadCall c(h, B, ws, w);
+  LL_TRY(run_prologue(c, hidden, target, st));
+  return run_body(c, ids, logp, st);
 }
 
 }  // namespace
@@ -400,11 +437,19 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
   cudaGetDevice(&h->device);
   void* embed_dev = nullptr;
   auto fail = [&](lilicorr_status_t s) {
+    (void)cudaGetLastError();
     if (embed_dev) cudaFree(embed_dev);
     if (h->pool) cudaFree(h->pool);
+    if (h->side) cudaStreamDestroy(h->side);
+    if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+    if (h->ev_join) cudaEventDestroy(h->ev_join);
     free(h);
     return s;
   };
+  if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess)
+    return fail(LILICORR_ERR_CUDA);
   if (cudaMalloc(&h->pool, pool_bytes) != cudaSuccess) return fail(LILICORR_ERR_CUDA);
   h->pool_bytes = pool_bytes;
   // the fold region is written on the device; copy everything after it
@@ -456,6 +501,9 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   cudaGetDevice(&cur);
   if (cur != h->device) cudaSetDevice(h->device);
   cudaError_t e = cudaFree(h->pool);
+  if (h->side) cudaStreamDestroy(h->side);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
   if (cur != h->device) cudaSetDevice(cur);
   free(h);
   return e == cudaSuccess ? LILICORR_OK : LILICORR_ERR_CUDA;
@@ -574,10 +622,19 @@ lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const 
   const int R = B * d.L;
   int32_t* ids = at<int32_t>(ws, w.ids);
   float* logp = at<float>(ws, w.logp);
+  // the candidate-independent projections run beside the top-K pass
+  lilicorr_head* hm = const_cast<lilicorr_head*>(head);
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_fork, stream));
+  LL_CUDA_TRY(cudaStreamWaitEvent(hm->side, hm->ev_fork, 0));
+  const HeadCall call(head, B, ws, w);
+  const lilicorr_status_t sp = run_prologue(call, drafter_hidden, target_hidden, hm->side);
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_join, hm->side));     // always rejoin, even on error
+  LL_TRY(sp);
   LL_TRY(launch_topk_lse(logits, d.dtype, R, d.V, d.K, ids, logp, at<float>(ws, w.lse),
                          at<uint32_t>(ws, w.status), at<uint32_t>(ws, w.counters),
                          at<void>(ws, w.partials), stream));
-  LL_TRY(run_head(head, B, ids, logp, drafter_hidden, target_hidden, ws, w, stream));
+  LL_CUDA_TRY(cudaStreamWaitEvent(stream, hm->ev_join, 0));
+  LL_TRY(run_body(call, ids, logp, stream));
   PairWalkArgs a;
   memset(&a, 0, sizeof(a));
   a.B = B; a.L = d.L; a.K = d.K; a.d = d.d;

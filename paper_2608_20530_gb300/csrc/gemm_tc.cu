@@ -211,13 +211,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   }
   __syncwarp();
 
-  // ---- epilogue: TMEM -> registers -> shared (transpose) -> global, row segments
+  // ---- epilogue: TMEM -> registers -> shared (transpose) -> global, row segments.
+  // Lane l of warp w owns column (c0 + l) of rows 32w..32w+31 of each 32-column chunk;
+  // the chunk's residual values are loaded before they are needed, all 32 in flight
+  // (the first chunk's while the tensor cores are still busy).
+  const int mrow0 = m0 + warp * 32;
+  float res[32];
+  auto load_residual = [&](int c0) {
+    const int n = n0 + c0 + lane;
+#pragma unroll
+    for (int rr = 0; rr < 32; ++rr)
+      res[rr] = (ep.residual && n < N && mrow0 + rr < M)
+                    ? ep.residual[(size_t)(mrow0 + rr) * ep.ldr + n] : 0.f;
+  };
+  load_residual(0);
   if (!mbar_wait(&done, 0, WAIT_LIMIT_NS)) atomicExch(&abort_flag, 1);
   tc_fence_after();
   __syncthreads();                         // the stage ring is drained: reuse it below
   if (!abort_flag) {
     float* tile = reinterpret_cast<float*>(smem) + warp * 32 * 33;   // this warp's 32 x 32
-    const int mrow0 = m0 + warp * 32;
 #pragma unroll 1
     for (int c0 = 0; c0 < BN; c0 += 32) {
       uint32_t r[32];
@@ -225,23 +237,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 #pragma unroll
       for (int j = 0; j < 32; ++j) tile[lane * 33 + j] = __uint_as_float(r[j]);
       __syncwarp();
-      const int n = n0 + c0 + lane;          // this lane's column; rows go one by one
+      const int n = n0 + c0 + lane;
       if (n < N) {
         const float bn = ep.bias ? ep.bias[n] : 0.f;
-#pragma unroll 4
+#pragma unroll
         for (int rr = 0; rr < 32; ++rr) {
           const int m = mrow0 + rr;
-          if (m >= M) break;
-          float v = tile[rr * 33 + lane] + bn;
-          if (ep.bias_rows) v += ep.bias_rows[(size_t)(m / ep.rows_per_bias) * N + n];
-          if (ep.act == ACT_SILU) v = silu_f(v);
-          if (ep.residual) v += ep.residual[(size_t)m * ep.ldr + n];
-          if (ep.c_bf16)
-            static_cast<__nv_bfloat16*>(ep.C)[(size_t)m * ep.ldc + n] = __float2bfloat16_rn(v);
-          else
-            static_cast<float*>(ep.C)[(size_t)m * ep.ldc + n] = v;
+          if (m < M) {
+            float v = tile[rr * 33 + lane] + bn;
+            if (ep.bias_rows) v += ep.bias_rows[(size_t)(m / ep.rows_per_bias) * N + n];
+            if (ep.act == ACT_SILU) v = silu_f(v);
+            v += res[rr];
+            if (ep.c_bf16)
+              static_cast<__nv_bfloat16*>(ep.C)[(size_t)m * ep.ldc + n] = __float2bfloat16_rn(v);
+            else
+              static_cast<float*>(ep.C)[(size_t)m * ep.ldc + n] = v;
+          }
         }
       }
+      if (c0 + 32 < BN) load_residual(c0 + 32);
       __syncwarp();
     }
   }

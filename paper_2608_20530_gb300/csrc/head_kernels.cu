@@ -132,16 +132,21 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
 #pragma unroll
         for (int e = 0; e < 8; ++e) w[j][e] = 0.f;
     }
+    // all row loads first (predicated, no early exit) so they are in flight together
+    float a[SK_MB][8];
 #pragma unroll
     for (int i = 0; i < SK_MB; ++i) {
-      if (i >= mb) break;
-      float a[8];
-      load8(A + (size_t)(m0 + i) * g.lda + k, a);
+      if (i < mb) load8(A + (size_t)(m0 + i) * g.lda + k, a[i]);
+      else
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[i][e] = 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < SK_MB; ++i)
 #pragma unroll
       for (int j = 0; j < SK_NB; ++j)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[i][j] = fmaf(a[e], w[j][e], acc[i][j]);
-    }
+        for (int e = 0; e < 8; ++e) acc[i][j] = fmaf(a[i][e], w[j][e], acc[i][j]);
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 #pragma unroll

@@ -115,6 +115,10 @@ struct HeadW {          // device pointers of one Transformer layer
 struct lilicorr_head {
   lilicorr_head_desc desc;
   int device;
+  // the projections that do not depend on the top-K pass run on a side stream that
+  // forks from and joins the caller's stream (a fork/join under graph capture)
+  cudaStream_t side;
+  cudaEvent_t ev_fork, ev_join;
   void* pool;                 // one device allocation holding everything below
   size_t pool_bytes;
   // matrices in head dtype; vectors and tables in fp32

@@ -6,15 +6,15 @@
 //   * grid = (splits, rows): each CTA streams one contiguous chunk of one row with
 //     16-byte loads, a batch of 4 per thread in flight;
 //   * every thread keeps an online (max, sum exp) pair, merged by warp shuffles;
-//   * candidates are kept as order-preserving 64-bit keys (value, then lower id
-//     first). The hot loop costs one compare per batch: a warp looks at a batch
-//     only if some lane's batch maximum reaches the threshold, the larger of the
-//     warp's own K-th value and the CTA's (shared memory; every warp's K-th value
-//     bounds the CTA's K-th from below). On such a batch the warp first raises the
-//     threshold to the K-th largest lane maximum (each lane maximum is a distinct
-//     element, so at least K elements reach it), then appends the elements that
-//     pass to a per-warp buffer, one ballot round per hot element of the busiest
-//     lane. A full buffer is merged into the warp's list by rank counting;
+//   * candidates are order-preserving 64-bit keys (value, then lower id first); each
+//     warp keeps its top-K as a sorted list in registers (lane i holds the i-th key).
+//     The hot loop costs one compare per batch: a warp looks at a batch only if some
+//     lane's batch maximum reaches the threshold, the larger of the warp's own K-th
+//     value and the CTA's (shared memory; every warp's K-th value bounds the CTA's
+//     K-th from below). While its list is not full, a warp raises the threshold to
+//     the K-th largest lane maximum of the batch (each lane maximum is a distinct
+//     element, so K elements reach it). Elements that pass are inserted one at a
+//     time with a ballot (position) and a shuffle (shift);
 //   * the CTA merges its warps' lists by rank counting; with several splits per
 //     row the last CTA to finish (atomic ticket, no waiting) merges the splits'
 //     partial (max, sum, top-K) records and writes ids, logp and lse.
@@ -26,7 +26,6 @@ namespace {
 
 constexpr int TK_THREADS = 256;
 constexpr int TK_WARPS = TK_THREADS / 32;
-constexpr int TK_CAP = 64;             // candidate buffer per warp
 constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch
 constexpr int TK_MAX_SPLITS = 64;
 constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
@@ -75,6 +74,38 @@ __device__ __forceinline__ void rank_place(const uint64_t* keys, int n, int K, u
     for (int j = 0; j < n; ++j) rank += keys[j] > c ? 1 : 0;
     if (rank < K) out[rank] = c;
   }
+}
+
+// K largest of groups[g][0..K) for g < ngroups (each group sorted descending, zeros =
+// empty), CTA-wide. Every group's K-th key bounds the answer's K-th from below, so only
+// keys >= the largest such bound survive; they are compacted and rank-counted.
+// surv: scratch of TK_MERGE_MAX keys; out[0..K) receives the result. All threads call.
+__device__ void cta_select(const uint64_t* groups, int ngroups, int stride, int K, uint64_t* surv,
+                           int* s_count, uint64_t* s_bound, uint64_t* out) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (warp == 0) {
+    uint64_t b = 0ull;
+    for (int g = lane; g < ngroups; g += 32) {
+      const uint64_t k = groups[(size_t)g * stride + K - 1];
+      b = k > b ? k : b;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const uint64_t x = __shfl_xor_sync(FULL, b, o);
+      b = x > b ? x : b;
+    }
+    if (lane == 0) { *s_bound = b; *s_count = 0; }
+  }
+  for (int i = tid; i < K; i += TK_THREADS) out[i] = 0ull;
+  __syncthreads();
+  const uint64_t bound = *s_bound;
+  for (int i = tid; i < ngroups * K; i += TK_THREADS) {
+    const uint64_t k = groups[(size_t)(i / K) * stride + i % K];
+    if (k != 0ull && k >= bound) surv[atomicAdd(s_count, 1)] = k;
+  }
+  __syncthreads();
+  rank_place(surv, *s_count, K, out, tid, TK_THREADS);
+  __syncthreads();
 }
 
 template <int N>
@@ -135,55 +166,28 @@ __device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
   return __shfl_sync(FULL, v, K - 1);
 }
 
-struct WarpTopK {
-  uint64_t* list;      // [LILICORR_MAX_K] descending, 0 = empty
-  uint64_t* buf;       // [TK_CAP]; list and buf contiguous (list first)
-  uint64_t* tmp;       // [LILICORR_MAX_K] scratch of the merge
-  uint32_t* cta_thr;   // CTA-wide threshold (order image), shared by the warps
-  int nbuf;
-  uint64_t thr;        // K-th key of the list (0 while not full)
-  float thr_val;       // value threshold of this warp (never decreases)
+// A warp's running top-K as a sorted list in registers: lane i holds the i-th largest
+// key (0 = empty; lanes >= K hold 0). Candidates are rare and inserted one at a time.
+struct WarpList {
+  uint64_t mine;       // this lane's entry
+  uint64_t thr;        // the K-th key (0 while not full)
+  float thr_val;       // value bound below which nothing can enter (never decreases)
 };
 
-// Merge the buffer into the list (rank counting over list + buffer) and raise the
-// thresholds. Warp-collective.
-__device__ __forceinline__ void warp_flush(WarpTopK& w, int K, int lane) {
-  __syncwarp();
-  const int n = LILICORR_MAX_K + w.nbuf;
-  if (lane < K) w.tmp[lane] = 0ull;
-  __syncwarp();
-  rank_place(w.list, n, K, w.tmp, lane, 32);
-  __syncwarp();
-  uint64_t mine = lane < K ? w.tmp[lane] : 0ull;
-  if (lane < LILICORR_MAX_K) w.list[lane] = mine;
-  w.thr = __shfl_sync(FULL, mine, K - 1);
-  if (w.thr) {
-    w.thr_val = fmaxf(w.thr_val, key_value(w.thr));
-    if (lane == 0) atomicMax(w.cta_thr, ord32(w.thr_val));
-  }
-  w.nbuf = 0;
-  __syncwarp();
+// Insert key c (the same in every lane, c > w.thr). Warp-collective.
+__device__ __forceinline__ void list_insert(WarpList& w, uint64_t c, int K, int lane) {
+  const int pos = __popc(__ballot_sync(FULL, lane < K && w.mine > c));   // larger entries
+  const uint64_t up = __shfl_up_sync(FULL, w.mine, 1);
+  if (lane == pos) w.mine = c;
+  else if (lane > pos && lane < K) w.mine = up;
+  w.thr = __shfl_sync(FULL, w.mine, K - 1);
+  if (w.thr) w.thr_val = fmaxf(w.thr_val, key_value(w.thr));
 }
 
-// Append x (id) to the warp buffer if `c`; warp-collective. Flushes when full.
-__device__ __forceinline__ void warp_append(WarpTopK& w, float x, uint32_t id, bool c, int K,
-                                            int lane) {
-  uint64_t key = make_key(x, id);
-  unsigned m = __ballot_sync(FULL, c && key > w.thr);
-  if (m == 0u) return;
-  if (w.nbuf + __popc(m) > TK_CAP) {
-    warp_flush(w, K, lane);
-    m = __ballot_sync(FULL, c && x >= w.thr_val && key > w.thr);
-    if (m == 0u) return;
-  }
-  if ((m >> lane) & 1u) w.buf[w.nbuf + __popc(m & ((1u << lane) - 1u))] = key;
-  w.nbuf += __popc(m);
-}
-
-// Offer the elements of one vector that reach thr: one ballot round per hot element
-// of the busiest lane. Warp-collective.
+// Offer this lane's N values (ids id0 + j) that reach `thr`. Warp-collective: one round
+// per hot element of the busiest lane; each round's candidates are inserted in turn.
 template <int N>
-__device__ __forceinline__ void warp_offer(WarpTopK& w, const float (&x)[N], uint32_t id0,
+__device__ __forceinline__ void warp_offer(WarpList& w, const float (&x)[N], uint32_t id0,
                                            bool valid, float thr, int K, int lane) {
   uint32_t hm = 0u;
 #pragma unroll
@@ -195,7 +199,14 @@ __device__ __forceinline__ void warp_offer(WarpTopK& w, const float (&x)[N], uin
     float xv = x[0];
 #pragma unroll
     for (int t = 1; t < N; ++t) xv = (j == t) ? x[t] : xv;
-    warp_append(w, xv, id0 + (uint32_t)j, has, K, lane);
+    const uint64_t key = make_key(xv, id0 + (uint32_t)j);
+    unsigned mk = __ballot_sync(FULL, has && key > w.thr);
+    while (mk) {
+      const int src = __ffs(mk) - 1;
+      mk &= mk - 1u;
+      const uint64_t c = __shfl_sync(FULL, key, src);
+      if (c > w.thr) list_insert(w, c, K, lane);     // w.thr rises as the list fills
+    }
   }
 }
 
@@ -205,19 +216,19 @@ struct Rec {            // partial record of one (row, split)
 };
 
 template <typename T>
-__global__ void __launch_bounds__(TK_THREADS)
+__global__ void __launch_bounds__(TK_THREADS, 4)
 topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chunk_vecs,
                 size_t rec_bytes, int32_t* __restrict__ ids, float* __restrict__ logp,
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
                 unsigned char* partials) {
   constexpr int VEC = Vec<T>::N;
-  __shared__ uint64_t s_keys[TK_WARPS][LILICORR_MAX_K + TK_CAP];
-  __shared__ uint64_t s_tmp[TK_WARPS][LILICORR_MAX_K];
+  __shared__ uint64_t s_keys[TK_MERGE_MAX];     // the warps' lists, later the splits' lists
   __shared__ uint64_t s_merge[TK_MERGE_MAX];
   __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ float s_m[TK_WARPS], s_s[TK_WARPS];
-  __shared__ uint32_t s_cta_thr;
-  __shared__ int s_last;
+  __shared__ uint32_t s_cta_thr;                // CTA-wide value bound (order image)
+  __shared__ int s_last, s_count;
+  __shared__ uint64_t s_bound;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int split = blockIdx.x;
@@ -231,15 +242,10 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   const int v_begin = min(split * chunk_vecs, nvec);
   const int v_end = min(v_begin + chunk_vecs, nvec);
 
-  WarpTopK w;
-  w.list = s_keys[warp];
-  w.buf = s_keys[warp] + LILICORR_MAX_K;
-  w.tmp = s_tmp[warp];
-  w.cta_thr = &s_cta_thr;
-  w.nbuf = 0;
+  WarpList w;
+  w.mine = 0ull;
   w.thr = 0ull;
   w.thr_val = -INFINITY;
-  w.list[lane] = 0ull;
   if (tid == 0) s_cta_thr = ord32(-INFINITY);
   __syncthreads();
 
@@ -257,6 +263,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       lse_update<1>(m, s, x, valid);
       warp_offer<1>(w, x, (uint32_t)e, valid, w.thr_val, K, lane);
     }
+    if (lane == 0 && w.thr) atomicMax(&s_cta_thr, ord32(w.thr_val));
   }
 
   // main stream: batches of TK_UNROLL 16-byte vectors per thread
@@ -268,20 +275,24 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       const int v = it + u * TK_THREADS + tid;
       raw[u] = v < v_end ? __ldcs(vp + v) : make_uint4(0, 0, 0, 0);
     }
+    float vmx[TK_UNROLL];                      // this lane's per-vector maxima
     float bmax = -INFINITY;
 #pragma unroll
     for (int u = 0; u < TK_UNROLL; ++u) {
       float x[VEC];
       Vec<T>::unpack(raw[u], x);
-      bmax = fmaxf(bmax, lse_update<VEC>(m, s, x, it + u * TK_THREADS + tid < v_end));
+      vmx[u] = lse_update<VEC>(m, s, x, it + u * TK_THREADS + tid < v_end);
+      bmax = fmaxf(bmax, vmx[u]);
     }
     float thr = fmaxf(w.thr_val, unord32(*(volatile uint32_t*)&s_cta_thr));
     if (__any_sync(FULL, bmax >= thr)) {
-      // raise the bound to the K-th largest lane maximum of this batch
-      thr = fmaxf(thr, warp_kth_largest(bmax, K, lane));
-      w.thr_val = thr;
+      // while the list is not full, raise the bound to the K-th largest lane maximum of
+      // this batch (each lane maximum is a distinct element, so K elements reach it)
+      if (w.thr == 0ull) thr = fmaxf(thr, warp_kth_largest(bmax, K, lane));
+      w.thr_val = fmaxf(w.thr_val, thr);
 #pragma unroll
       for (int u = 0; u < TK_UNROLL; ++u) {
+        if (!__any_sync(FULL, vmx[u] >= w.thr_val)) continue;
         const int v = it + u * TK_THREADS + tid;
         float x[VEC];
         Vec<T>::unpack(raw[u], x);
@@ -290,20 +301,16 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr_val));
     }
   }
-  warp_flush(w, K, lane);
+  s_keys[warp * LILICORR_MAX_K + lane] = w.mine;     // publish the warp's list
 
   // (max, sum) of the warp, then of the CTA
   const float wm = warp_max(m);
   float ws = (m == -INFINITY) ? 0.f : s * ex2((m - wm) * LOG2E);
   ws = warp_sum(ws);
   if (lane == 0) { s_m[warp] = wm; s_s[warp] = ws; }
-  // CTA top-K over the warps' lists: gather them, rank-count with all threads
-  for (int i = tid; i < TK_WARPS * LILICORR_MAX_K; i += TK_THREADS)
-    s_merge[i] = s_keys[i / LILICORR_MAX_K][i % LILICORR_MAX_K];
-  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
+  // CTA top-K over the warps' lists
   __syncthreads();
-  rank_place(s_merge, TK_WARPS * LILICORR_MAX_K, K, s_top, tid, TK_THREADS);
-  __syncthreads();
+  cta_select(s_keys, TK_WARPS, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
 
   float cm = -INFINITY, cs = 0.f;
   if (warp == 0) {
@@ -345,16 +352,14 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   if (!s_last) return;
   __threadfence();
 
-  // last CTA of the row: merge all splits
+  // last CTA of the row: merge all splits (their lists staged in shared memory)
   const int n = splits * K;
   for (int i = tid; i < n; i += TK_THREADS) {
     const Rec* r = reinterpret_cast<const Rec*>(partials + ((size_t)row * splits + i / K) * rec_bytes);
-    s_merge[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
+    s_keys[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
   }
-  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
   __syncthreads();
-  rank_place(s_merge, n, K, s_top, tid, TK_THREADS);
-  __syncthreads();
+  cta_select(s_keys, splits, K, K, s_merge, &s_count, &s_bound, s_top);
   if (warp == 0) {
     float pm = -INFINITY, ps = 0.f;
     for (int i = lane; i < splits; i += 32) {
