@@ -134,6 +134,33 @@ lilicorr_status_t lilicorr_topk_lse(const void* logits, lilicorr_dtype_t dtype, 
                                     int K, int32_t* ids, float* logp, float* lse, void* ws,
                                     size_t ws_bytes, cudaStream_t stream);
 
+/* Step (1) without a caller workspace. Not from the paper (it has no counterpart
+ * there): an addition for callers that cannot allocate device memory at the point
+ * where they select a block. Examples: a serving process whose memory pool has claimed
+ * the free device memory up front, a runtime that forbids allocation after start-up
+ * (cudaMalloc may synchronise the device and fail late), or a plug-in running on a
+ * stream it does not own. It computes what lilicorr_topk_lse computes, same arguments
+ * minus the workspace, but keeps its scratch (status word, per-row tickets, per-split
+ * partial records) in one fixed array of lilicorr_topk_lse_noalloc_max_bytes() = 4 MiB
+ * compiled into the library; every GPU that loads the library holds that array until
+ * the process exits. It calls no cudaMalloc, cudaFree or allocating routine.
+ *   - Sizes whose scratch would exceed the array are rejected with
+ *     LILICORR_ERR_WORKSPACE before anything is enqueued (4 MiB covers, e.g., 4096
+ *     rows of V = 151936 at K = 16; the scratch grows with rows and K).
+ *   - The first call on each device looks up the array's device address (once per
+ *     device, with that device current); make that first call before any stream
+ *     capture.
+ *   - Every call clears the array's status word and tickets on `stream` first (the
+ *     array keeps whatever the previous call left) and then reuses it, so two calls
+ *     that overlap on the GPU (different streams, or different host threads) race
+ *     and give undefined results; order them on one stream.
+ *   - A non-finite row is detected as in lilicorr_topk_lse, but the status word lives
+ *     in the fixed array and is not reported; that row's outputs are undefined. */
+size_t lilicorr_topk_lse_noalloc_max_bytes(void);
+lilicorr_status_t lilicorr_topk_lse_noalloc(const void* logits, lilicorr_dtype_t dtype, int rows,
+                                            int V, int K, int32_t* ids, float* logp, float* lse,
+                                            cudaStream_t stream);
+
 /* Step (2): the scoring network over B sequences' candidates (Sec. 3.2; App. A).
  *   ids, logp         [B, L, K] from step (1) (logp in rank order)
  *   drafter_hidden    [B, L, H] of head dtype, the drafter's state per slot

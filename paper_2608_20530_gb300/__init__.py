@@ -63,6 +63,8 @@ _SIGS = {
     "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
+    "lilicorr_topk_lse_noalloc_max_bytes": (_S, []),
+    "lilicorr_topk_lse_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
     "lilicorr_test_linear": (_I, [_P, _I, _I, _P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I,
                                   _P, _P]),
 }
@@ -239,6 +241,23 @@ def topk_lse(logits: torch.Tensor, K: int, ws: Optional[Workspace] = None):
     _check(lib().lilicorr_topk_lse(logits.data_ptr(), _dtype_code(logits), rows, V, K,
                                    ids.data_ptr(), logp.data_ptr(), lse.data_ptr(), ws.ptr,
                                    ws.nbytes, _stream()), "topk_lse")
+    return ids, logp, lse
+
+
+def topk_lse_noalloc(logits: torch.Tensor, K: int):
+    """topk_lse without a caller workspace: the library's fixed device scratch is used
+    instead (for callers that cannot allocate device memory; see lilicorr.h). Calls that
+    overlap on the GPU race on that scratch."""
+    _dev(logits, "logits")
+    V = logits.shape[-1]
+    rows = logits.numel() // V if V else 0
+    lead = tuple(logits.shape[:-1])
+    ids = torch.empty(lead + (K,), dtype=torch.int32, device=logits.device)
+    logp = torch.empty(lead + (K,), dtype=torch.float32, device=logits.device)
+    lse = torch.empty(lead, dtype=torch.float32, device=logits.device)
+    _check(lib().lilicorr_topk_lse_noalloc(logits.data_ptr(), _dtype_code(logits), rows, V, K,
+                                           ids.data_ptr(), logp.data_ptr(), lse.data_ptr(),
+                                           _stream()), "topk_lse_noalloc")
     return ids, logp, lse
 
 

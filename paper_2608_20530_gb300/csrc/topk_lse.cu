@@ -18,6 +18,8 @@
 //   * the CTA merges its warps' lists by rank counting; with several splits per
 //     row the last CTA to finish (atomic ticket, no waiting) merges the splits'
 //     partial (max, sum, top-K) records and writes ids, logp and lse.
+#include <mutex>
+
 #include "internal.cuh"
 
 namespace lilicorr {
@@ -427,3 +429,70 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
 }
 
 }  // namespace lilicorr
+
+// ----------------------------------------------------------------------------- no-allocation variant
+// Scratch of lilicorr_topk_lse_noalloc: a fixed array in the library's device image, so
+// the call needs no workspace from its caller. Every GPU that loads the library holds it
+// until the process exits.
+namespace lilicorr {
+namespace {
+
+constexpr size_t NOALLOC_SCRATCH_BYTES = 4u << 20;   // 4 MiB
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_SCRATCH_BYTES];
+
+std::mutex g_noalloc_mutex;
+void* g_noalloc_ptr[64] = {};
+
+// Device address of the scratch on the current device. In host code the array's name
+// stands for a host-side shadow, not a device address; cudaGetSymbolAddress (called once
+// per device, with that device current) gives the address the kernel must receive.
+lilicorr_status_t noalloc_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return LILICORR_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= 64) return LILICORR_ERR_ARG;
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+      (void)cudaGetLastError();
+      return LILICORR_ERR_CUDA;
+    }
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return LILICORR_OK;
+}
+
+}  // namespace
+}  // namespace lilicorr
+
+extern "C" size_t lilicorr_topk_lse_noalloc_max_bytes(void) {
+  return lilicorr::NOALLOC_SCRATCH_BYTES;
+}
+
+extern "C" lilicorr_status_t lilicorr_topk_lse_noalloc(const void* logits, lilicorr_dtype_t dtype,
+                                                       int rows, int V, int K, int32_t* ids,
+                                                       float* logp, float* lse,
+                                                       cudaStream_t stream) {
+  using namespace lilicorr;
+  if (dtype != LILICORR_F32 && dtype != LILICORR_BF16) return LILICORR_ERR_DTYPE;
+  if (rows < 0 || V <= 0 || K <= 0 || K > LILICORR_MAX_K || K > V) return LILICORR_ERR_SHAPE;
+  if (rows == 0) return LILICORR_OK;
+  if (!logits || !ids || !logp || !lse) return LILICORR_ERR_ARG;
+  if (!aligned16(logits)) return LILICORR_ERR_ARG;
+  if (topk_ws_bytes(rows, V, K, dtype) > NOALLOC_SCRATCH_BYTES) return LILICORR_ERR_WORKSPACE;
+  void* ws = nullptr;
+  LL_TRY(noalloc_scratch(&ws));
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  // the status word and the per-row tickets must start at zero; the array keeps whatever
+  // the previous call left, so clear them on the caller's stream first
+  const size_t counters_bytes = align_up((size_t)rows * 4, 256);
+  LL_CUDA_TRY(cudaMemsetAsync(w, 0, 256 + counters_bytes, stream));
+  return launch_topk_lse(logits, dtype, rows, V, K, ids, logp, lse,
+                         reinterpret_cast<uint32_t*>(w), reinterpret_cast<uint32_t*>(w + 256),
+                         w + 256 + counters_bytes, stream);
+}
