@@ -139,6 +139,31 @@ class ClockSampler:
                 "samples": len(rows)}
 
 
+def profiled_traffic(kernel_src: str, workload: str):
+    """DRAM bytes per launch of the top-K kernel from the committed ncu summary
+    (profiles/topk_lse_kernel.<workload>.md), or None when that summary is missing or was
+    taken on a different revision of the kernel source."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"topk_lse_kernel.{workload}.md")
+    src = os.path.join(ROOT, "paper_2608_20530_gb300", "csrc", kernel_src)
+    try:
+        text = open(path).read()
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    vals = {}
+    for line in text.splitlines():
+        if ":" in line and line.startswith("- "):
+            k, v = line[2:].split(":", 1)
+            vals[k.strip()] = v.strip().strip("`")
+    if vals.get("kernel source sha256") != digest:
+        return None
+    try:
+        return float(vals["dram bytes per launch"])
+    except (KeyError, ValueError):
+        return None
+
+
 def peaks():
     try:
         return json.load(open(PEAKS_FILE)), "measured"
@@ -363,8 +388,8 @@ def run_ours(args, world, rank, local):
     achieved = alg_bytes / (tk_ms / 1e3) / 1e9
     roofline = {"kernel": "topk_lse_kernel", "bound": "hbm", "achieved": round(achieved, 1),
                 "peak": hbm, "peak_kind": pk_kind, "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                "traffic": None, "alg_bytes_per_launch": alg_bytes,
-                "us_per_launch": round(tk_ms * 1e3, 3)}
+                "traffic": profiled_traffic("topk_lse.cu", wl.name),
+                "alg_bytes_per_launch": alg_bytes, "us_per_launch": round(tk_ms * 1e3, 3)}
 
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,

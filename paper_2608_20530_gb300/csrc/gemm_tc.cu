@@ -11,7 +11,7 @@
 //   * all four warps then read the accumulator back with tcgen05.ld (warp w owns
 //     rows 32w..32w+31) and apply bias / per-sequence bias / SiLU / residual before
 //     storing fp32 or bf16.
-// Every wait is bounded (1 s); on timeout the CTA records LILICORR_ERR_TIMEOUT in
+// Every wait is bounded (about 2 s); on timeout the CTA records LILICORR_ERR_TIMEOUT in
 // the status word, waits (bounded) for its copies in flight, frees its tensor
 // memory and exits.
 #include <cuda.h>
@@ -25,7 +25,7 @@ namespace {
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;                  // 64 bf16 = 128 bytes: one swizzle atom row
 constexpr int TC_THREADS = 128;
-constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;
+constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s at the SM clock
 
 struct TcEpilogue {
   void* C; int ldc; int c_bf16;
@@ -37,11 +37,6 @@ struct TcEpilogue {
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
 }
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
@@ -61,12 +56,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase of parity `parity` to complete; false after `limit_ns`.
-__device__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+// Wait for the phase of parity `parity` to complete; false after `limit` SM cycles
+// (the bound is read from the SM's own cycle counter, which is cheap to poll).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
+  const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity))
-    if (globaltimer() - t0 > limit_ns) return false;
+    if (clock64() - t0 > limit) return false;
   return true;
 }
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
@@ -181,7 +177,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     for (int i = 0; i < nk; ++i) {
       const int s = i % S;
       const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(&empty[s], ph ^ 1u, WAIT_LIMIT_NS)) {
+      if (!mbar_wait(&empty[s], ph ^ 1u, WAIT_LIMIT_CYCLES)) {
         atomicExch(&abort_flag, 1);
         break;
       }
@@ -195,7 +191,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     for (int i = 0; i < nk; ++i) {
       const int s = i % S;
       const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(&full[s], ph, WAIT_LIMIT_NS)) {
+      if (!mbar_wait(&full[s], ph, WAIT_LIMIT_CYCLES)) {
         atomicExch(&abort_flag, 1);
         break;
       }
@@ -225,7 +221,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     ? ep.residual[(size_t)(mrow0 + rr) * ep.ldr + n] : 0.f;
   };
   load_residual(0);
-  if (!mbar_wait(&done, 0, WAIT_LIMIT_NS)) atomicExch(&abort_flag, 1);
+  if (!mbar_wait(&done, 0, WAIT_LIMIT_CYCLES)) atomicExch(&abort_flag, 1);
   tc_fence_after();
   __syncthreads();                         // the stage ring is drained: reuse it below
   if (!abort_flag) {
@@ -269,7 +265,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       // let copies still in flight land before the shared memory is released
       for (int s = 0; s < S && s < nk; ++s) {
         const int last = ((nk - 1 - s) / S) * S + s;
-        mbar_wait(&full[s], (uint32_t)(last / S) & 1u, WAIT_LIMIT_NS / 10);
+        mbar_wait(&full[s], (uint32_t)(last / S) & 1u, WAIT_LIMIT_CYCLES / 10);
       }
     }
     __syncthreads();

@@ -168,46 +168,129 @@ __device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
   return __shfl_sync(FULL, v, K - 1);
 }
 
-// A warp's running top-K as a sorted list in registers: lane i holds the i-th largest
-// key (0 = empty; lanes >= K hold 0). Candidates are rare and inserted one at a time.
-struct WarpList {
-  uint64_t mine;       // this lane's entry
-  uint64_t thr;        // the K-th key (0 while not full)
-  float thr_val;       // value bound below which nothing can enter (never decreases)
+// A warp's candidates: keys appended to a shared-memory buffer, plus a value bound
+// below which no element can be in the CTA's top-K. The bound is the larger of
+//   * the K-th largest running maximum over the warp's lanes (each lane's running maximum
+//     is a distinct element, so K elements reach it), and
+//   * the K-th key of the buffer after a compaction, and the CTA-wide bound (the largest
+//     bound any warp of the CTA has published).
+// Appending costs a ballot and a store; the buffer is compacted to its K largest keys by
+// rank counting only when it fills.
+constexpr int TK_CAP = 96;
+
+struct WarpCand {
+  uint64_t* buf;       // [TK_CAP] in shared memory
+  uint64_t* tmp;       // [LILICORR_MAX_K] scratch of the compaction
+  int n;               // keys in buf (warp-uniform)
+  float thr;           // value bound (warp-uniform, never decreases)
 };
 
-// Insert key c (the same in every lane, c > w.thr). Warp-collective.
-__device__ __forceinline__ void list_insert(WarpList& w, uint64_t c, int K, int lane) {
-  const int pos = __popc(__ballot_sync(FULL, lane < K && w.mine > c));   // larger entries
-  const uint64_t up = __shfl_up_sync(FULL, w.mine, 1);
-  if (lane == pos) w.mine = c;
-  else if (lane > pos && lane < K) w.mine = up;
-  w.thr = __shfl_sync(FULL, w.mine, K - 1);
-  if (w.thr) w.thr_val = fmaxf(w.thr_val, key_value(w.thr));
+__device__ __forceinline__ void warp_compact(WarpCand& w, int K, int lane) {
+  __syncwarp();
+  if (lane < K) w.tmp[lane] = 0ull;
+  __syncwarp();
+  for (int i = lane; i < w.n; i += 32) {
+    const uint64_t c = w.buf[i];
+    int rank = 0;
+    for (int j = 0; j < w.n; ++j) rank += w.buf[j] > c ? 1 : 0;
+    if (rank < K) w.tmp[rank] = c;
+  }
+  __syncwarp();
+  const uint64_t mine = lane < K ? w.tmp[lane] : 0ull;
+  const uint64_t kth = w.tmp[K - 1];
+  __syncwarp();
+  if (lane < K) w.buf[lane] = mine;
+  w.n = min(w.n, K);
+  if (kth) w.thr = fmaxf(w.thr, key_value(kth));
+  __syncwarp();
 }
 
-// Offer this lane's N values (ids id0 + j) that reach `thr`. Warp-collective: one round
-// per hot element of the busiest lane; each round's candidates are inserted in turn.
+// Append this lane's N values (ids id0 + j) that reach the bound. Warp-collective: one
+// ballot round per hot element of the busiest lane.
 template <int N>
-__device__ __forceinline__ void warp_offer(WarpList& w, const float (&x)[N], uint32_t id0,
-                                           bool valid, float thr, int K, int lane) {
+__device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], uint32_t id0,
+                                            bool valid, int K, int lane) {
   uint32_t hm = 0u;
 #pragma unroll
-  for (int j = 0; j < N; ++j) hm |= (valid && x[j] >= thr) ? (1u << j) : 0u;
+  for (int j = 0; j < N; ++j) hm |= (valid && x[j] >= w.thr) ? (1u << j) : 0u;
   while (__any_sync(FULL, hm != 0u)) {
+    if (w.n + 32 > TK_CAP) {
+      warp_compact(w, K, lane);
+#pragma unroll
+      for (int j = 0; j < N; ++j) hm &= (x[j] >= w.thr) ? ~0u : ~(1u << j);
+      if (!__any_sync(FULL, hm != 0u)) break;
+    }
     const bool has = hm != 0u;
     const int j = has ? __ffs(hm) - 1 : 0;
     hm &= hm - 1u;
     float xv = x[0];
 #pragma unroll
     for (int t = 1; t < N; ++t) xv = (j == t) ? x[t] : xv;
-    const uint64_t key = make_key(xv, id0 + (uint32_t)j);
-    unsigned mk = __ballot_sync(FULL, has && key > w.thr);
-    while (mk) {
-      const int src = __ffs(mk) - 1;
-      mk &= mk - 1u;
-      const uint64_t c = __shfl_sync(FULL, key, src);
-      if (c > w.thr) list_insert(w, c, K, lane);     // w.thr rises as the list fills
+    const unsigned mk = __ballot_sync(FULL, has);
+    if (has) w.buf[w.n + __popc(mk & ((1u << lane) - 1u))] = make_key(xv, id0 + (uint32_t)j);
+    w.n += __popc(mk);
+  }
+}
+
+// One batch: TK_UNROLL 16-byte vectors per thread (vectors it + u*TK_THREADS + tid).
+// CHECK = false: every vector is inside the chunk (no predicates). The values stay in
+// registers; the online (max, sum exp) takes one rescale check per batch; the warp looks
+// at the values for candidates only if some lane's batch maximum reaches the bound.
+template <typename T, bool CHECK>
+__device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int it, int v_end,
+                                              uint32_t id_base, int K, int tid, int lane,
+                                              float& m, float& s, WarpCand& w,
+                                              uint32_t* s_cta_thr) {
+  constexpr int VEC = Vec<T>::N;
+  uint4 raw[TK_UNROLL];
+#pragma unroll
+  for (int u = 0; u < TK_UNROLL; ++u) {
+    const int v = it + u * TK_THREADS + tid;
+    raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(0, 0, 0, 0);
+  }
+  float x[TK_UNROLL][VEC];
+  float vmx[TK_UNROLL];
+  float bmax = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < TK_UNROLL; ++u) {
+    Vec<T>::unpack(raw[u], x[u]);
+    if (CHECK && it + u * TK_THREADS + tid >= v_end)
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) x[u][j] = -INFINITY;   // contributes nothing
+    float mx = x[u][0];
+#pragma unroll
+    for (int j = 1; j < VEC; ++j) mx = fmaxf(mx, x[u][j]);
+    vmx[u] = mx;
+    bmax = fmaxf(bmax, mx);
+  }
+  // online log-sum-exp, one rescale per batch (rarely taken after the first batches)
+  if (bmax > m) {
+    s *= ex2((m - bmax) * LOG2E);
+    m = bmax;
+  }
+  if (m != -INFINITY) {
+    const float ml = m * LOG2E;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int u = 0; u < TK_UNROLL; ++u)
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) acc[j & 3] += ex2(fmaf(x[u][j], LOG2E, -ml));
+    s += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  }
+  // candidates: only when some lane's batch maximum reaches the current bound
+  w.thr = fmaxf(w.thr, unord32(*(volatile uint32_t*)s_cta_thr));
+  if (__any_sync(FULL, bmax >= w.thr)) {
+    // tighten the bound with the K-th largest running lane maximum first
+    const float tb = warp_kth_largest(m, K, lane);
+    if (tb > w.thr) {
+      w.thr = tb;
+      if (lane == 0) atomicMax(s_cta_thr, ord32(tb));
+    }
+#pragma unroll
+    for (int u = 0; u < TK_UNROLL; ++u) {
+      if (!__any_sync(FULL, vmx[u] >= w.thr)) continue;
+      const int v = it + u * TK_THREADS + tid;
+      warp_append<VEC>(w, x[u], id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
     }
   }
 }
@@ -224,7 +307,9 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
                 unsigned char* partials) {
   constexpr int VEC = Vec<T>::N;
-  __shared__ uint64_t s_keys[TK_MERGE_MAX];     // the warps' lists, later the splits' lists
+  __shared__ uint64_t s_buf[TK_WARPS][TK_CAP];   // the warps' candidates
+  __shared__ uint64_t s_tmp[TK_WARPS][LILICORR_MAX_K];
+  __shared__ uint64_t s_keys[TK_MERGE_MAX];       // the splits' lists (last CTA)
   __shared__ uint64_t s_merge[TK_MERGE_MAX];
   __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ float s_m[TK_WARPS], s_s[TK_WARPS];
@@ -244,10 +329,11 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   const int v_begin = min(split * chunk_vecs, nvec);
   const int v_end = min(v_begin + chunk_vecs, nvec);
 
-  WarpList w;
-  w.mine = 0ull;
-  w.thr = 0ull;
-  w.thr_val = -INFINITY;
+  WarpCand w;
+  w.buf = s_buf[warp];
+  w.tmp = s_tmp[warp];
+  w.n = 0;
+  w.thr = -INFINITY;
   if (tid == 0) s_cta_thr = ord32(-INFINITY);
   __syncthreads();
 
@@ -263,56 +349,53 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
       const int e = valid ? (i < e0 ? i : tail0 + (i - e0)) : 0;
       float x[1] = {valid ? Vec<T>::scalar(rp, e) : -INFINITY};
       lse_update<1>(m, s, x, valid);
-      warp_offer<1>(w, x, (uint32_t)e, valid, w.thr_val, K, lane);
+      warp_append<1>(w, x, (uint32_t)e, valid, K, lane);
     }
-    if (lane == 0 && w.thr) atomicMax(&s_cta_thr, ord32(w.thr_val));
   }
 
-  // main stream: batches of TK_UNROLL 16-byte vectors per thread
+  // main stream: full batches without predicates, then the remainder
   const uint4* vp = reinterpret_cast<const uint4*>(rp + e0);
-  for (int it = v_begin; it < v_end; it += TK_UNROLL * TK_THREADS) {
-    uint4 raw[TK_UNROLL];
-#pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u) {
-      const int v = it + u * TK_THREADS + tid;
-      raw[u] = v < v_end ? __ldcs(vp + v) : make_uint4(0, 0, 0, 0);
-    }
-    float vmx[TK_UNROLL];                      // this lane's per-vector maxima
-    float bmax = -INFINITY;
-#pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u) {
-      float x[VEC];
-      Vec<T>::unpack(raw[u], x);
-      vmx[u] = lse_update<VEC>(m, s, x, it + u * TK_THREADS + tid < v_end);
-      bmax = fmaxf(bmax, vmx[u]);
-    }
-    float thr = fmaxf(w.thr_val, unord32(*(volatile uint32_t*)&s_cta_thr));
-    if (__any_sync(FULL, bmax >= thr)) {
-      // while the list is not full, raise the bound to the K-th largest lane maximum of
-      // this batch (each lane maximum is a distinct element, so K elements reach it)
-      if (w.thr == 0ull) thr = fmaxf(thr, warp_kth_largest(bmax, K, lane));
-      w.thr_val = fmaxf(w.thr_val, thr);
-#pragma unroll
-      for (int u = 0; u < TK_UNROLL; ++u) {
-        if (!__any_sync(FULL, vmx[u] >= w.thr_val)) continue;
-        const int v = it + u * TK_THREADS + tid;
-        float x[VEC];
-        Vec<T>::unpack(raw[u], x);
-        warp_offer<VEC>(w, x, (uint32_t)(e0 + v * VEC), v < v_end, w.thr_val, K, lane);
-      }
-      if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr_val));
-    }
-  }
-  s_keys[warp * LILICORR_MAX_K + lane] = w.mine;     // publish the warp's list
+  constexpr int STEP = TK_UNROLL * TK_THREADS;
+  const int full_end = v_begin + (v_end - v_begin) / STEP * STEP;
+  for (int it = v_begin; it < full_end; it += STEP)
+    process_batch<T, false>(vp, it, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr);
+  if (full_end < v_end)
+    process_batch<T, true>(vp, full_end, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr);
 
   // (max, sum) of the warp, then of the CTA
   const float wm = warp_max(m);
   float ws = (m == -INFINITY) ? 0.f : s * ex2((m - wm) * LOG2E);
   ws = warp_sum(ws);
   if (lane == 0) { s_m[warp] = wm; s_s[warp] = ws; }
-  // CTA top-K over the warps' lists
+  // CTA top-K: keys of every warp's buffer at or above the CTA-wide bound, rank-counted.
+  // (the bound never exceeds the CTA's K-th value, so the K largest keys all survive)
+  if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr));
+  if (tid == 0) s_count = 0;
+  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
   __syncthreads();
-  cta_select(s_keys, TK_WARPS, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
+  {
+    const float bound = unord32(s_cta_thr);
+    const int nw = w.n;
+    for (int i = lane; i < nw; i += 32) {
+      const uint64_t k = w.buf[i];
+      if (key_value(k) >= bound) {
+        const int pos = atomicAdd(&s_count, 1);
+        if (pos < TK_MERGE_MAX) s_merge[pos] = k;
+      }
+    }
+  }
+  __syncthreads();
+  if (s_count > TK_MERGE_MAX) {
+    // more survivors than the merge area holds (only with massive ties at the bound):
+    // compact every warp's buffer to its own top-K first, then merge those
+    warp_compact(w, K, lane);
+    if (lane < LILICORR_MAX_K) s_keys[warp * LILICORR_MAX_K + lane] = lane < w.n ? w.buf[lane] : 0ull;
+    __syncthreads();
+    cta_select(s_keys, TK_WARPS, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
+  } else {
+    rank_place(s_merge, s_count, K, s_top, tid, TK_THREADS);
+    __syncthreads();
+  }
 
   float cm = -INFINITY, cs = 0.f;
   if (warp == 0) {
@@ -392,11 +475,12 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
 TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   const int vec = dt == LILICORR_BF16 ? 8 : 4;
   const int nvec = V / vec;
-  // about two waves of resident CTAs (4 per SM) when rows are many, one when few
+  // Few rows: split each over CTAs until the resident slots (4 CTAs per SM) are covered.
+  // Once the rows alone fill half of the slots, one CTA per row: every split adds a
+  // partial record and a merge, which costs more than the imbalance it removes.
   const int slots = num_sms() * 4;
-  const int target_ctas = rows >= slots ? 2 * slots : slots;
   const int min_chunk = 256;                 // vectors (4 KB) per CTA at least
-  int splits = ceil_div(target_ctas, rows);
+  int splits = rows * 2 >= slots ? 1 : ceil_div(slots, rows);
   splits = max(1, min(splits, ceil_div(max(nvec, 1), min_chunk)));
   splits = min(splits, min(TK_MAX_SPLITS, TK_MERGE_MAX / K));
   TopkPlan p;
