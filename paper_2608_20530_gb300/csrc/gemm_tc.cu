@@ -1,19 +1,22 @@
 // Tensor-core linear layer of the bf16 head (5th-generation tensor cores, sm_103a).
 //
 // C[M, N] = epilogue(A[M, Kd] W[N, Kd]^T) with bf16 A (activations) and W (weights),
-// fp32 accumulation in tensor memory. One CTA computes a 128 x BN tile:
-//   * warp 0 lane 0 streams 128 x 64 tiles of A and BN x 64 tiles of W into a ring
-//     of shared-memory stages with 2-D TMA copies (128-byte swizzle), each stage
-//     guarded by a "full" mbarrier (transaction bytes) and an "empty" mbarrier;
-//   * warp 1 allocates BN columns of tensor memory, and its lane 0 issues
-//     tcgen05.mma (M = 128, N = BN, K = 16) four times per stage, releasing the
-//     stage with tcgen05.commit;
-//   * all four warps then read the accumulator back with tcgen05.ld (warp w owns
-//     rows 32w..32w+31) and apply bias / per-sequence bias / SiLU / residual before
-//     storing fp32 or bf16.
-// Every wait is bounded (about 2 s); on timeout the CTA records LILICORR_ERR_TIMEOUT in
-// the status word, waits (bounded) for its copies in flight, frees its tensor
-// memory and exits.
+// fp32 accumulation in tensor memory. A persistent, warp-specialised kernel: one CTA
+// per SM walks output tiles of 128 x BN.
+//   * warp 0 (one lane) streams 128 x 64 tiles of A and BN x 64 tiles of W into a ring
+//     of shared-memory stages with 2-D TMA copies (128-byte swizzle); each stage has a
+//     "full" mbarrier (transaction bytes) and an "empty" mbarrier;
+//   * warp 1 allocates two accumulators of BN tensor-memory columns and its lane 0
+//     issues tcgen05.mma (M = 128, N = BN, K = 16), four per stage, releasing stages
+//     with tcgen05.commit and handing finished accumulators to the epilogue;
+//   * warps 2-5 drain an accumulator with tcgen05.ld while the next tile's products
+//     run on the other one. Per chunk of 128 rows x 128 bytes they add bias /
+//     per-sequence bias / SiLU / the residual (brought in by a TMA load), write the
+//     chunk into a 128-byte-swizzled staging buffer and store it with one TMA bulk
+//     tensor store (double-buffered staging and residual buffers).
+// Every mbarrier wait is bounded (about 2 s of SM cycles); on timeout the kernel records
+// LILICORR_ERR_TIMEOUT in the status word, stops issuing work while keeping every
+// thread on its barriers, lets copies in flight land, frees its tensor memory, returns.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -24,14 +27,15 @@ namespace {
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;                  // 64 bf16 = 128 bytes: one swizzle atom row
-constexpr int TC_THREADS = 128;
+constexpr int TC_THREADS = 192;            // producer, MMA, 4 epilogue warps
+constexpr int EPI_THREADS = 128;
+constexpr uint32_t CHUNK_BYTES = 128 * 128;   // staging chunk: 128 rows x 128 bytes
 constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s at the SM clock
 
 struct TcEpilogue {
-  void* C; int ldc; int c_bf16;
   const float* bias;
   const float* bias_rows; int rows_per_bias;
-  const float* residual; int ldr;
+  int has_residual;
   int act;
 };
 
@@ -46,6 +50,9 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
                "r"(bytes)
                : "memory");
 }
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -56,8 +63,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase of parity `parity` to complete; false after `limit` SM cycles
-// (the bound is read from the SM's own cycle counter, which is cheap to poll).
+// Wait for the phase of parity `parity` to complete; false after `limit` SM cycles.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
@@ -72,6 +78,30 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(smem_u32(src))
+      : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void tma_store_wait_read_le1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void tma_store_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void epi_bar() {   // the 4 epilogue warps only
+  asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
 }
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups
@@ -121,34 +151,47 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : "r"(taddr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+// byte offset of 16-byte piece j of row r inside a 128-byte-swizzled chunk
+__device__ __forceinline__ uint32_t swz(int r, int j) {
+  return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
+}
 
-template <int BN>
+template <int BN, bool OUT_BF16>
 struct TcCfg {
   static constexpr int STAGES = BN >= 256 ? 3 : 4;
   static constexpr uint32_t A_BYTES = TC_BM * TC_BK * 2;
   static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * (A_BYTES + B_BYTES);
-  static constexpr uint32_t TMEM_COLS = BN < 32 ? 32 : BN;
+  static constexpr int CH = OUT_BF16 ? 64 : 32;        // output columns per 128-byte chunk
+  static constexpr int NCH = BN / CH;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;         // two accumulators
+  static constexpr size_t RING = (size_t)STAGES * (A_BYTES + B_BYTES);
+  static constexpr size_t SMEM = 1024 + RING + 4 * (size_t)CHUNK_BYTES + BN * sizeof(float);
 };
 
-template <int BN>
+template <int BN, bool OUT_BF16>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
-                   const __grid_constant__ CUtensorMap mapW, TcEpilogue ep, int M, int N, int Kd,
+                   const __grid_constant__ CUtensorMap mapW,
+                   const __grid_constant__ CUtensorMap mapC,
+                   const __grid_constant__ CUtensorMap mapR, TcEpilogue ep, int M, int N, int Kd,
                    uint32_t* status) {
-  using Cfg = TcCfg<BN>;
-  constexpr int S = Cfg::STAGES;
+  using Cfg = TcCfg<BN, OUT_BF16>;
+  constexpr int S = Cfg::STAGES, CH = Cfg::CH, NCH = Cfg::NCH;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * Cfg::A_BYTES;
-  __shared__ __align__(8) uint64_t full[S], empty[S], done;
+  uint8_t* s_out = smem + Cfg::RING;                   // 2 staging chunks
+  uint8_t* s_res = s_out + 2 * CHUNK_BYTES;            // 2 residual chunks
+  float* s_bias = reinterpret_cast<float*>(s_res + 2 * CHUNK_BYTES);
+  __shared__ __align__(8) uint64_t full[S], empty[S], acc_full[2], acc_empty[2], res_full[2];
   __shared__ uint32_t tmem_base;
-  __shared__ int abort_flag;
+  __shared__ volatile int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.y * TC_BM, n0 = blockIdx.x * BN;
+  const int tiles_n = (N + BN - 1) / BN;
+  const int tiles = ((M + TC_BM - 1) / TC_BM) * tiles_n;
   const int nk = (Kd + TC_BK - 1) / TC_BK;
 
   if (threadIdx.x == 0) {
@@ -156,7 +199,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(&done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], EPI_THREADS / 32);
+      mbar_init(&res_full[b], 1);
+    }
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -172,88 +219,154 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = tmem_base;
 
-  if (warp == 0 && lane == 0) {
-    // ---- producer: TMA into the stage ring
-    for (int i = 0; i < nk; ++i) {
-      const int s = i % S;
-      const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(&empty[s], ph ^ 1u, WAIT_LIMIT_CYCLES)) {
-        atomicExch(&abort_flag, 1);
-        break;
-      }
-      mbar_expect_tx(&full[s], Cfg::A_BYTES + Cfg::B_BYTES);
-      tma_load_2d(sA + (size_t)s * Cfg::A_BYTES, &mapA, &full[s], i * TC_BK, m0);
-      tma_load_2d(sB + (size_t)s * Cfg::B_BYTES, &mapW, &full[s], i * TC_BK, n0);
-    }
-  } else if (warp == 1 && lane == 0) {
-    // ---- MMA issuer
-    constexpr uint32_t idesc = instr_desc(TC_BM, BN);
-    for (int i = 0; i < nk; ++i) {
-      const int s = i % S;
-      const uint32_t ph = (uint32_t)(i / S) & 1u;
-      if (!mbar_wait(&full[s], ph, WAIT_LIMIT_CYCLES)) {
-        atomicExch(&abort_flag, 1);
-        break;
-      }
-      tc_fence_after();
-      const uint64_t ad = smem_desc(sA + (size_t)s * Cfg::A_BYTES);
-      const uint64_t bd = smem_desc(sB + (size_t)s * Cfg::B_BYTES);
-#pragma unroll
-      for (int k = 0; k < TC_BK / 16; ++k)
-        mma_bf16(tmem, ad + 2ull * k, bd + 2ull * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
-      mma_commit(&empty[s]);
-    }
-    mma_commit(&done);
-  }
-  __syncwarp();
-
-  // ---- epilogue: TMEM -> registers -> shared (transpose) -> global, row segments.
-  // Lane l of warp w owns column (c0 + l) of rows 32w..32w+31 of each 32-column chunk;
-  // the chunk's residual values are loaded before they are needed, all 32 in flight
-  // (the first chunk's while the tensor cores are still busy).
-  const int mrow0 = m0 + warp * 32;
-  float res[32];
-  auto load_residual = [&](int c0) {
-    const int n = n0 + c0 + lane;
-#pragma unroll
-    for (int rr = 0; rr < 32; ++rr)
-      res[rr] = (ep.residual && n < N && mrow0 + rr < M)
-                    ? ep.residual[(size_t)(mrow0 + rr) * ep.ldr + n] : 0.f;
-  };
-  load_residual(0);
-  if (!mbar_wait(&done, 0, WAIT_LIMIT_CYCLES)) atomicExch(&abort_flag, 1);
-  tc_fence_after();
-  __syncthreads();                         // the stage ring is drained: reuse it below
-  if (!abort_flag) {
-    float* tile = reinterpret_cast<float*>(smem) + warp * 32 * 33;   // this warp's 32 x 32
-#pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 32) {
-      uint32_t r[32];
-      tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, r);
-#pragma unroll
-      for (int j = 0; j < 32; ++j) tile[lane * 33 + j] = __uint_as_float(r[j]);
-      __syncwarp();
-      const int n = n0 + c0 + lane;
-      if (n < N) {
-        const float bn = ep.bias ? ep.bias[n] : 0.f;
-#pragma unroll
-        for (int rr = 0; rr < 32; ++rr) {
-          const int m = mrow0 + rr;
-          if (m < M) {
-            float v = tile[rr * 33 + lane] + bn;
-            if (ep.bias_rows) v += ep.bias_rows[(size_t)(m / ep.rows_per_bias) * N + n];
-            if (ep.act == ACT_SILU) v = silu_f(v);
-            v += res[rr];
-            if (ep.c_bf16)
-              static_cast<__nv_bfloat16*>(ep.C)[(size_t)m * ep.ldc + n] = __float2bfloat16_rn(v);
-            else
-              static_cast<float*>(ep.C)[(size_t)m * ep.ldc + n] = v;
+  if (warp == 0) {
+    // ---- producer: TMA into the stage ring, tile after tile
+    if (lane == 0) {
+      uint32_t g = 0;                            // k-blocks issued so far
+      for (int t = blockIdx.x; t < tiles && !abort_flag; t += gridDim.x) {
+        const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
+        for (int i = 0; i < nk; ++i, ++g) {
+          const int s = (int)(g % S);
+          const uint32_t ph = (g / S) & 1u;
+          if (!mbar_wait(&empty[s], ph ^ 1u, WAIT_LIMIT_CYCLES)) {
+            abort_flag = 1;
+            break;
           }
+          mbar_expect_tx(&full[s], Cfg::A_BYTES + Cfg::B_BYTES);
+          tma_load_2d(sA + (size_t)s * Cfg::A_BYTES, &mapA, &full[s], i * TC_BK, m0);
+          tma_load_2d(sB + (size_t)s * Cfg::B_BYTES, &mapW, &full[s], i * TC_BK, n0);
         }
       }
-      if (c0 + 32 < BN) load_residual(c0 + 32);
-      __syncwarp();
     }
+  } else if (warp == 1) {
+    // ---- MMA issuer: one accumulator per tile, alternating
+    if (lane == 0) {
+      constexpr uint32_t idesc = instr_desc(TC_BM, BN);
+      uint32_t g = 0, lt = 0;
+      for (int t = blockIdx.x; t < tiles && !abort_flag; t += gridDim.x, ++lt) {
+        const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
+        if (!mbar_wait(&acc_empty[acc], aph ^ 1u, WAIT_LIMIT_CYCLES)) {
+          abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + acc * BN;
+        for (int i = 0; i < nk; ++i, ++g) {
+          const int s = (int)(g % S);
+          const uint32_t ph = (g / S) & 1u;
+          if (!mbar_wait(&full[s], ph, WAIT_LIMIT_CYCLES)) {
+            abort_flag = 1;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = smem_desc(sA + (size_t)s * Cfg::A_BYTES);
+          const uint64_t bd = smem_desc(sB + (size_t)s * Cfg::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            mma_bf16(d, ad + 2ull * k, bd + 2ull * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          mma_commit(&empty[s]);
+        }
+        mma_commit(&acc_full[acc]);
+      }
+    }
+  } else {
+    // ---- epilogue warps 2..5: warp w reads tensor-memory lanes 32*(w%4)..+31
+    const int q = warp & 3;
+    const int row = q * 32 + lane;               // row inside the tile
+    const bool leader = (warp == 2 && lane == 0);
+    uint32_t cc = 0, lt = 0;                     // chunks and tiles handled so far
+    // residual chunks come in by TMA, one chunk ahead
+    auto issue_res = [&](int t, int c, uint32_t k) {
+      const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
+      uint64_t* bar = &res_full[k & 1u];
+      mbar_expect_tx(bar, CHUNK_BYTES);
+      tma_load_2d(s_res + (k & 1u) * CHUNK_BYTES, &mapR, bar, n0 + c * CH, m0);
+    };
+    if (ep.has_residual && leader && (int)blockIdx.x < tiles) issue_res(blockIdx.x, 0, 0);
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
+      const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
+      const uint32_t acc = lt & 1u;
+      epi_bar();                                  // s_bias free again
+      for (int j = threadIdx.x - 64; j < BN; j += EPI_THREADS)
+        s_bias[j] = (ep.bias && n0 + j < N) ? ep.bias[n0 + j] : 0.f;
+      if (!abort_flag && !mbar_wait(&acc_full[acc], (lt >> 1) & 1u, WAIT_LIMIT_CYCLES))
+        abort_flag = 1;
+      tc_fence_after();
+      epi_bar();
+      const int m = m0 + row;
+      const float* brow = (ep.bias_rows && m < M)
+                              ? ep.bias_rows + (size_t)(m / ep.rows_per_bias) * N : nullptr;
+#pragma unroll 1
+      for (int c = 0; c < NCH; ++c, ++cc) {
+        const uint32_t b = cc & 1u;
+        // prefetch the next chunk's residual (its buffer was drained a chunk ago)
+        if (ep.has_residual && leader && !abort_flag) {
+          if (c + 1 < NCH) issue_res(t, c + 1, cc + 1);
+          else if (t + (int)gridDim.x < tiles) issue_res(t + gridDim.x, 0, cc + 1);
+        }
+        float v[CH];
+#pragma unroll
+        for (int h = 0; h < CH / 32; ++h) {
+          uint32_t r[32];
+          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + acc * BN + c * CH + h * 32, r);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[h * 32 + j] = __uint_as_float(r[j]);
+        }
+        if (c == NCH - 1) {
+          // accumulator drained: hand it back to the MMA warp
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[acc]);
+        }
+        if (ep.has_residual && !abort_flag &&
+            !mbar_wait(&res_full[b], (cc >> 1) & 1u, WAIT_LIMIT_CYCLES))
+          abort_flag = 1;
+#pragma unroll
+        for (int j = 0; j < CH; j += 4) {
+          float4 x = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+          const float4 bb = *reinterpret_cast<const float4*>(s_bias + c * CH + j);
+          x.x += bb.x; x.y += bb.y; x.z += bb.z; x.w += bb.w;
+          if (brow && n0 + c * CH + j < N) {
+            const float4 br = *reinterpret_cast<const float4*>(brow + n0 + c * CH + j);
+            x.x += br.x; x.y += br.y; x.z += br.z; x.w += br.w;
+          }
+          if (ep.act == ACT_SILU) {
+            x.x = silu_f(x.x); x.y = silu_f(x.y); x.z = silu_f(x.z); x.w = silu_f(x.w);
+          }
+          if (ep.has_residual) {            // fp32 output only: 4 columns = 16 bytes
+            const float4 rr =
+                *reinterpret_cast<const float4*>(s_res + b * CHUNK_BYTES + swz(row, j >> 2));
+            x.x += rr.x; x.y += rr.y; x.z += rr.z; x.w += rr.w;
+          }
+          v[j] = x.x; v[j + 1] = x.y; v[j + 2] = x.z; v[j + 3] = x.w;
+        }
+        epi_bar();          // staging buffer b: its store two chunks ago has been read
+        uint8_t* stg = s_out + b * CHUNK_BYTES;
+        if (OUT_BF16) {
+#pragma unroll
+          for (int p = 0; p < 8; ++p) {     // 8 pieces of 8 bf16
+            uint4 w;
+            w.x = pack_bf16x2(v[8 * p + 0], v[8 * p + 1]);
+            w.y = pack_bf16x2(v[8 * p + 2], v[8 * p + 3]);
+            w.z = pack_bf16x2(v[8 * p + 4], v[8 * p + 5]);
+            w.w = pack_bf16x2(v[8 * p + 6], v[8 * p + 7]);
+            *reinterpret_cast<uint4*>(stg + swz(row, p)) = w;
+          }
+        } else {
+#pragma unroll
+          for (int p = 0; p < 8; ++p)       // 8 pieces of 4 floats
+            *reinterpret_cast<float4*>(stg + swz(row, p)) =
+                make_float4(v[4 * p], v[4 * p + 1], v[4 * p + 2], v[4 * p + 3]);
+        }
+        fence_async_shared();
+        epi_bar();
+        if (leader && !abort_flag && n0 + c * CH < N) {
+          tma_store_2d(&mapC, stg, n0 + c * CH, m0);
+          tma_store_wait_read_le1();         // the other buffer is free for the next chunk
+        }
+      }
+    }
+    if (leader) tma_store_wait_all();
   }
 
   // ---- teardown
@@ -263,9 +376,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     if (threadIdx.x == 0) {
       set_status(status, LILICORR_ERR_TIMEOUT);
       // let copies still in flight land before the shared memory is released
-      for (int s = 0; s < S && s < nk; ++s) {
-        const int last = ((nk - 1 - s) / S) * S + s;
-        mbar_wait(&full[s], (uint32_t)(last / S) & 1u, WAIT_LIMIT_CYCLES / 10);
+      const long long t0 = clock64();
+      while (clock64() - t0 < WAIT_LIMIT_CYCLES / 10) {
       }
     }
     __syncthreads();
@@ -295,38 +407,65 @@ EncodeTiledFn encode_fn() {
                                          &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
       fn = reinterpret_cast<EncodeTiledFn>(p);
+    else
+      (void)cudaGetLastError();
   }
   return fn;
 }
 
-// 2-D bf16 tensor map over rows x cols (row stride ld elements), box box_rows x 64.
-bool make_map(CUtensorMap* map, const void* base, int rows, int cols, int ld, int box_rows) {
+// 2-D tensor map over rows x cols (row stride ld elements of es bytes), box
+// box_rows x box_cols, 128-byte swizzle (box_cols * es must be 128).
+bool make_map(CUtensorMap* map, const void* base, CUtensorMapDataType type, size_t es, int rows,
+              int cols, int ld, int box_rows, int box_cols) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-  cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * es};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  return fn(map, type, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN>
-lilicorr_status_t launch_bn(const GemmArgs& g, uint32_t* status, cudaStream_t st) {
-  using Cfg = TcCfg<BN>;
+template <int BN, bool OUT_BF16>
+lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
+  using Cfg = TcCfg<BN, OUT_BF16>;
   static bool configured[64] = {false};
-  LL_TRY(allow_max_dynamic_smem(gemm_tc_kernel<BN>, configured));
-  CUtensorMap ma, mw;
-  if (!make_map(&ma, g.A, g.M, g.Kd, g.lda, TC_BM)) return LILICORR_ERR_CUDA;
-  if (!make_map(&mw, g.W, g.N, g.Kd, g.ldw, BN)) return LILICORR_ERR_CUDA;
+  LL_TRY(allow_max_dynamic_smem(gemm_tc_kernel<BN, OUT_BF16>, configured));
+  CUtensorMap ma, mw, mc, mr;
+  const CUtensorMapDataType bf = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  const CUtensorMapDataType f32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+  if (!make_map(&ma, g.A, bf, 2, g.M, g.Kd, g.lda, TC_BM, TC_BK)) return LILICORR_ERR_CUDA;
+  if (!make_map(&mw, g.W, bf, 2, g.N, g.Kd, g.ldw, BN, TC_BK)) return LILICORR_ERR_CUDA;
+  if (!make_map(&mc, g.C, OUT_BF16 ? bf : f32, OUT_BF16 ? 2 : 4, g.M, g.N, g.ldc, TC_BM, Cfg::CH))
+    return LILICORR_ERR_CUDA;
+  if (g.residual) {
+    if (!make_map(&mr, g.residual, f32, 4, g.M, g.N, g.ldr, TC_BM, 32)) return LILICORR_ERR_CUDA;
+  } else {
+    mr = mc;                                   // never read
+  }
   TcEpilogue ep;
-  ep.C = g.C; ep.ldc = g.ldc; ep.c_bf16 = g.c_dt == LILICORR_BF16;
-  ep.bias = g.bias; ep.bias_rows = g.bias_rows; ep.rows_per_bias = g.rows_per_bias;
-  ep.residual = g.residual; ep.ldr = g.ldr; ep.act = g.act;
-  dim3 grid(ceil_div(g.N, BN), ceil_div(g.M, TC_BM));
-  gemm_tc_kernel<BN><<<grid, TC_THREADS, Cfg::SMEM, st>>>(ma, mw, ep, g.M, g.N, g.Kd, status);
+  ep.bias = g.bias;
+  ep.bias_rows = g.bias_rows;
+  ep.rows_per_bias = g.rows_per_bias;
+  ep.has_residual = g.residual != nullptr;
+  ep.act = g.act;
+  const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
+  const int grid = tiles < num_sms() ? tiles : num_sms();
+  gemm_tc_kernel<BN, OUT_BF16><<<grid, TC_THREADS, Cfg::SMEM, st>>>(ma, mw, mc, mr, ep, g.M, g.N,
+                                                                     g.Kd, g.status);
   return last_launch();
+}
+
+template <bool OUT_BF16>
+lilicorr_status_t launch_out(const GemmArgs& g, cudaStream_t st) {
+  // column tile: the widest of 256/128/64 that still gives every SM a tile
+  const int mt = ceil_div(g.M, TC_BM);
+  const int sms = num_sms();
+  if (g.N >= 256 && mt * ceil_div(g.N, 256) >= sms) return launch_bn<256, OUT_BF16>(g, st);
+  if (g.N >= 128 && mt * ceil_div(g.N, 128) >= sms / 2) return launch_bn<128, OUT_BF16>(g, st);
+  return launch_bn<64, OUT_BF16>(g, st);
 }
 
 }  // namespace
@@ -334,18 +473,17 @@ lilicorr_status_t launch_bn(const GemmArgs& g, uint32_t* status, cudaStream_t st
 bool gemm_tc_supported(const GemmArgs& g) {
   if (g.a_dt != LILICORR_BF16 || g.w_dt != LILICORR_BF16) return false;
   if (g.M <= 0 || g.N <= 0 || g.Kd <= 0) return false;
-  // TMA: 16-byte aligned bases and row strides
-  if (!aligned16(g.A) || !aligned16(g.W) || (g.lda % 8) || (g.ldw % 8) || (g.Kd % 8)) return false;
+  // TMA: 16-byte aligned bases and row strides, outputs in 16-byte column groups
+  if (!aligned16(g.A) || !aligned16(g.W) || !aligned16(g.C)) return false;
+  if ((g.lda % 8) || (g.ldw % 8) || (g.Kd % 8) || (g.N % 8) || (g.ldc % 8)) return false;
+  if (g.residual && (g.c_dt != LILICORR_F32 || !aligned16(g.residual) || (g.ldr % 4)))
+    return false;
+  if (g.bias_rows && (g.N % 4)) return false;
   return encode_fn() != nullptr;
 }
 
 lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st) {
-  // column tile: the widest of 256/128/64 that still gives the grid a few waves of CTAs
-  const int mt = ceil_div(g.M, TC_BM);
-  const int sms = num_sms();
-  if (g.N >= 256 && mt * ceil_div(g.N, 256) >= sms) return launch_bn<256>(g, g.status, st);
-  if (g.N >= 128 && mt * ceil_div(g.N, 128) >= sms / 2) return launch_bn<128>(g, g.status, st);
-  return launch_bn<64>(g, g.status, st);
+  return g.c_dt == LILICORR_BF16 ? launch_out<true>(g, st) : launch_out<false>(g, st);
 }
 
 }  // namespace lilicorr
