@@ -210,8 +210,9 @@ struct HeadCall {
   lilicorr_dtype_t wdt, adt, qkv_dt;     // weights; matrix-product operands; q|k|v buffer
   bool tc_attn;                          // tensor-core attention core
   uint32_t* status;
-  float *hproj, *tn, *t, *anc, *cb, *x, *oi;
-  void *c1, *xn, *qkv, *att, *hf, *u;
+  lilicorr_dtype_t tn_dt;                // normalised target state (an operand of W_t)
+  float *hproj, *t, *anc, *cb, *x, *oi;
+  void *tn, *c1, *xn, *qkv, *att, *hf, *u;
 
   HeadCall(const lilicorr_head* head, int b, void* ws, const WsLayout& w)
       : h(head), d(head->desc), B(b) {
@@ -228,7 +229,9 @@ struct HeadCall {
     qkv_dt = tc_attn ? LILICORR_BF16 : LILICORR_F32;
     status = at<uint32_t>(ws, w.status);
     hproj = at<float>(ws, w.hproj);
-    tn = at<float>(ws, w.tn);
+    tn = at<void>(ws, w.tn);
+    // rows up to 16384 are normalised in registers; longer ones pass through tn in fp32
+    tn_dt = d.H <= 16384 ? wdt : LILICORR_F32;
     t = at<float>(ws, w.t);
     anc = at<float>(ws, w.anc);
     cb = at<float>(ws, w.cb);
@@ -262,8 +265,8 @@ lilicorr_status_t run_prologue(const HeadCall& c, const void* hidden, const void
   g.bias = h->hid_b;
   LL_TRY(run_gemm(g, st));
   // target state t = W_t RMSNorm(mean of the captured layers) + b_t
-  LL_TRY(launch_target_norm(target, c.wdt, c.B, d.n_tgt, d.H, h->tgt_norm, c.tn, st));
-  g = c.G(c.tn, F32, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
+  LL_TRY(launch_target_norm(target, c.wdt, c.B, d.n_tgt, d.H, h->tgt_norm, c.tn, c.tn_dt, st));
+  g = c.G(c.tn, c.tn_dt, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
   g.bias = h->tgt_b;
   LL_TRY(run_gemm(g, st));
   // anchor out vector o_0 = unit(W_a t + b_a)

@@ -191,10 +191,10 @@ lilicorr_status_t skinny_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t s
 // keeps its means in registers between the two passes (up to TN_VPT vectors).
 constexpr int TN_THREADS = 512, TN_VPT = 4;
 
-template <typename T>
+template <typename T, typename TO>
 __global__ void __launch_bounds__(TN_THREADS)
 target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H, const float* __restrict__ gain,
-                   float* __restrict__ tn) {
+                   TO* __restrict__ tn) {
   __shared__ float red[TN_THREADS / 32];
   __shared__ float s_total;
   const int b = blockIdx.x;
@@ -234,7 +234,7 @@ target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H, const float* __r
     for (int e = 0; e < 8; ++e) {
       acc[e] *= inv_p;
       ss += acc[e] * acc[e];
-      tn[(size_t)b * H + v * 8 + e] = acc[e];
+      st_elem(tn, (size_t)b * H + v * 8 + e, acc[e]);
     }
   }
   ss = warp_sum(ss);
@@ -253,12 +253,14 @@ target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H, const float* __r
     if (v >= nv) continue;
 #pragma unroll
     for (int e = 0; e < 8; ++e)
-      tn[(size_t)b * H + v * 8 + e] = mean[q][e] * r * gain[v * 8 + e];
+      st_elem(tn, (size_t)b * H + v * 8 + e, mean[q][e] * r * gain[v * 8 + e]);
   }
   for (int v = threadIdx.x + TN_VPT * TN_THREADS; v < nv; v += TN_THREADS)
 #pragma unroll
-    for (int e = 0; e < 8; ++e)
-      tn[(size_t)b * H + v * 8 + e] = tn[(size_t)b * H + v * 8 + e] * r * gain[v * 8 + e];
+    for (int e = 0; e < 8; ++e) {
+      const size_t o = (size_t)b * H + v * 8 + e;
+      st_elem(tn, o, ld_elem(tn, o) * r * gain[v * 8 + e]);
+    }
 }
 
 // ----------------------------------------------------------------------------- nodes
@@ -463,14 +465,20 @@ lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st) {
 }
 
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
-                                     const float* gain, float* tn, cudaStream_t st) {
+                                     const float* gain, void* tn, lilicorr_dtype_t tn_dt,
+                                     cudaStream_t st) {
   if (B == 0) return LILICORR_OK;
-  if (dt == LILICORR_F32)
-    target_norm_kernel<float><<<B, TN_THREADS, 0, st>>>(static_cast<const float*>(T), n_tgt, H, gain,
-                                                        tn);
+  if (dt == LILICORR_F32 && tn_dt == LILICORR_F32)
+    target_norm_kernel<float, float><<<B, TN_THREADS, 0, st>>>(
+        static_cast<const float*>(T), n_tgt, H, gain, static_cast<float*>(tn));
+  else if (dt == LILICORR_BF16 && tn_dt == LILICORR_F32)
+    target_norm_kernel<__nv_bfloat16, float><<<B, TN_THREADS, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<float*>(tn));
+  else if (dt == LILICORR_BF16)
+    target_norm_kernel<__nv_bfloat16, __nv_bfloat16><<<B, TN_THREADS, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<__nv_bfloat16*>(tn));
   else
-    target_norm_kernel<__nv_bfloat16><<<B, TN_THREADS, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, tn);
+    return LILICORR_ERR_DTYPE;
   return last_launch();
 }
 

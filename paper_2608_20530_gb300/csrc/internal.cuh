@@ -186,7 +186,8 @@ lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
 
 // scoring-network helpers (head_kernels.cu)
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
-                                     const float* gain, float* tn, cudaStream_t st);
+                                     const float* gain, void* tn, lilicorr_dtype_t tn_dt,
+                                     cudaStream_t st);
 lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
                                     const float* logp, const float* hproj, void* c1,
                                     lilicorr_dtype_t c1_dt, float* x, uint32_t* status,
