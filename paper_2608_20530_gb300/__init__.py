@@ -63,6 +63,7 @@ _SIGS = {
     "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
+    "lilicorr_test_fused_path": (_I, [_P, _I]),
     "lilicorr_topk_lse_noalloc_max_bytes": (_S, []),
     "lilicorr_topk_lse_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
     "lilicorr_test_linear": (_I, [_P, _I, _I, _P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I,
@@ -340,6 +341,13 @@ def test_linear(A: torch.Tensor, W: torch.Tensor, out_dtype=torch.float32, bias=
                                       C.stride(0), M, N, Kd, _ptr(bias), _ptr(residual), act,
                                       path, _ptr(status), _stream()), "test_linear")
     return C
+
+
+def test_fused_path(head: Optional[Head], enable: bool) -> bool:
+    """Test hook: allow (True) or forbid (False) the fused scoring-network kernel for
+    every head in the process; returns whether ``head`` takes it when allowed."""
+    h = head._h if head is not None else _P()
+    return bool(lib().lilicorr_test_fused_path(h, 1 if enable else 0))
 
 
 def select_block_intermediates(head: Head, B: int, ws: Workspace) -> Dict[str, torch.Tensor]:

@@ -17,6 +17,7 @@ size_t attention_smem_bytes(int LK, int hd, int warps);
 size_t pair_walk_smem_bytes(int L, int K, int d);
 
 static std::atomic<uint64_t> g_launches{0};
+int g_fused_enabled = 1;
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int num_sms() {
@@ -288,6 +289,8 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   const lilicorr_head_desc& d = c.d;
   const lilicorr_dtype_t F32 = LILICORR_F32, adt = c.adt;
   const int D = c.D, F = c.F, N = c.N;
+  if (h->net_maps && g_fused_enabled)
+    return launch_net_fused(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
   LL_TRY(launch_node_build(h, c.B, ids, logp, c.hproj, c.c1, adt, c.x, c.status, st));
   GemmArgs g = c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D);
@@ -494,6 +497,7 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(LILICORR_ERR_CUDA);
   cudaFree(embed_dev);
   embed_dev = nullptr;
+  h->net_maps = net_fused_maps_create(h);
   *out = h;
   return LILICORR_OK;
 }
@@ -504,6 +508,7 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   cudaGetDevice(&cur);
   if (cur != h->device) cudaSetDevice(h->device);
   cudaError_t e = cudaFree(h->pool);
+  net_fused_maps_free(h->net_maps);
   if (h->side) cudaStreamDestroy(h->side);
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
   if (h->ev_join) cudaEventDestroy(h->ev_join);
@@ -686,6 +691,11 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
     case 3: return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_DTYPE;
   }
   return LILICORR_ERR_ARG;
+}
+
+int lilicorr_test_fused_path(const lilicorr_head* head, int enable) {
+  g_fused_enabled = enable ? 1 : 0;
+  return head && head->net_maps ? 1 : 0;
 }
 
 uint64_t lilicorr_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }

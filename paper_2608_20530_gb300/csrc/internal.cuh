@@ -137,6 +137,7 @@ struct lilicorr_head {
   const void* woi;            // [2d, D]: out_w rows then in_w rows
   const float* boi;           // [2d]
   const void* anc_w; const float* anc_b;
+  void* net_maps;             // tensor maps of the fused scoring network, or null
 };
 
 namespace lilicorr {
@@ -185,6 +186,16 @@ bool gemm_tc_supported(const GemmArgs& g);
 lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
 
 // scoring-network helpers (head_kernels.cu)
+// fused scoring network (net_fused.cu): one CTA per sequence, bf16 head with D = 256,
+// 8 heads, FFN 2D, L*K <= 128. Writes oi like run_body's unfused chain.
+bool net_fused_supported(const lilicorr_head_desc& d);
+void* net_fused_maps_create(const lilicorr_head* h);
+void net_fused_maps_free(void* maps);
+lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t* ids,
+                                   const float* logp, const float* hproj, const float* t,
+                                   const float* cb, float* oi, uint32_t* status, cudaStream_t st);
+extern int g_fused_enabled;   // testing switch: 0 keeps every head on the unfused chain
+
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
                                      const float* gain, void* tn, lilicorr_dtype_t tn_dt,
                                      cudaStream_t st);

@@ -1,0 +1,943 @@
+// Step (2), candidate-dependent part, fused: the node features, the two-layer scoring
+// Transformer, the fusion layer and the out / in heads for one sequence in one CTA
+// (Sec. 3.2; App. A), on the bf16 head with D = 256, 8 heads, FFN 2D, L*K <= 128.
+//
+// The L*K nodes of a sequence are the 128 rows (zero-padded) of one tensor-core tile.
+// The residual stream x[128, 256] lives in tensor memory (fp32, columns 0-255) for the
+// whole network; the matrix products accumulate into it directly. Columns 256-511 are
+// the scratch accumulator of the other products. Activations that feed a product (c1,
+// RMSNorm outputs, the attention output, the FFN hidden state, the fusion input) are
+// written by the row workers as bf16 into shared memory in the 128-byte-swizzled
+// K-major layout the tensor cores read. Weights stream through a two-stage ring by TMA,
+// one copy per 64-wide K chunk of a product: the chunk's 256 (or, for q|k|v of a head
+// pair, 192) rows arrive as one 32 KB (24 KB) swizzled tile and feed four MMAs of
+// N = 256 (192). One SM completes about one TMA copy per 0.3 us almost independently of
+// its size up to 64 KB, so the tiles are as large as shared memory allows. Bias and gain
+// vectors and the confidence-network weights are staged in shared memory.
+//
+// Warp roles (320 threads):
+//   warp 0    one lane: TMA producer of the weight ring
+//   warp 1    tensor-memory allocation; one lane issues tcgen05.mma (M 128, N 256/192, K 16)
+//   warps 2-9 row workers. Warp w reads tensor-memory lanes 32*(w%4)..+31, so thread
+//             (set s = (w-2)/4, row r) owns row r and the column half s of a 256-wide
+//             region. They build the nodes, drain accumulators (bias, SiLU, RMSNorm),
+//             and run the attention core with warp-level mma.sync: set s takes head
+//             2g+s of head pair g, each warp 32 queries, all L*K keys in one pass.
+//
+// Products, in issue order (A operand in shared memory, accumulator in tensor memory):
+//   conf2                 x += c1 W_c2^T                      (x preloaded with the node base)
+//   per layer l, pair g:  q|k|v of heads 2g, 2g+1 = xn Wqkv_g^T  -> scratch
+//                         x += att_g W_o[:, 64g:64g+64]^T     (attention output, per pair)
+//                         h_a = xn2 W_1[0:256]^T, h_b = xn2 W_1[256:512]^T -> scratch
+//                         x += SiLU(h_a) W_2[:, 0:256]^T + SiLU(h_b) W_2[:, 256:512]^T
+//   fusion                u = [xf | xf*t] W_f,x^T             -> scratch (+ the t block, per sequence)
+//   heads                 [o | i] = u W_oi^T                  -> scratch, 256 columns at a time
+// Biases that add into x (b_o, b_2) are added by the row workers on the next RMSNorm
+// pass, which writes x back to tensor memory.
+//
+// Hand-offs are mbarriers, one per event and sequence (phase parity = the CTA's
+// sequence count), so no barrier is ever more than one phase ahead of its waiter.
+// Every wait is bounded; on timeout the CTA records LILICORR_ERR_TIMEOUT, stops issuing
+// copies and products, runs its remaining barriers through and frees tensor memory.
+#include <new>
+
+#include "tc_ptx.cuh"
+
+namespace lilicorr {
+
+namespace {
+using namespace tc;
+
+constexpr int NF_D = 256;                 // node width
+constexpr int NF_F = 512;                 // FFN width
+constexpr int NF_NH = 8;                  // heads
+constexpr int NF_HD = 32;                 // head width
+constexpr int NF_M = 128;                 // node rows per CTA
+constexpr int NF_STAGES = 2;              // weight ring depth
+constexpr int NF_MAX_LAYERS = 4;
+constexpr int NF_MAX_L = 64;
+constexpr int NF_RW = 256;                // row-worker threads
+constexpr int NF_THREADS = 64 + NF_RW;
+constexpr uint32_t STAGE_BYTES = 256 * 64 * 2;   // one K chunk of 256 weight rows
+constexpr uint32_t CHUNK = 128 * 128;     // 128 rows x 64 bf16, one swizzled K chunk
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t X_COL = 0, SCR_COL = 256;
+constexpr long long WAIT_LIMIT = 4000000000ll;   // about 2 s of SM cycles
+constexpr float LOG2E = 1.4426950408889634f;
+constexpr float NF_RMS_EPS = 1e-6f;
+
+// shared-memory layout (offsets from the 1024-aligned base)
+constexpr uint32_t OFF_RING = 0;
+constexpr uint32_t OFF_ACT = OFF_RING + NF_STAGES * STAGE_BYTES;   // 64 KB: 4 chunks
+constexpr uint32_t OFF_HF = OFF_ACT + 4 * CHUNK;                   // 64 KB: 4 chunks
+constexpr uint32_t OFF_ATT = OFF_HF + 3 * CHUNK;                   // attention output chunk
+constexpr uint32_t QKV_SET = 3 * 8192;                             // q, k, v of one head
+constexpr uint32_t OFF_VEC = OFF_HF + 4 * CHUNK;                   // staged vectors (floats)
+// float offsets inside the vector area
+constexpr int V_AN = 0, V_FN = 256, V_BO = 512, V_B1 = 768, V_BQKV = 1280, V_B2 = 2048,
+              V_C1W = 2560, V_C1B = 3840, V_C2B = 4096, V_FIN = 4352, V_BOI = 4608, V_T = 5120,
+              V_CB = 5376, V_END = 5632;
+constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [2][128] float
+constexpr uint32_t OFF_DIST = OFF_SS + 2 * NF_M * 4;               // [8][127] float
+constexpr uint32_t OFF_SAME = OFF_DIST + NF_NH * (2 * NF_MAX_L - 1) * 4;
+constexpr uint32_t OFF_SLOT = OFF_SAME + NF_NH * 4;                // [128] slot of each node
+constexpr uint32_t OFF_BAR = (OFF_SLOT + NF_M + 63) & ~63u;
+constexpr int N_EV = 52;                                           // per direction
+constexpr uint32_t NF_SMEM_USED = OFF_BAR + (2 * NF_STAGES + 2 * N_EV) * 8;
+constexpr size_t NF_SMEM = 1024 + NF_SMEM_USED;
+static_assert(NF_SMEM <= 227 * 1024, "shared memory of the fused network kernel");
+static_assert(OFF_ACT % 1024 == 0 && OFF_HF % 1024 == 0 && OFF_ATT % 1024 == 0, "swizzle atoms");
+
+enum { G_CONF2, G_QKV, G_WO, G_W1, G_W2, G_FUSE, G_WOI };
+
+// event ids: MMA -> row workers (commits) and row workers -> MMA (8 warp arrivals)
+__device__ __forceinline__ int lb(int l) { return 1 + 11 * l; }
+__device__ __forceinline__ int done_id(int kind, int l, int g, int nl) {
+  switch (kind) {
+    case G_CONF2: return 0;
+    case G_QKV: return lb(l) + g;
+    case G_WO: return lb(l) + 4 + g;
+    case G_W1: return lb(l) + 8 + g;
+    case G_W2: return g == 1 ? lb(l) + 10 : -1;
+    case G_FUSE: return lb(nl);
+    default: return lb(nl) + 1 + g;
+  }
+}
+__device__ __forceinline__ int ready_id(int kind, int l, int g, int nl) {
+  switch (kind) {
+    case G_CONF2: return 0;
+    case G_QKV: return g == 0 ? lb(l) : lb(l) + g;        // xn, then "q|k|v of pair g-1 drained"
+    case G_WO: return lb(l) + 4 + g;                     // attention output of pair g
+    case G_W1: return lb(l) + 8 + g;                     // xn2; then h_a drained into HF
+    case G_W2: return g == 1 ? lb(l) + 10 : -1;          // h_b in ACT
+    case G_FUSE: return lb(nl);
+    default: return lb(nl) + 1 + g;                      // u; then head half g-1 drained
+  }
+}
+// ids the row workers use
+__device__ __forceinline__ int D_QKV(int l, int g) { return lb(l) + g; }
+__device__ __forceinline__ int D_WO(int l, int g) { return lb(l) + 4 + g; }
+__device__ __forceinline__ int D_FFN(int l, int h) { return lb(l) + 8 + h; }
+__device__ __forceinline__ int D_LAYER(int l) { return lb(l) + 10; }
+__device__ __forceinline__ int R_XN(int l) { return lb(l); }
+__device__ __forceinline__ int R_QKV_DRAINED(int l, int g) { return lb(l) + 1 + g; }
+__device__ __forceinline__ int R_ATT(int l, int g) { return lb(l) + 4 + g; }
+__device__ __forceinline__ int R_XN2(int l) { return lb(l) + 8; }
+__device__ __forceinline__ int R_HFA(int l) { return lb(l) + 9; }
+__device__ __forceinline__ int R_HFB(int l) { return lb(l) + 10; }
+
+struct NetMaps {
+  CUtensorMap conf2, fuse, woi;
+  CUtensorMap wqkv[NF_MAX_LAYERS], wo[NF_MAX_LAYERS], w1[NF_MAX_LAYERS], w2[NF_MAX_LAYERS];
+};
+
+struct NetArgs {
+  int B, L, K, LK, V, n_layers, d2;
+  const int32_t* ids;
+  const float* logp;
+  const float* hproj;       // [B*L, D]
+  const float* t;           // [B, D]
+  const float* cb;          // [B, D]: t block of the fusion layer plus its bias
+  const float* fold;        // [V, D]
+  const float *slot, *rank, *conf1_w, *conf1_b, *conf2_b;
+  const float* bqkv[NF_MAX_LAYERS];
+  const float* bo[NF_MAX_LAYERS];
+  const float* b1[NF_MAX_LAYERS];
+  const float* b2[NF_MAX_LAYERS];
+  const float* an[NF_MAX_LAYERS];
+  const float* fn[NF_MAX_LAYERS];
+  const float* dist[NF_MAX_LAYERS];
+  const float* same[NF_MAX_LAYERS];
+  const float* final_norm;
+  const float* boi;
+  float* oi;                // [B*LK, d2]
+  uint32_t* status;
+};
+
+// K chunks of a product and the rows (output columns) of each chunk's weight tile
+__device__ __forceinline__ int n_chunks(int kind) {
+  switch (kind) {
+    case G_WO: return 1;
+    case G_FUSE: return 8;
+    default: return 4;
+  }
+}
+__device__ __forceinline__ int tile_rows(int kind) { return kind == G_QKV ? 192 : 256; }
+
+// Copy K chunk kc of product (kind, l, g)'s weights into a ring stage.
+__device__ __forceinline__ void load_chunk(const NetMaps& m, int kind, int l, int g, int kc,
+                                           void* dst, uint64_t* bar) {
+  switch (kind) {
+    case G_CONF2: tma_load_3d(dst, &m.conf2, bar, 0, 0, kc); break;
+    // q, k, v rows of head pair g, gathered from [3D, D] by a 5-D view
+    case G_QKV: tma_load_5d(dst, &m.wqkv[l], bar, 0, 0, g, 0, kc); break;
+    case G_WO: tma_load_3d(dst, &m.wo[l], bar, 0, 0, g); break;
+    case G_W1: tma_load_3d(dst, &m.w1[l], bar, 0, 256 * g, kc); break;
+    case G_W2: tma_load_3d(dst, &m.w2[l], bar, 0, 0, 4 * g + kc); break;
+    case G_FUSE: tma_load_3d(dst, &m.fuse, bar, 0, 0, kc); break;
+    default: tma_load_3d(dst, &m.woi, bar, 0, 256 * g, kc); break;
+  }
+}
+
+// The product sequence of one sequence, shared by the producer and the MMA issuer.
+template <class Op>
+__device__ __forceinline__ void schedule(const NetArgs& a, Op& op) {
+  op.gemm(G_CONF2, 0, 0);
+  for (int l = 0; l < a.n_layers; ++l) {
+    op.gemm(G_QKV, l, 0);
+    for (int g = 0; g < 4; ++g) {
+      if (g + 1 < 4) op.gemm(G_QKV, l, g + 1);
+      op.gemm(G_WO, l, g);
+    }
+    op.gemm(G_W1, l, 0);
+    op.gemm(G_W1, l, 1);
+    op.gemm(G_W2, l, 0);
+    op.gemm(G_W2, l, 1);
+  }
+  op.gemm(G_FUSE, 0, 0);
+  for (int h = 0; h * 256 < a.d2; ++h) op.gemm(G_WOI, 0, h);
+}
+
+struct Shared {
+  uint8_t* base;
+  uint64_t *full, *empty, *done, *ready;
+  volatile int* abort;
+};
+
+__device__ __forceinline__ bool ev_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (*abort) return false;
+  if (!mbar_wait(bar, parity, WAIT_LIMIT)) {
+    *abort = 1;
+    return false;
+  }
+  return true;
+}
+
+struct Producer {
+  const NetMaps* m;
+  const NetArgs* a;
+  Shared sh;
+  uint32_t n;                              // chunks issued so far
+  __device__ void gemm(int kind, int l, int g) {
+    const int nk = n_chunks(kind);
+    const uint32_t bytes = (uint32_t)tile_rows(kind) * 128u;
+    for (int kc = 0; kc < nk; ++kc, ++n) {
+      const int s = (int)(n % NF_STAGES);
+      const uint32_t ph = (n / NF_STAGES) & 1u;
+      if (!ev_wait(&sh.empty[s], ph ^ 1u, sh.abort)) continue;
+      mbar_expect_tx(&sh.full[s], bytes);
+      load_chunk(*m, kind, l, g, kc, sh.base + OFF_RING + (size_t)s * STAGE_BYTES, &sh.full[s]);
+    }
+  }
+};
+
+struct Issuer {
+  const NetArgs* a;
+  Shared sh;
+  uint32_t n, tmem, parity;
+  __device__ void gemm(int kind, int l, int g) {
+    const int nl = a->n_layers;
+    const int rd = ready_id(kind, l, g, nl);
+    if (rd >= 0) {
+      ev_wait(&sh.ready[rd], parity, sh.abort);
+      tc_fence_after();
+    }
+    const int nk = n_chunks(kind);
+    const bool onto_x = kind == G_CONF2 || kind == G_WO || kind == G_W2;
+    const uint32_t d = tmem + (onto_x ? X_COL : SCR_COL);
+    const uint32_t idesc = kind == G_QKV ? instr_desc(128, 192) : instr_desc(128, 256);
+    for (int kc = 0; kc < nk; ++kc, ++n) {
+      uint32_t a_off;
+      switch (kind) {
+        case G_WO: a_off = OFF_ATT; break;
+        case G_W2: a_off = (g == 0 ? OFF_HF : OFF_ACT) + kc * CHUNK; break;
+        case G_FUSE: a_off = kc < 4 ? OFF_ACT + kc * CHUNK : OFF_HF + (kc - 4) * CHUNK; break;
+        default: a_off = OFF_ACT + kc * CHUNK; break;
+      }
+      const int s = (int)(n % NF_STAGES);
+      const uint32_t ph = (n / NF_STAGES) & 1u;
+      if (!ev_wait(&sh.full[s], ph, sh.abort)) continue;
+      tc_fence_after();
+      const uint64_t ad = smem_desc(sh.base + a_off);
+      const uint64_t bd = smem_desc(sh.base + OFF_RING + (size_t)s * STAGE_BYTES);
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        mma_bf16(d, ad + 2ull * k, bd + 2ull * k, idesc, (onto_x || kc > 0 || k > 0) ? 1u : 0u);
+      mma_commit(&sh.empty[s]);
+    }
+    const int dn = done_id(kind, l, g, nl);
+    if (dn >= 0 && !*sh.abort) mma_commit(&sh.done[dn]);
+  }
+};
+
+// ---------------------------------------------------------------- row-worker helpers
+__device__ __forceinline__ uint32_t swz(int r, int j) {     // 16-byte piece j of row r
+  return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
+}
+// q / k / v of one head: [128 rows][32] bf16, 64-byte rows, pieces XOR-swizzled by row
+// pair so that ldmatrix over 8 consecutive rows touches 8 distinct bank groups
+__device__ __forceinline__ uint32_t qkv_off(int row, int piece) {
+  return (uint32_t)(row * 64 + ((piece ^ ((row >> 1) & 3)) << 4));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ void rw_bar() { named_bar(1, NF_RW); }
+// 16-byte asynchronous global -> shared copies (L2 only), many in flight per thread
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
+}
+// SiLU with the fast reciprocal: z / (1 + e^-z)
+__device__ __forceinline__ float silu_fast(float z) { return __fdividef(z, 1.0f + __expf(-z)); }
+__device__ __forceinline__ void set_bar(int set) { named_bar(2 + set, NF_RW / 2); }
+
+// One warp's arrival on a row-worker -> MMA event, after its shared-memory writes
+// (generic proxy, read by the tensor cores through the async proxy) and tensor-memory
+// stores.
+__device__ __forceinline__ void rw_signal(uint64_t* bar, int lane) {
+  fence_async_shared();
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(bar);
+}
+
+// 8 bf16 of v[p*8 .. p*8+7] as one 16-byte piece
+__device__ __forceinline__ uint4 pack8(const float* v) {
+  uint4 w;
+  w.x = pack_bf16x2(v[0], v[1]);
+  w.y = pack_bf16x2(v[2], v[3]);
+  w.z = pack_bf16x2(v[4], v[5]);
+  w.w = pack_bf16x2(v[6], v[7]);
+  return w;
+}
+
+// Write 32 values (columns c0..c0+31 of row r) as bf16 into a swizzled operand buffer
+// holding 64-column chunks.
+__device__ __forceinline__ void put32(uint8_t* buf, int r, int c0, const float (&v)[32]) {
+  uint8_t* ch = buf + (c0 >> 6) * CHUNK;
+  const int p0 = (c0 & 63) >> 3;
+#pragma unroll
+  for (int p = 0; p < 4; ++p) *reinterpret_cast<uint4*>(ch + swz(r, p0 + p)) = pack8(v + 8 * p);
+}
+
+__device__ __forceinline__ void ld32f(uint32_t taddr, float (&v)[32]) {
+  uint32_t u[32];
+  tmem_ld32(taddr, u);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(u[j]);
+}
+__device__ __forceinline__ void st32f(uint32_t taddr, const float (&v)[32]) {
+  uint32_t u[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(v[j]);
+  tmem_st32(taddr, u);
+}
+
+// RMSNorm statistics of row r over the 256 columns of x (each thread its half): adds
+// `bias` (shared memory) into x first (and writes x back to tensor memory when write_back). Returns
+// 1 / rms.
+__device__ float row_rstd(uint32_t tx, const float* bias, bool write_back, int set, int r,
+                          float* s_ss) {
+  float ss = 0.f;
+#pragma unroll 1
+  for (int j = 0; j < 4; ++j) {
+    const int c0 = 128 * set + 32 * j;
+    float v[32];
+    ld32f(tx + c0, v);
+    if (bias) {
+#pragma unroll
+      for (int e = 0; e < 32; ++e) v[e] += bias[c0 + e];
+      if (write_back) st32f(tx + c0, v);
+    }
+#pragma unroll
+    for (int e = 0; e < 32; ++e) ss = fmaf(v[e], v[e], ss);
+  }
+  if (bias && write_back) tmem_wait_st();
+  s_ss[set * NF_M + r] = ss;
+  rw_bar();
+  const float tot = s_ss[r] + s_ss[NF_M + r];
+  rw_bar();                                  // s_ss free for the next statistics
+  return rsqrtf(tot / (float)NF_D + NF_RMS_EPS);
+}
+
+// xn = x * rstd * gain (+ bias already in x) -> bf16 into ACT; with t, also xn * t -> HF
+__device__ void row_normed(uint8_t* sm, uint32_t tx, const float* bias, float rstd,
+                           const float* gain, const float* t, int set, int r) {
+#pragma unroll 1
+  for (int j = 0; j < 4; ++j) {
+    const int c0 = 128 * set + 32 * j;
+    float v[32];
+    ld32f(tx + c0, v);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      const float b = bias ? bias[c0 + e] : 0.f;
+      v[e] = (v[e] + b) * rstd * gain[c0 + e];
+    }
+    put32(sm + OFF_ACT, r, c0, v);
+    if (t) {
+#pragma unroll
+      for (int e = 0; e < 32; ++e) v[e] *= t[c0 + e];
+      put32(sm + OFF_HF, r, c0, v);
+    }
+  }
+}
+
+// Drain 256 scratch columns: v + bias (+ per-sequence row bias), SiLU -> bf16 into buf.
+__device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, const float* bias2,
+                           int set, int r) {
+#pragma unroll 1
+  for (int j = 0; j < 4; ++j) {
+    const int c0 = 128 * set + 32 * j;
+    float v[32];
+    ld32f(tscr + c0, v);
+#pragma unroll
+    for (int e = 0; e < 32; ++e) {
+      float z = v[e] + bias[c0 + e];
+      if (bias2) z += bias2[c0 + e];
+      v[e] = silu_fast(z);
+    }
+    put32(buf, r, c0, v);
+  }
+}
+
+// ---------------------------------------------------------------- the kernel
+__global__ void __launch_bounds__(NF_THREADS, 1)
+    net_fused_kernel(const __grid_constant__ NetMaps maps, const __grid_constant__ NetArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  __shared__ uint32_t tmem_base;
+  __shared__ volatile int abort_flag;
+  Shared sh;
+  sh.base = sm;
+  sh.full = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
+  sh.empty = sh.full + NF_STAGES;
+  sh.done = sh.empty + NF_STAGES;
+  sh.ready = sh.done + N_EV;
+  sh.abort = &abort_flag;
+  float* s_ss = reinterpret_cast<float*>(sm + OFF_SS);
+  float* s_dist = reinterpret_cast<float*>(sm + OFF_DIST);
+  float* s_same = reinterpret_cast<float*>(sm + OFF_SAME);
+  uint8_t* s_slot = sm + OFF_SLOT;
+  float* vec = reinterpret_cast<float*>(sm + OFF_VEC);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < NF_STAGES; ++s) {
+      mbar_init(&sh.full[s], 1);
+      mbar_init(&sh.empty[s], 1);
+    }
+    for (int e = 0; e < N_EV; ++e) {
+      mbar_init(&sh.done[e], 1);
+      mbar_init(&sh.ready[e], NF_RW / 32);
+    }
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(&tmem_base, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int i = 0; i < 19; ++i)
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(
+                         reinterpret_cast<const CUtensorMap*>(&maps) + i))
+                     : "memory");
+      Producer p{&maps, &a, sh, 0u};
+      for (int b = blockIdx.x; b < a.B; b += gridDim.x) schedule(a, p);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      Issuer is{&a, sh, 0u, tmem, 0u};
+      for (int b = blockIdx.x; b < a.B; b += gridDim.x, is.parity ^= 1u) schedule(a, is);
+    }
+  } else {
+    // ------------------------------------------------------------ row workers
+    const int set = (warp - 2) >> 2;                 // column half / head of the pair
+    const int wi = (warp - 2) & 3;                   // warp inside the set
+    const int q = warp & 3;                          // tensor-memory lane quarter
+    const int r = q * 32 + lane;                     // node row
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const uint32_t tx = tmem + lane_off + X_COL, tscr = tmem + lane_off + SCR_COL;
+    const int L = a.L, K = a.K, LK = a.LK, nl = a.n_layers;
+    const int nd = 2 * L - 1;
+    const int tid = threadIdx.x - 64;
+    // vectors used by every sequence: confidence-network weights (transposed to [5][D]),
+    // b_c2, the final RMSNorm gain, the out / in head biases
+    for (int i = tid; i < NF_D; i += NF_RW) {
+#pragma unroll
+      for (int j = 0; j < LILICORR_N_CONF; ++j)
+        vec[V_C1W + j * NF_D + i] = a.conf1_w[i * LILICORR_N_CONF + j];
+      vec[V_C1B + i] = a.conf1_b[i];
+      vec[V_C2B + i] = a.conf2_b[i];
+      vec[V_FIN + i] = a.final_norm[i];
+    }
+    for (int i = tid; i < a.d2; i += NF_RW) vec[V_BOI + i] = a.boi[i];
+    uint32_t par = 0;
+    for (int b = blockIdx.x; b < a.B; b += gridDim.x, par ^= 1u) {
+      for (int i = tid; i < NF_D; i += NF_RW) {           // this sequence's t and t block
+        vec[V_T + i] = a.t[(size_t)b * NF_D + i];
+        vec[V_CB + i] = a.cb[(size_t)b * NF_D + i];
+      }
+      rw_bar();
+      // ---- nodes: x = fold[id] + W_h h_s + b_h + slot[s] + rank[k] + b_c2, c1 = SiLU(W_c1 f + b_c1)
+      {
+        const bool ok = r < LK;
+        float f[LILICORR_N_CONF] = {0.f, 0.f, 0.f, 0.f, 0.f};
+        if (ok) {
+          const int s = r / K, k = r % K;
+          const size_t rk = ((size_t)b * L + s) * K;
+          const float lp = a.logp[rk + k], lp0 = a.logp[rk];
+          f[0] = lp;
+          f[1] = expf(lp);
+          f[2] = lp0 - lp;
+          f[3] = K > 1 ? (float)k / (float)(K - 1) : 0.f;
+          f[4] = k == 0 ? 1.f : 0.f;
+        }
+        // node base rows. cp.async brings, all at once, the drafter-state rows W_h h_s + b_h,
+        // the slot and rank tables (into ACT, which c1 fills afterwards) and the folded
+        // embedding rows of 64 nodes at a time (into HF, 16-byte pieces XOR-swizzled by row);
+        // the thread owning a row then sums its half from shared memory into tensor memory.
+        float* tab = reinterpret_cast<float*>(sm + OFF_ACT);     // rows: hproj+slot+b_c2 [L], rank [K]
+        uint8_t* stg = sm + OFF_HF;
+        const int wr = warp - 2;
+        for (int i = tid; i < (2 * L + K) * (NF_D / 4); i += NF_RW) {
+          const int row = i / (NF_D / 4), c = (i % (NF_D / 4)) * 4;
+          const float* src = row < L ? a.hproj + ((size_t)b * L + row) * NF_D + c
+                           : row < 2 * L ? a.slot + (size_t)(row - L) * NF_D + c
+                                         : a.rank + (size_t)(row - 2 * L) * NF_D + c;
+          cp_async16(tab + (size_t)row * NF_D + c, src);
+        }
+        auto fetch_fold = [&](int p) {
+          for (int nloc = wr; nloc < 64; nloc += NF_RW / 32) {
+            const int n = 64 * p + nloc;
+            if (n >= LK) break;
+            int id = a.ids[((size_t)b * L + n / K) * K + n % K];
+            if (id < 0 || id >= a.V) {              // an id outside the vocabulary: flag, read row 0
+              if (lane == 0) set_status(a.status, LILICORR_ERR_ARG);
+              id = 0;
+            }
+            const float* src = a.fold + (size_t)id * NF_D + 8 * lane;
+            uint8_t* row = stg + nloc * 1024;
+            cp_async16(row + (((2 * lane) ^ (nloc & 7)) << 4), src);
+            cp_async16(row + (((2 * lane + 1) ^ (nloc & 7)) << 4), src + 4);
+          }
+        };
+        fetch_fold(0);
+        cp_async_wait_all();
+        rw_bar();
+        for (int i = tid; i < L * (NF_D / 4); i += NF_RW) {   // S[s] = hproj + slot + b_c2
+          const int row = i / (NF_D / 4), c = (i % (NF_D / 4)) * 4;
+          float4 x = *reinterpret_cast<float4*>(tab + (size_t)row * NF_D + c);
+          const float4 y = *reinterpret_cast<const float4*>(tab + (size_t)(L + row) * NF_D + c);
+          const float4 z = *reinterpret_cast<const float4*>(vec + V_C2B + c);
+          x.x += y.x + z.x; x.y += y.y + z.y; x.z += y.z + z.z; x.w += y.w + z.w;
+          *reinterpret_cast<float4*>(tab + (size_t)row * NF_D + c) = x;
+        }
+        rw_bar();
+#pragma unroll 1
+        for (int p = 0; p < 2; ++p) {
+          if ((q >> 1) == p) {                      // rows 64p .. 64p+63 belong to quarters 2p, 2p+1
+            const int nr = r - 64 * p;
+            const bool okr = r < LK;
+            const uint8_t* row = stg + nr * 1024;
+            const float* S = tab + (size_t)(okr ? r / K : 0) * NF_D;
+            const float* R = tab + (size_t)(2 * L + (okr ? r % K : 0)) * NF_D;
+#pragma unroll 1
+            for (int j = 0; j < 4; ++j) {
+              const int c0 = 128 * set + 32 * j;
+              float v[32];
+#pragma unroll
+              for (int u = 0; u < 8; ++u) {
+                const float4 x =
+                    *reinterpret_cast<const float4*>(row + ((((c0 >> 2) + u) ^ (nr & 7)) << 4));
+                const float4 y = *reinterpret_cast<const float4*>(S + c0 + 4 * u);
+                const float4 z = *reinterpret_cast<const float4*>(R + c0 + 4 * u);
+                v[4 * u] = okr ? x.x + y.x + z.x : 0.f;
+                v[4 * u + 1] = okr ? x.y + y.y + z.y : 0.f;
+                v[4 * u + 2] = okr ? x.z + y.z + z.z : 0.f;
+                v[4 * u + 3] = okr ? x.w + y.w + z.w : 0.f;
+              }
+              st32f(tx + c0, v);
+            }
+          }
+          rw_bar();                                 // staging free for the next 64 nodes
+          if (p == 0 && LK > 64) {
+            fetch_fold(1);
+            cp_async_wait_all();
+            rw_bar();
+          }
+        }
+        // c1 of this thread's row and column half, 4 columns per step (ACT is free again)
+#pragma unroll 1
+        for (int j = 0; j < 4; ++j) {
+          const int c0 = 128 * set + 32 * j;
+          float c1[32];
+#pragma unroll
+          for (int e = 0; e < 32; e += 4) {
+            float4 z = *reinterpret_cast<const float4*>(vec + V_C1B + c0 + e);
+#pragma unroll
+            for (int i = 0; i < LILICORR_N_CONF; ++i) {
+              const float4 w = *reinterpret_cast<const float4*>(vec + V_C1W + i * NF_D + c0 + e);
+              z.x = fmaf(w.x, f[i], z.x);
+              z.y = fmaf(w.y, f[i], z.y);
+              z.z = fmaf(w.z, f[i], z.z);
+              z.w = fmaf(w.w, f[i], z.w);
+            }
+            c1[e] = ok ? silu_fast(z.x) : 0.f;
+            c1[e + 1] = ok ? silu_fast(z.y) : 0.f;
+            c1[e + 2] = ok ? silu_fast(z.z) : 0.f;
+            c1[e + 3] = ok ? silu_fast(z.w) : 0.f;
+          }
+          put32(sm + OFF_ACT, r, c0, c1);
+        }
+        tmem_wait_st();
+        if (set == 0) s_slot[r] = (uint8_t)min(r / K, L - 1);   // read after the next rw_bar
+        rw_signal(&sh.ready[0], lane);
+      }
+      // ---- Transformer layers
+      for (int l = 0; l < nl; ++l) {
+        ev_wait(&sh.done[l == 0 ? 0 : D_LAYER(l - 1)], par, sh.abort);
+        tc_fence_after();
+        // this layer's vectors (the previous layer's readers are past this barrier)
+        rw_bar();
+        for (int i = tid; i < NF_D; i += NF_RW) {
+          vec[V_AN + i] = a.an[l][i];
+          vec[V_FN + i] = a.fn[l][i];
+          vec[V_BO + i] = a.bo[l][i];
+          vec[V_B2 + (l & 1) * NF_D + i] = a.b2[l][i];
+        }
+        for (int i = tid; i < NF_F; i += NF_RW) vec[V_B1 + i] = a.b1[l][i];
+        for (int i = tid; i < 3 * NF_D; i += NF_RW) vec[V_BQKV + i] = a.bqkv[l][i];
+        for (int i = tid; i < NF_NH * nd; i += NF_RW) s_dist[i] = a.dist[l][i] * LOG2E;
+        if (tid < NF_NH) s_same[tid] = a.same[l][tid] * LOG2E;
+        // x += b_2 of the previous layer (staged then), RMSNorm statistics
+        const float* b2p = l == 0 ? nullptr : vec + V_B2 + ((l - 1) & 1) * NF_D;
+        float rstd = row_rstd(tx, b2p, true, set, r, s_ss);
+        row_normed(sm, tx, nullptr, rstd, vec + V_AN, nullptr, set, r);
+        rw_signal(&sh.ready[R_XN(l)], lane);
+
+        for (int g = 0; g < 4; ++g) {
+          // q | k | v of head 2g+set -> shared memory (bias added, bf16)
+          ev_wait(&sh.done[D_QKV(l, g)], par, sh.abort);
+          tc_fence_after();
+          set_bar(set);                              // the set's previous head is done
+          uint8_t* qs = sm + OFF_HF + set * QKV_SET;
+          const int hh = 2 * g + set;
+#pragma unroll 1
+          for (int part = 0; part < 3; ++part) {
+            float v[32];
+            ld32f(tscr + 64 * part + 32 * set, v);
+            const float* bq = vec + V_BQKV + part * NF_D + hh * NF_HD;
+            const bool zero = part > 0 && r >= LK;   // padded keys and values
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] = zero ? 0.f : v[e] + bq[e];
+            uint8_t* dst = qs + part * 8192;
+#pragma unroll
+            for (int p = 0; p < 4; ++p)
+              *reinterpret_cast<uint4*>(dst + qkv_off(r, p)) = pack8(v + 8 * p);
+          }
+          if (g < 3) rw_signal(&sh.ready[R_QKV_DRAINED(l, g)], lane);
+          set_bar(set);
+          // attention core of head hh: warp wi takes queries 32wi .. 32wi+31
+          const uint32_t qb = smem_u32(qs), kb = qb + 8192, vb = qb + 16384;
+          const int g8 = lane >> 2, t4 = lane & 3;
+          const float qscale = rsqrtf((float)NF_HD) * LOG2E;
+          const float same_l2 = s_same[hh];
+          const float* sd = s_dist + hh * nd + (L - 1);
+          uint8_t* att = sm + OFF_ATT;
+#pragma unroll 1
+          for (int mt = 0; mt < 2; ++mt) {
+            const int q0 = 32 * wi + 16 * mt;
+            uint32_t qa[2][4];
+#pragma unroll
+            for (int ks = 0; ks < 2; ++ks)
+              ldsm_x4(qb + qkv_off(q0 + (lane & 15), ks * 2 + (lane >> 4)), qa[ks]);
+            float s[16][4];
+#pragma unroll
+            for (int nb = 0; nb < 16; ++nb) s[nb][0] = s[nb][1] = s[nb][2] = s[nb][3] = 0.f;
+#pragma unroll
+            for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+              for (int nb = 0; nb < 16; nb += 2) {
+                uint32_t bf[4];
+                const int key = nb * 8 + (lane & 7) + ((lane >> 4) << 3);
+                ldsm_x4(kb + qkv_off(key, ks * 2 + ((lane >> 3) & 1)), bf);
+                mma16816(s[nb], qa[ks], bf[0], bf[1]);
+                mma16816(s[nb + 1], qa[ks], bf[2], bf[3]);
+              }
+            const int i0 = q0 + g8, i1 = i0 + 8;
+            const int si0 = s_slot[i0], si1 = s_slot[i1];
+            float m0 = -INFINITY, m1 = -INFINITY;
+#pragma unroll
+            for (int nb = 0; nb < 16; ++nb) {
+              const int j0 = nb * 8 + 2 * t4;
+              const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int j = j0 + (e & 1);
+                const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
+                const int si = e < 2 ? si0 : si1;
+                const float v = j < LK ? s[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
+                                       : -INFINITY;
+                s[nb][e] = v;
+                if (e < 2) m0 = fmaxf(m0, v); else m1 = fmaxf(m1, v);
+              }
+            }
+            m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 1));
+            m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 2));
+            m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 1));
+            m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 2));
+            float l0 = 0.f, l1 = 0.f;
+            uint32_t pa[8][4];
+#pragma unroll
+            for (int nb = 0; nb < 16; ++nb) {
+              const float p0 = ex2f(s[nb][0] - m0), p1 = ex2f(s[nb][1] - m0);
+              const float p2 = ex2f(s[nb][2] - m1), p3 = ex2f(s[nb][3] - m1);
+              l0 += p0 + p1;
+              l1 += p2 + p3;
+              const int kk = nb >> 1;
+              if ((nb & 1) == 0) {
+                pa[kk][0] = pack_bf16x2(p0, p1);
+                pa[kk][1] = pack_bf16x2(p2, p3);
+              } else {
+                pa[kk][2] = pack_bf16x2(p0, p1);
+                pa[kk][3] = pack_bf16x2(p2, p3);
+              }
+            }
+            float o[4][4];
+#pragma unroll
+            for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+              for (int nb = 0; nb < 4; nb += 2) {
+                uint32_t vf[4];
+                const int key = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                ldsm_x4_t(vb + qkv_off(key, nb + (lane >> 4)), vf);
+                mma16816(o[nb], pa[kk], vf[0], vf[1]);
+                mma16816(o[nb + 1], pa[kk], vf[2], vf[3]);
+              }
+            l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+            l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+            l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+            const float inv0 = 1.0f / l0, inv1 = 1.0f / l1;
+            // the attention-output buffer is free once the previous pair's W_o product ran
+            if (mt == 0 && g > 0) ev_wait(&sh.done[D_WO(l, g - 1)], par, sh.abort);
+#pragma unroll
+            for (int nb = 0; nb < 4; ++nb) {
+              const int piece = 4 * set + nb;
+              *reinterpret_cast<uint32_t*>(att + swz(i0, piece) + 4 * t4) =
+                  pack_bf16x2(o[nb][0] * inv0, o[nb][1] * inv0);
+              *reinterpret_cast<uint32_t*>(att + swz(i1, piece) + 4 * t4) =
+                  pack_bf16x2(o[nb][2] * inv1, o[nb][3] * inv1);
+            }
+          }
+          rw_signal(&sh.ready[R_ATT(l, g)], lane);
+        }
+        // ---- FFN: x += b_o, xn2 = RMSNorm(x)
+        ev_wait(&sh.done[D_WO(l, 3)], par, sh.abort);
+        tc_fence_after();
+        rstd = row_rstd(tx, vec + V_BO, true, set, r, s_ss);
+        row_normed(sm, tx, nullptr, rstd, vec + V_FN, nullptr, set, r);
+        rw_signal(&sh.ready[R_XN2(l)], lane);
+        ev_wait(&sh.done[D_FFN(l, 0)], par, sh.abort);
+        tc_fence_after();
+        drain_silu(sm + OFF_HF, tscr, vec + V_B1, nullptr, set, r);
+        rw_signal(&sh.ready[R_HFA(l)], lane);
+        ev_wait(&sh.done[D_FFN(l, 1)], par, sh.abort);
+        tc_fence_after();
+        drain_silu(sm + OFF_ACT, tscr, vec + V_B1 + 256, nullptr, set, r);
+        rw_signal(&sh.ready[R_HFB(l)], lane);
+      }
+      // ---- fusion: xf = RMSNorm(x + b_2) -> ACT, xf * t -> HF; u = SiLU(. + cb) -> ACT
+      ev_wait(&sh.done[D_LAYER(nl - 1)], par, sh.abort);
+      tc_fence_after();
+      {
+        const float* b2l = vec + V_B2 + ((nl - 1) & 1) * NF_D;
+        const float rstd = row_rstd(tx, b2l, false, set, r, s_ss);
+        row_normed(sm, tx, b2l, rstd, vec + V_FIN, vec + V_T, set, r);
+      }
+      rw_signal(&sh.ready[lb(nl)], lane);
+      ev_wait(&sh.done[lb(nl)], par, sh.abort);
+      tc_fence_after();
+      drain_silu(sm + OFF_ACT, tscr, vec + V_CB, nullptr, set, r);
+      rw_signal(&sh.ready[lb(nl) + 1], lane);
+      // ---- out / in heads: 256 columns of [o | i] at a time -> oi (fp32, not yet unit).
+      // Each column half goes through a staging buffer (128 rows x 128 floats, pieces
+      // swizzled by row) so that the global stores are row-contiguous.
+      for (int h = 0; h * 256 < a.d2; ++h) {
+        ev_wait(&sh.done[lb(nl) + 1 + h], par, sh.abort);
+        tc_fence_after();
+        uint8_t* stg = sm + OFF_HF;
+        const int wr = warp - 2;
+#pragma unroll 1
+        for (int hs = 0; hs < 2; ++hs) {
+          if (set == hs) {
+#pragma unroll 1
+            for (int j = 0; j < 4; ++j) {
+              float v[32];
+              ld32f(tscr + 128 * hs + 32 * j, v);
+              const float* bo = vec + V_BOI + 256 * h + 128 * hs + 32 * j;
+#pragma unroll
+              for (int u = 0; u < 8; ++u)
+                *reinterpret_cast<float4*>(stg + r * 512 + (((8 * j + u) ^ (r & 7)) << 4)) =
+                    make_float4(v[4 * u] + bo[4 * u], v[4 * u + 1] + bo[4 * u + 1],
+                                v[4 * u + 2] + bo[4 * u + 2], v[4 * u + 3] + bo[4 * u + 3]);
+            }
+          }
+          rw_bar();
+          for (int row = wr; row < LK; row += NF_RW / 32)
+            *reinterpret_cast<float4*>(a.oi + ((size_t)b * LK + row) * a.d2 + 256 * h + 128 * hs +
+                                       4 * lane) =
+                *reinterpret_cast<const float4*>(stg + row * 512 + ((lane ^ (row & 7)) << 4));
+          rw_bar();
+        }
+        if ((h + 1) * 256 < a.d2) rw_signal(&sh.ready[lb(nl) + 2 + h], lane);
+      }
+      tc_fence_before();
+      rw_bar();                                      // s_dist / s_ss reuse by the next sequence
+    }
+  }
+
+  // ---- teardown
+  tc_fence_before();
+  __syncthreads();
+  if (abort_flag) {
+    if (threadIdx.x == 0) {
+      set_status(a.status, LILICORR_ERR_TIMEOUT);
+      const long long t0 = clock64();            // let copies and products in flight land
+      while (clock64() - t0 < WAIT_LIMIT / 10) {
+      }
+    }
+    __syncthreads();
+  }
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+}  // namespace
+
+// ----------------------------------------------------------------------------- host side
+struct NetFusedMaps {
+  NetMaps m;
+};
+
+bool net_fused_supported(const lilicorr_head_desc& d) {
+  return d.dtype == LILICORR_BF16 && d.D == NF_D && d.ffn == NF_F && d.n_heads == NF_NH &&
+         d.n_layers >= 1 && d.n_layers <= NF_MAX_LAYERS && d.L >= 1 && d.L <= NF_MAX_L &&
+         d.K >= 1 && d.L * d.K <= NF_M && 2 * d.L + d.K <= 64 &&   // node tables fit in ACT
+         (2 * d.d) % 256 == 0 && 2 * d.d <= 512 &&
+         encode_fn() != nullptr;
+}
+
+namespace {
+// W [rows, cols] bf16 row-major as (64, rows, cols / 64): box (64, box_rows, 1) is one K chunk
+// of box_rows rows, 128-byte swizzled.
+bool chunk_map(CUtensorMap* m, const void* W, int rows, int cols, int box_rows) {
+  const uint64_t dims[3] = {64, (uint64_t)rows, (uint64_t)(cols / 64)};
+  const uint64_t strides[3] = {2, (uint64_t)cols * 2, 128};
+  const uint32_t box[3] = {64, (uint32_t)box_rows, 1};
+  return make_map_nd(m, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, dims, strides, box);
+}
+// W_qkv [3D, D] as (64 k, 64 rows, 4 head pairs, 3 parts q/k/v, D / 64 chunks): box
+// (64, 64, 1, 3, 1) brings the q, k and v rows of one head pair for one K chunk.
+bool qkv_map(CUtensorMap* m, const void* W) {
+  const uint64_t dims[5] = {64, 64, NF_D / 64, 3, NF_D / 64};
+  const uint64_t strides[5] = {2, NF_D * 2, 64ull * NF_D * 2, (uint64_t)NF_D * NF_D * 2, 128};
+  const uint32_t box[5] = {64, 64, 1, 3, 1};
+  return make_map_nd(m, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, dims, strides, box);
+}
+}  // namespace
+
+void* net_fused_maps_create(const lilicorr_head* h) {
+  const lilicorr_head_desc& d = h->desc;
+  if (!net_fused_supported(d)) return nullptr;
+  NetFusedMaps* nm = new (std::nothrow) NetFusedMaps;
+  if (!nm) return nullptr;
+  memset(nm, 0, sizeof(*nm));
+  bool ok = chunk_map(&nm->m.conf2, h->conf2_w, NF_D, NF_D, 256) &&
+            chunk_map(&nm->m.fuse, h->fuse_x, NF_D, 2 * NF_D, 256) &&
+            chunk_map(&nm->m.woi, h->woi, 2 * d.d, NF_D, 256);
+  for (int l = 0; l < d.n_layers && ok; ++l) {
+    const HeadW& w = h->layer[l];
+    ok = qkv_map(&nm->m.wqkv[l], w.wqkv) && chunk_map(&nm->m.wo[l], w.wo, NF_D, NF_D, 256) &&
+         chunk_map(&nm->m.w1[l], w.w1, NF_F, NF_D, 256) &&
+         chunk_map(&nm->m.w2[l], w.w2, NF_D, NF_F, 256);
+  }
+  for (int l = d.n_layers; l < NF_MAX_LAYERS && ok; ++l) {   // unused slots: valid maps
+    nm->m.wqkv[l] = nm->m.wqkv[0];
+    nm->m.wo[l] = nm->m.wo[0];
+    nm->m.w1[l] = nm->m.w1[0];
+    nm->m.w2[l] = nm->m.w2[0];
+  }
+  if (!ok) {
+    delete nm;
+    return nullptr;
+  }
+  return nm;
+}
+
+void net_fused_maps_free(void* p) { delete static_cast<NetFusedMaps*>(p); }
+
+lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t* ids,
+                                   const float* logp, const float* hproj, const float* t,
+                                   const float* cb, float* oi, uint32_t* status, cudaStream_t st) {
+  if (B == 0) return LILICORR_OK;
+  const NetFusedMaps* nm = static_cast<const NetFusedMaps*>(h->net_maps);
+  if (!nm) return LILICORR_ERR_SHAPE;
+  const lilicorr_head_desc& d = h->desc;
+  NetArgs a;
+  memset(&a, 0, sizeof(a));
+  a.B = B; a.L = d.L; a.K = d.K; a.LK = d.L * d.K; a.V = d.V; a.n_layers = d.n_layers;
+  a.d2 = 2 * d.d;
+  a.ids = ids; a.logp = logp; a.hproj = hproj; a.t = t; a.cb = cb;
+  a.fold = static_cast<const float*>(h->fold);
+  a.slot = h->slot; a.rank = h->rank;
+  a.conf1_w = h->conf1_w; a.conf1_b = h->conf1_b; a.conf2_b = h->conf2_b;
+  for (int l = 0; l < NF_MAX_LAYERS; ++l) {
+    const HeadW& w = h->layer[l < d.n_layers ? l : 0];
+    a.bqkv[l] = w.bqkv; a.bo[l] = w.bo; a.b1[l] = w.b1; a.b2[l] = w.b2;
+    a.an[l] = w.an; a.fn[l] = w.fn; a.dist[l] = w.dist; a.same[l] = w.same;
+  }
+  a.final_norm = h->final_norm;
+  a.boi = h->boi;
+  a.oi = oi;
+  a.status = status;
+  static bool configured[64] = {false};
+  LL_TRY(allow_max_dynamic_smem(net_fused_kernel, configured));
+  const int grid = B < num_sms() ? B : num_sms();
+  net_fused_kernel<<<grid, NF_THREADS, NF_SMEM, st>>>(nm->m, a);
+  return last_launch();
+}
+
+}  // namespace lilicorr
