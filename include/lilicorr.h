@@ -28,10 +28,11 @@
  *   - Workspaces must be zero-filled once before first use (lilicorr_workspace_init);
  *     every call leaves them reusable. Two calls that run concurrently must not
  *     share a workspace.
- *   - lilicorr_select_block runs the candidate-independent projections on a side
- *     stream owned by the head, forked from and joined back to the caller's stream
- *     (a fork/join node pair under graph capture). Calls that use one head must be
- *     issued from one host thread at a time.
+ *   - lilicorr_select_block and lilicorr_embed_in_out run the candidate-independent
+ *     projections on two side streams owned by the head (the drafter-state
+ *     projection on one, the target-state chain on the other), forked from and
+ *     joined back to the caller's stream (fork/join nodes under graph capture).
+ *     Calls that use one head must be issued from one host thread at a time.
  */
 #ifndef LILICORR_H_
 #define LILICORR_H_

@@ -26,13 +26,13 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
                                        const float* bias, const float* residual, int act, int path,
                                        uint32_t* status, cudaStream_t stream);
 
-/* Switch for the fused scoring-network kernel (one CTA per sequence; used on bf16
- * heads with D = 256, 8 heads, FFN 2D and L*K <= 128). enable = 1 (the default)
- * lets such heads use it, 0 sends every head through the unfused chain of kernels,
- * so a test can run both on the same inputs. Process-wide; set it between calls,
- * not while another thread is enqueueing. Returns 1 if `head` (may be NULL) takes
- * the fused kernel when it is enabled, else 0. */
-int lilicorr_test_fused_path(const lilicorr_head* head, int enable);
+/* Switch for the fused scoring-network kernel (one CTA per sequence; bf16 heads with
+ * D = 256, 8 heads, FFN 2D, L*K <= 128 and 2L + K <= 64). mode 1 (the default) uses
+ * it for calls of 8 or more sequences, mode 2 for every call, mode 0 never, so a test
+ * can run both paths on the same inputs. Process-wide; set it between calls, not
+ * while another thread is enqueueing. Returns 1 if `head` (may be NULL) can take the
+ * fused kernel, else 0. */
+int lilicorr_test_fused_path(const lilicorr_head* head, int mode);
 
 #ifdef __cplusplus
 }

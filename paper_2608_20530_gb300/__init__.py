@@ -343,11 +343,12 @@ def test_linear(A: torch.Tensor, W: torch.Tensor, out_dtype=torch.float32, bias=
     return C
 
 
-def test_fused_path(head: Optional[Head], enable: bool) -> bool:
-    """Test hook: allow (True) or forbid (False) the fused scoring-network kernel for
-    every head in the process; returns whether ``head`` takes it when allowed."""
+def test_fused_path(head: Optional[Head], mode: int) -> bool:
+    """Test hook: the fused scoring-network kernel for every head in the process is used
+    never (0), from 8 sequences on (1, the default) or always (2); returns whether
+    ``head`` can take it."""
     h = head._h if head is not None else _P()
-    return bool(lib().lilicorr_test_fused_path(h, 1 if enable else 0))
+    return bool(lib().lilicorr_test_fused_path(h, int(mode)))
 
 
 def select_block_intermediates(head: Head, B: int, ws: Workspace) -> Dict[str, torch.Tensor]:

@@ -253,35 +253,55 @@ struct HeadCall {
   }
 };
 
-// Candidate-independent part of the scoring network (Sec. 3.2; App. A): the drafter
-// state projection, the target state, the anchor out vector and the fusion layer's t block.
-lilicorr_status_t run_prologue(const HeadCall& c, const void* hidden, const void* target,
-                               cudaStream_t st) {
+// Candidate-independent part of the scoring network (Sec. 3.2; App. A), two chains.
+// (a) the drafter state projection W_h h_s + b_h, one row per slot.
+lilicorr_status_t run_drafter_proj(const HeadCall& c, const void* hidden, cudaStream_t st) {
+  const lilicorr_head* h = c.h;
+  const lilicorr_head_desc& d = c.d;
+  GemmArgs g = c.G(hidden, c.wdt, d.H, h->hid_w, d.H, c.hproj, LILICORR_F32, c.D, c.R, c.D, d.H);
+  g.bias = h->hid_b;
+  return run_gemm(g, st);
+}
+// (b) the target state t = W_t RMSNorm(mean of the captured layers) + b_t, the anchor out
+// vector W_a t + b_a (its consumers normalise it) and the fusion layer's t block, constant
+// per sequence: cb = W_f[:, t] t + b_f.
+lilicorr_status_t run_target(const HeadCall& c, const void* target, cudaStream_t st) {
   const lilicorr_head* h = c.h;
   const lilicorr_head_desc& d = c.d;
   const lilicorr_dtype_t F32 = LILICORR_F32;
   const int D = c.D;
-  // drafter state projection W_h h_s + b_h, one row per slot (shared by its K candidates)
-  GemmArgs g = c.G(hidden, c.wdt, d.H, h->hid_w, d.H, c.hproj, F32, D, c.R, D, d.H);
-  g.bias = h->hid_b;
-  LL_TRY(run_gemm(g, st));
-  // target state t = W_t RMSNorm(mean of the captured layers) + b_t
   LL_TRY(launch_target_norm(target, c.wdt, c.B, d.n_tgt, d.H, h->tgt_norm, c.tn, c.tn_dt, st));
-  g = c.G(c.tn, c.tn_dt, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
+  GemmArgs g = c.G(c.tn, c.tn_dt, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
   g.bias = h->tgt_b;
   LL_TRY(run_gemm(g, st));
-  // anchor out vector o_0 = unit(W_a t + b_a)
   g = c.G(c.t, F32, D, h->anc_w, D, c.anc, F32, d.d, c.B, d.d, D);
   g.bias = h->anc_b;
   LL_TRY(run_gemm(g, st));
-  LL_TRY(launch_unit_rows(c.anc, c.B, d.d, d.d, c.anc, d.d, st));
-  // the t block of the fusion layer is constant per sequence: cb = W_f[:, t] t + b_f
   g = c.G(c.t, F32, D, h->fuse_t, D, c.cb, F32, D, c.B, D, D);
   g.bias = h->fuse_b;
   return run_gemm(g, st);
 }
+// Fork both chains from `st` onto the head's side streams; join_prologue makes `st` wait
+// for them. The joins are recorded even when a launch fails, so a capture stays balanced.
+lilicorr_status_t fork_prologue(const HeadCall& c, const void* hidden, const void* target,
+                                cudaStream_t st) {
+  lilicorr_head* hm = const_cast<lilicorr_head*>(c.h);
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_fork, st));
+  LL_CUDA_TRY(cudaStreamWaitEvent(hm->side, hm->ev_fork, 0));
+  LL_CUDA_TRY(cudaStreamWaitEvent(hm->side2, hm->ev_fork, 0));
+  const lilicorr_status_t s1 = run_drafter_proj(c, hidden, hm->side);
+  const lilicorr_status_t s2 = run_target(c, target, hm->side2);
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_join, hm->side));
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_join2, hm->side2));
+  return s1 != LILICORR_OK ? s1 : s2;
+}
+lilicorr_status_t join_prologue(const lilicorr_head* h, cudaStream_t st) {
+  LL_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_join, 0));
+  LL_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_join2, 0));
+  return LILICORR_OK;
+}
 
-// Candidate-dependent part, after run_prologue: nodes, the Transformer, fusion and the
+// Candidate-dependent part, after the prologue: nodes, the Transformer, fusion and the
 // out/in heads. Writes oi = [W_o u + b_o | W_i u + b_i] (not yet normalised).
 lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* logp,
                            cudaStream_t st) {
@@ -289,7 +309,9 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   const lilicorr_head_desc& d = c.d;
   const lilicorr_dtype_t F32 = LILICORR_F32, adt = c.adt;
   const int D = c.D, F = c.F, N = c.N;
-  if (h->net_maps && g_fused_enabled)
+  // the fused kernel puts a sequence on one SM: it wins once several sequences share the
+  // GPU; a lone sequence runs faster as the chain of kernels below, each spread over SMs
+  if (h->net_maps && (g_fused_enabled == 2 || (g_fused_enabled == 1 && c.B >= FUSED_MIN_B)))
     return launch_net_fused(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
   LL_TRY(launch_node_build(h, c.B, ids, logp, c.hproj, c.c1, adt, c.x, c.status, st));
@@ -341,7 +363,9 @@ lilicorr_status_t run_head(const lilicorr_head* h, int B, const int32_t* ids, co
                            const void* hidden, const void* target, void* ws, const WsLayout& w,
                            cudaStream_t st) {
   const HeadCall c(h, B, ws, w);
-  LL_TRY(run_prologue(c, hidden, target, st));
+  const lilicorr_status_t sp = fork_prologue(c, hidden, target, st);
+  LL_TRY(join_prologue(h, st));
+  LL_TRY(sp);
   return run_body(c, ids, logp, st);
 }
 
@@ -447,14 +471,18 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
     if (embed_dev) cudaFree(embed_dev);
     if (h->pool) cudaFree(h->pool);
     if (h->side) cudaStreamDestroy(h->side);
+    if (h->side2) cudaStreamDestroy(h->side2);
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
     if (h->ev_join) cudaEventDestroy(h->ev_join);
+    if (h->ev_join2) cudaEventDestroy(h->ev_join2);
     free(h);
     return s;
   };
   if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->side2, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess)
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join2, cudaEventDisableTiming) != cudaSuccess)
     return fail(LILICORR_ERR_CUDA);
   if (cudaMalloc(&h->pool, pool_bytes) != cudaSuccess) return fail(LILICORR_ERR_CUDA);
   h->pool_bytes = pool_bytes;
@@ -510,8 +538,10 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   cudaError_t e = cudaFree(h->pool);
   net_fused_maps_free(h->net_maps);
   if (h->side) cudaStreamDestroy(h->side);
+  if (h->side2) cudaStreamDestroy(h->side2);
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
   if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->ev_join2) cudaEventDestroy(h->ev_join2);
   if (cur != h->device) cudaSetDevice(cur);
   free(h);
   return e == cudaSuccess ? LILICORR_OK : LILICORR_ERR_CUDA;
@@ -631,17 +661,14 @@ lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const 
   int32_t* ids = at<int32_t>(ws, w.ids);
   float* logp = at<float>(ws, w.logp);
   // the candidate-independent projections run beside the top-K pass
-  lilicorr_head* hm = const_cast<lilicorr_head*>(head);
-  LL_CUDA_TRY(cudaEventRecord(hm->ev_fork, stream));
-  LL_CUDA_TRY(cudaStreamWaitEvent(hm->side, hm->ev_fork, 0));
   const HeadCall call(head, B, ws, w);
-  const lilicorr_status_t sp = run_prologue(call, drafter_hidden, target_hidden, hm->side);
-  LL_CUDA_TRY(cudaEventRecord(hm->ev_join, hm->side));     // always rejoin, even on error
-  LL_TRY(sp);
-  LL_TRY(launch_topk_lse(logits, d.dtype, R, d.V, d.K, ids, logp, at<float>(ws, w.lse),
-                         at<uint32_t>(ws, w.status), at<uint32_t>(ws, w.counters),
-                         at<void>(ws, w.partials), stream));
-  LL_CUDA_TRY(cudaStreamWaitEvent(stream, hm->ev_join, 0));
+  const lilicorr_status_t sp = fork_prologue(call, drafter_hidden, target_hidden, stream);
+  const lilicorr_status_t st = sp != LILICORR_OK ? sp
+      : launch_topk_lse(logits, d.dtype, R, d.V, d.K, ids, logp, at<float>(ws, w.lse),
+                        at<uint32_t>(ws, w.status), at<uint32_t>(ws, w.counters),
+                        at<void>(ws, w.partials), stream);
+  LL_TRY(join_prologue(head, stream));                      // always rejoin, even on error
+  LL_TRY(st);
   LL_TRY(run_body(call, ids, logp, stream));
   PairWalkArgs a;
   memset(&a, 0, sizeof(a));
@@ -693,8 +720,8 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
   return LILICORR_ERR_ARG;
 }
 
-int lilicorr_test_fused_path(const lilicorr_head* head, int enable) {
-  g_fused_enabled = enable ? 1 : 0;
+int lilicorr_test_fused_path(const lilicorr_head* head, int mode) {
+  g_fused_enabled = mode < 0 ? 0 : mode > 2 ? 2 : mode;
   return head && head->net_maps ? 1 : 0;
 }
 

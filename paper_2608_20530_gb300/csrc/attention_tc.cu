@@ -56,6 +56,7 @@ __global__ void __launch_bounds__(AT_WARPS * 32)
 attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D, int n_heads,
                      const float* __restrict__ dist, const float* __restrict__ same,
                      __nv_bfloat16* __restrict__ out) {
+  pdl_wait();
   constexpr int HP = HD + 8;                 // padded row, elements
   constexpr int KS = HD / 16;                // k-steps of Q K^T
   constexpr int NB = HD / 8;                 // 8-wide dim blocks of O
@@ -222,9 +223,9 @@ lilicorr_status_t launch_hd(const __nv_bfloat16* qkv, int B, int L, int K, int D
   const size_t smem = sizeof(__nv_bfloat16) * (size_t)(2 * LKp + AT_QROWS) * (HD + 8) +
                       sizeof(float) * (2 * L - 1);
   dim3 grid(B * n_heads, ceil_div(LK, AT_QROWS));
-  attention_mma_kernel<HD><<<grid, AT_WARPS * 32, smem, st>>>(qkv, L, K, D, n_heads, dist, same,
-                                                               out);
-  return last_launch();
+  LL_TRY(launch_k(attention_mma_kernel<HD>, grid, AT_WARPS * 32, smem, st, qkv, L, K, D, n_heads, dist, same,
+                                                               out));
+  return LILICORR_OK;
 }
 
 }  // namespace

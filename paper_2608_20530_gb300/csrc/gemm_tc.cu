@@ -104,6 +104,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base;
+  pdl_wait();                      // inputs come from the preceding launch
 
   if (warp == 0) {
     // ---- producer: TMA into the stage ring, tile after tile
@@ -301,9 +302,9 @@ lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   ep.act = g.act;
   const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<BN, OUT_BF16><<<grid, TC_THREADS, Cfg::SMEM, st>>>(ma, mw, mc, mr, ep, g.M, g.N,
-                                                                     g.Kd, g.status);
-  return last_launch();
+  LL_TRY(launch_k(gemm_tc_kernel<BN, OUT_BF16>, grid, TC_THREADS, Cfg::SMEM, st, ma, mw, mc, mr, ep, g.M, g.N,
+                                                                     g.Kd, g.status));
+  return LILICORR_OK;
 }
 
 template <bool OUT_BF16>

@@ -19,6 +19,7 @@ constexpr int GB_M = 64, GB_N = 64, GB_K = 16, G_THREADS = 256;
 
 template <typename TA, typename TW, typename TC>
 __global__ void __launch_bounds__(G_THREADS) gemm_simt_kernel(GemmArgs g) {
+  pdl_wait();
   __shared__ float As[GB_K][GB_M + 4];
   __shared__ __align__(16) float Ws[GB_K][GB_N + 4];
   const TA* A = static_cast<const TA*>(g.A);
@@ -79,9 +80,9 @@ __global__ void __launch_bounds__(G_THREADS) gemm_simt_kernel(GemmArgs g) {
 
 template <typename TA, typename TW>
 lilicorr_status_t gemm_dispatch_c(const GemmArgs& g, dim3 grid, cudaStream_t st) {
-  if (g.c_dt == LILICORR_F32) gemm_simt_kernel<TA, TW, float><<<grid, G_THREADS, 0, st>>>(g);
-  else gemm_simt_kernel<TA, TW, __nv_bfloat16><<<grid, G_THREADS, 0, st>>>(g);
-  return last_launch();
+  if (g.c_dt == LILICORR_F32) LL_TRY(launch_k(gemm_simt_kernel<TA, TW, float>, grid, G_THREADS, 0, st, g));
+  else LL_TRY(launch_k(gemm_simt_kernel<TA, TW, __nv_bfloat16>, grid, G_THREADS, 0, st, g));
+  return LILICORR_OK;
 }
 template <typename TA>
 lilicorr_status_t gemm_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st) {
@@ -113,6 +114,7 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
 
 template <typename TA, typename TW, typename TC>
 __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
+  pdl_wait();
   __shared__ float red[SK_THREADS / 32][SK_MB * SK_NB];
   const TA* A = static_cast<const TA*>(g.A);
   const TW* W = static_cast<const TW*>(g.W);
@@ -175,9 +177,9 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
 
 template <typename TA, typename TW>
 lilicorr_status_t skinny_dispatch_c(const GemmArgs& g, dim3 grid, cudaStream_t st) {
-  if (g.c_dt == LILICORR_F32) gemm_skinny_kernel<TA, TW, float><<<grid, SK_THREADS, 0, st>>>(g);
-  else gemm_skinny_kernel<TA, TW, __nv_bfloat16><<<grid, SK_THREADS, 0, st>>>(g);
-  return last_launch();
+  if (g.c_dt == LILICORR_F32) LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, float>, grid, SK_THREADS, 0, st, g));
+  else LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, __nv_bfloat16>, grid, SK_THREADS, 0, st, g));
+  return LILICORR_OK;
 }
 template <typename TA>
 lilicorr_status_t skinny_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st) {
@@ -195,6 +197,7 @@ template <typename T, typename TO>
 __global__ void __launch_bounds__(TN_THREADS)
 target_norm_kernel(const T* __restrict__ Tin, int n_tgt, int H, const float* __restrict__ gain,
                    TO* __restrict__ tn) {
+  pdl_wait();
   __shared__ float red[TN_THREADS / 32];
   __shared__ float s_total;
   const int b = blockIdx.x;
@@ -276,6 +279,7 @@ __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __r
                                   const float* __restrict__ rank, const float* __restrict__ w1,
                                   const float* __restrict__ b1, TC1* __restrict__ c1,
                                   float* __restrict__ x, uint32_t* status) {
+  pdl_wait();
   __shared__ float f[LILICORR_MAX_K][LILICORR_N_CONF];
   __shared__ int sid[LILICORR_MAX_K];
   const int r = blockIdx.x;
@@ -327,6 +331,7 @@ __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __r
 template <typename TY>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int D,
                                const float* __restrict__ gain, TY* __restrict__ y) {
+  pdl_wait();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
@@ -344,6 +349,7 @@ template <typename TY>
 __global__ void fusion_input_kernel(const float* __restrict__ x, int M, int LK, int D,
                                     const float* __restrict__ gain, const float* __restrict__ t,
                                     TY* __restrict__ fin) {
+  pdl_wait();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
@@ -363,6 +369,7 @@ __global__ void fusion_input_kernel(const float* __restrict__ x, int M, int LK, 
 // dst[row] = src[row] / max(||src[row]||, 1e-12), rows of n floats.
 __global__ void unit_rows_kernel(const float* __restrict__ src, int rows, int n, int ld_src,
                                  float* __restrict__ dst, int ld_dst) {
+  pdl_wait();
   const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -382,6 +389,7 @@ template <typename TO>
 __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, int D, int n_heads,
                                  int q_per_cta, const float* __restrict__ dist,
                                  const float* __restrict__ same, TO* __restrict__ out) {
+  pdl_wait();
   extern __shared__ float sm[];
   const int LK = L * K, hd = D / n_heads;
   const int b = blockIdx.x / n_heads, h = blockIdx.x % n_heads;
@@ -469,17 +477,17 @@ lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, 
                                      cudaStream_t st) {
   if (B == 0) return LILICORR_OK;
   if (dt == LILICORR_F32 && tn_dt == LILICORR_F32)
-    target_norm_kernel<float, float><<<B, TN_THREADS, 0, st>>>(
-        static_cast<const float*>(T), n_tgt, H, gain, static_cast<float*>(tn));
+    LL_TRY(launch_k(target_norm_kernel<float, float>, B, TN_THREADS, 0, st, 
+        static_cast<const float*>(T), n_tgt, H, gain, static_cast<float*>(tn)));
   else if (dt == LILICORR_BF16 && tn_dt == LILICORR_F32)
-    target_norm_kernel<__nv_bfloat16, float><<<B, TN_THREADS, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<float*>(tn));
+    LL_TRY(launch_k(target_norm_kernel<__nv_bfloat16, float>, B, TN_THREADS, 0, st, 
+        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<float*>(tn)));
   else if (dt == LILICORR_BF16)
-    target_norm_kernel<__nv_bfloat16, __nv_bfloat16><<<B, TN_THREADS, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<__nv_bfloat16*>(tn));
+    LL_TRY(launch_k(target_norm_kernel<__nv_bfloat16, __nv_bfloat16>, B, TN_THREADS, 0, st, 
+        static_cast<const __nv_bfloat16*>(T), n_tgt, H, gain, static_cast<__nv_bfloat16*>(tn)));
   else
     return LILICORR_ERR_DTYPE;
-  return last_launch();
+  return LILICORR_OK;
 }
 
 lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t* ids,
@@ -490,14 +498,14 @@ lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t
   if (B == 0) return LILICORR_OK;
   const float* fold = static_cast<const float*>(h->fold);
   if (c1_dt == LILICORR_F32)
-    node_build_kernel<float><<<B * d.L, 256, 0, st>>>(d.L, d.K, d.D, d.V, ids, logp, fold, hproj,
+    LL_TRY(launch_k(node_build_kernel<float>, B * d.L, 256, 0, st, d.L, d.K, d.D, d.V, ids, logp, fold, hproj,
                                                       h->slot, h->rank, h->conf1_w, h->conf1_b,
-                                                      static_cast<float*>(c1), x, status);
+                                                      static_cast<float*>(c1), x, status));
   else
-    node_build_kernel<__nv_bfloat16><<<B * d.L, 256, 0, st>>>(
+    LL_TRY(launch_k(node_build_kernel<__nv_bfloat16>, B * d.L, 256, 0, st, 
         d.L, d.K, d.D, d.V, ids, logp, fold, hproj, h->slot, h->rank, h->conf1_w, h->conf1_b,
-        static_cast<__nv_bfloat16*>(c1), x, status);
-  return last_launch();
+        static_cast<__nv_bfloat16*>(c1), x, status));
+  return LILICORR_OK;
 }
 
 lilicorr_status_t launch_rmsnorm(const float* x, int M, int D, const float* gain, void* y,
@@ -505,11 +513,11 @@ lilicorr_status_t launch_rmsnorm(const float* x, int M, int D, const float* gain
   if (M == 0) return LILICORR_OK;
   const int grid = ceil_div(M, 8);
   if (y_dt == LILICORR_F32)
-    rmsnorm_kernel<float><<<grid, 256, 0, st>>>(x, M, D, gain, static_cast<float*>(y));
+    LL_TRY(launch_k(rmsnorm_kernel<float>, grid, 256, 0, st, x, M, D, gain, static_cast<float*>(y)));
   else
-    rmsnorm_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, M, D, gain,
-                                                        static_cast<__nv_bfloat16*>(y));
-  return last_launch();
+    LL_TRY(launch_k(rmsnorm_kernel<__nv_bfloat16>, grid, 256, 0, st, x, M, D, gain,
+                                                        static_cast<__nv_bfloat16*>(y)));
+  return LILICORR_OK;
 }
 
 lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, const float* gain,
@@ -519,18 +527,18 @@ lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, cons
   if (M == 0) return LILICORR_OK;
   const int grid = ceil_div(M, 8);
   if (dt == LILICORR_F32)
-    fusion_input_kernel<float><<<grid, 256, 0, st>>>(x, M, LK, D, gain, t, static_cast<float*>(fin));
+    LL_TRY(launch_k(fusion_input_kernel<float>, grid, 256, 0, st, x, M, LK, D, gain, t, static_cast<float*>(fin)));
   else
-    fusion_input_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(x, M, LK, D, gain, t,
-                                                             static_cast<__nv_bfloat16*>(fin));
-  return last_launch();
+    LL_TRY(launch_k(fusion_input_kernel<__nv_bfloat16>, grid, 256, 0, st, x, M, LK, D, gain, t,
+                                                             static_cast<__nv_bfloat16*>(fin)));
+  return LILICORR_OK;
 }
 
 lilicorr_status_t launch_unit_rows(const float* src, int rows, int n, int ld_src, float* dst,
                                    int ld_dst, cudaStream_t st) {
   if (rows == 0) return LILICORR_OK;
-  unit_rows_kernel<<<ceil_div(rows, 8), 256, 0, st>>>(src, rows, n, ld_src, dst, ld_dst);
-  return last_launch();
+  LL_TRY(launch_k(unit_rows_kernel, ceil_div(rows, 8), 256, 0, st, src, rows, n, ld_src, dst, ld_dst));
+  return LILICORR_OK;
 }
 
 lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D, int n_heads,
@@ -550,12 +558,12 @@ lilicorr_status_t launch_attention(const float* qkv, int B, int L, int K, int D,
   qblocks = ceil_div(LK, q_per_cta);
   dim3 grid(B * n_heads, qblocks);
   if (out_dt == LILICORR_F32)
-    attention_kernel<float><<<grid, warps * 32, smem, st>>>(qkv, L, K, D, n_heads, q_per_cta, dist,
-                                                            same, static_cast<float*>(out));
+    LL_TRY(launch_k(attention_kernel<float>, grid, warps * 32, smem, st, qkv, L, K, D, n_heads, q_per_cta, dist,
+                                                            same, static_cast<float*>(out)));
   else
-    attention_kernel<__nv_bfloat16><<<grid, warps * 32, smem, st>>>(
-        qkv, L, K, D, n_heads, q_per_cta, dist, same, static_cast<__nv_bfloat16*>(out));
-  return last_launch();
+    LL_TRY(launch_k(attention_kernel<__nv_bfloat16>, grid, warps * 32, smem, st, 
+        qkv, L, K, D, n_heads, q_per_cta, dist, same, static_cast<__nv_bfloat16*>(out)));
+  return LILICORR_OK;
 }
 
 }  // namespace lilicorr

@@ -2,6 +2,8 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <string.h>
+#include <utility>
 #include <cuda_bf16.h>
 #include <stdint.h>
 #include <stddef.h>
@@ -32,6 +34,42 @@ void count_launch();   // host-side launch counter (lilicorr_launch_count)
 inline lilicorr_status_t last_launch() {
   count_launch();
   return cudaGetLastError() == cudaSuccess ? LILICORR_OK : LILICORR_ERR_CUDA;
+}
+
+// Launch with programmatic dependent launch allowed: the kernel may start while its
+// predecessor on the stream finishes. Every kernel of this library begins with
+// pdl_wait() before it reads or writes memory that an earlier launch touches, so the
+// stream order of results is unchanged; what overlaps is the launch itself and the
+// setup that needs no inputs.
+template <typename... KArgs, typename... Args>
+lilicorr_status_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                           cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+  count_launch();
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    return LILICORR_ERR_CUDA;
+  }
+  return LILICORR_OK;
+}
+
+// Wait for the preceding launch on the stream to complete and its writes to be visible
+// (a no-op when the kernel was not launched as a dependent), then let the next launch
+// on the stream start its own setup.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -115,10 +153,10 @@ struct HeadW {          // device pointers of one Transformer layer
 struct lilicorr_head {
   lilicorr_head_desc desc;
   int device;
-  // the projections that do not depend on the top-K pass run on a side stream that
-  // forks from and joins the caller's stream (a fork/join under graph capture)
-  cudaStream_t side;
-  cudaEvent_t ev_fork, ev_join;
+  // the projections that do not depend on the top-K pass run on two side streams that
+  // fork from and join the caller's stream (fork/join nodes under graph capture)
+  cudaStream_t side, side2;
+  cudaEvent_t ev_fork, ev_join, ev_join2;
   void* pool;                 // one device allocation holding everything below
   size_t pool_bytes;
   // matrices in head dtype; vectors and tables in fp32
@@ -194,7 +232,8 @@ void net_fused_maps_free(void* maps);
 lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t* ids,
                                    const float* logp, const float* hproj, const float* t,
                                    const float* cb, float* oi, uint32_t* status, cudaStream_t st);
-extern int g_fused_enabled;   // testing switch: 0 keeps every head on the unfused chain
+extern int g_fused_enabled;   // 0 never, 1 from FUSED_MIN_B sequences on (default), 2 always
+constexpr int FUSED_MIN_B = 8;
 
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,
                                      const float* gain, void* tn, lilicorr_dtype_t tn_dt,

@@ -15,14 +15,14 @@
 // its size up to 64 KB, so the tiles are as large as shared memory allows. Bias and gain
 // vectors and the confidence-network weights are staged in shared memory.
 //
-// Warp roles (320 threads):
+// Warp roles (576 threads):
 //   warp 0    one lane: TMA producer of the weight ring
 //   warp 1    tensor-memory allocation; one lane issues tcgen05.mma (M 128, N 256/192, K 16)
-//   warps 2-9 row workers. Warp w reads tensor-memory lanes 32*(w%4)..+31, so thread
-//             (set s = (w-2)/4, row r) owns row r and the column half s of a 256-wide
-//             region. They build the nodes, drain accumulators (bias, SiLU, RMSNorm),
-//             and run the attention core with warp-level mma.sync: set s takes head
-//             2g+s of head pair g, each warp 32 queries, all L*K keys in one pass.
+//   warps 2-17 row workers. Warp w reads tensor-memory lanes 32*(w%4)..+31, so thread
+//             (column group c = (w-2)/4, row r) owns row r and columns 64c..64c+63 of a
+//             256-wide region. They build the nodes, drain accumulators (bias, SiLU,
+//             RMSNorm), and run the attention core with warp-level mma.sync: groups
+//             0-1 take head 2g, groups 2-3 head 2g+1 of head pair g, 16 queries per warp.
 //
 // Products, in issue order (A operand in shared memory, accumulator in tensor memory):
 //   conf2                 x += c1 W_c2^T                      (x preloaded with the node base)
@@ -56,7 +56,9 @@ constexpr int NF_M = 128;                 // node rows per CTA
 constexpr int NF_STAGES = 2;              // weight ring depth
 constexpr int NF_MAX_LAYERS = 4;
 constexpr int NF_MAX_L = 64;
-constexpr int NF_RW = 256;                // row-worker threads
+constexpr int NF_RW = 512;                // row-worker threads (16 warps)
+constexpr int NF_CG = 4;                  // a row's 256 columns split over 4 threads
+constexpr int NF_CW = NF_D / NF_CG;       // 64 columns per thread
 constexpr int NF_THREADS = 64 + NF_RW;
 constexpr uint32_t STAGE_BYTES = 256 * 64 * 2;   // one K chunk of 256 weight rows
 constexpr uint32_t CHUNK = 128 * 128;     // 128 rows x 64 bf16, one swizzled K chunk
@@ -77,8 +79,8 @@ constexpr uint32_t OFF_VEC = OFF_HF + 4 * CHUNK;                   // staged vec
 constexpr int V_AN = 0, V_FN = 256, V_BO = 512, V_B1 = 768, V_BQKV = 1280, V_B2 = 2048,
               V_C1W = 2560, V_C1B = 3840, V_C2B = 4096, V_FIN = 4352, V_BOI = 4608, V_T = 5120,
               V_CB = 5376, V_END = 5632;
-constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [2][128] float
-constexpr uint32_t OFF_DIST = OFF_SS + 2 * NF_M * 4;               // [8][127] float
+constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [4][128] float
+constexpr uint32_t OFF_DIST = OFF_SS + NF_CG * NF_M * 4;           // [8][127] float
 constexpr uint32_t OFF_SAME = OFF_DIST + NF_NH * (2 * NF_MAX_L - 1) * 4;
 constexpr uint32_t OFF_SLOT = OFF_SAME + NF_NH * 4;                // [128] slot of each node
 constexpr uint32_t OFF_BAR = (OFF_SLOT + NF_M + 63) & ~63u;
@@ -274,8 +276,8 @@ struct Issuer {
 __device__ __forceinline__ uint32_t swz(int r, int j) {     // 16-byte piece j of row r
   return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
 }
-// q / k / v of one head: [128 rows][32] bf16, 64-byte rows, pieces XOR-swizzled by row
-// pair so that ldmatrix over 8 consecutive rows touches 8 distinct bank groups
+// q / k / v of one head: [128 rows][32] 16-bit values, 64-byte rows, pieces XOR-swizzled
+// by row pair so that ldmatrix over 8 consecutive rows touches 8 distinct bank groups
 __device__ __forceinline__ uint32_t qkv_off(int row, int piece) {
   return (uint32_t)(row * 64 + ((piece ^ ((row >> 1) & 3)) << 4));
 }
@@ -289,10 +291,19 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                : "r"(addr));
 }
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
+// warp-level products: S = Q K^T with bf16 operands, O += P V with fp16 operands
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                              uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
       "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
@@ -302,7 +313,27 @@ __device__ __forceinline__ float ex2f(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// two fp32 -> fp16x2 (round to nearest), and 2^x on both halves in one instruction
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
+  const __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t ex2_h2(uint32_t x) {
+  uint32_t y;
+  asm("ex2.approx.f16x2 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+__device__ __forceinline__ float2 h2_to_f2(uint32_t x) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&x));
+}
+// SiLU(z) = z sigmoid(z) = z (1 + tanh(z / 2)) / 2, one MUFU operation
+__device__ __forceinline__ float silu_fast(float z) {
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * z));
+  return 0.5f * z * (1.0f + t);
+}
 __device__ __forceinline__ void rw_bar() { named_bar(1, NF_RW); }
+__device__ __forceinline__ void set_bar(int set) { named_bar(2 + set, NF_RW / 2); }
 // 16-byte asynchronous global -> shared copies (L2 only), many in flight per thread
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
@@ -310,9 +341,6 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
 }
-// SiLU with the fast reciprocal: z / (1 + e^-z)
-__device__ __forceinline__ float silu_fast(float z) { return __fdividef(z, 1.0f + __expf(-z)); }
-__device__ __forceinline__ void set_bar(int set) { named_bar(2 + set, NF_RW / 2); }
 
 // One warp's arrival on a row-worker -> MMA event, after its shared-memory writes
 // (generic proxy, read by the tensor cores through the async proxy) and tensor-memory
@@ -324,13 +352,21 @@ __device__ __forceinline__ void rw_signal(uint64_t* bar, int lane) {
   if (lane == 0) mbar_arrive(bar);
 }
 
-// 8 bf16 of v[p*8 .. p*8+7] as one 16-byte piece
+// 8 bf16 / fp16 of v[0..7] as one 16-byte piece
 __device__ __forceinline__ uint4 pack8(const float* v) {
   uint4 w;
   w.x = pack_bf16x2(v[0], v[1]);
   w.y = pack_bf16x2(v[2], v[3]);
   w.z = pack_bf16x2(v[4], v[5]);
   w.w = pack_bf16x2(v[6], v[7]);
+  return w;
+}
+__device__ __forceinline__ uint4 pack8h(const float* v) {
+  uint4 w;
+  w.x = pack_h2(v[0], v[1]);
+  w.y = pack_h2(v[2], v[3]);
+  w.z = pack_h2(v[4], v[5]);
+  w.w = pack_h2(v[6], v[7]);
   return w;
 }
 
@@ -356,15 +392,15 @@ __device__ __forceinline__ void st32f(uint32_t taddr, const float (&v)[32]) {
   tmem_st32(taddr, u);
 }
 
-// RMSNorm statistics of row r over the 256 columns of x (each thread its half): adds
-// `bias` (shared memory) into x first (and writes x back to tensor memory when write_back). Returns
-// 1 / rms.
-__device__ float row_rstd(uint32_t tx, const float* bias, bool write_back, int set, int r,
+// RMSNorm statistics of row r over the 256 columns of x (4 threads, 64 columns each):
+// adds `bias` (shared memory) into x first, and writes x back to tensor memory when
+// write_back. Returns 1 / rms.
+__device__ float row_rstd(uint32_t tx, const float* bias, bool write_back, int cg, int r,
                           float* s_ss) {
   float ss = 0.f;
 #pragma unroll 1
-  for (int j = 0; j < 4; ++j) {
-    const int c0 = 128 * set + 32 * j;
+  for (int j = 0; j < 2; ++j) {
+    const int c0 = NF_CW * cg + 32 * j;
     float v[32];
     ld32f(tx + c0, v);
     if (bias) {
@@ -376,19 +412,19 @@ __device__ float row_rstd(uint32_t tx, const float* bias, bool write_back, int s
     for (int e = 0; e < 32; ++e) ss = fmaf(v[e], v[e], ss);
   }
   if (bias && write_back) tmem_wait_st();
-  s_ss[set * NF_M + r] = ss;
+  s_ss[cg * NF_M + r] = ss;
   rw_bar();
-  const float tot = s_ss[r] + s_ss[NF_M + r];
+  const float tot = (s_ss[r] + s_ss[NF_M + r]) + (s_ss[2 * NF_M + r] + s_ss[3 * NF_M + r]);
   rw_bar();                                  // s_ss free for the next statistics
   return rsqrtf(tot / (float)NF_D + NF_RMS_EPS);
 }
 
-// xn = x * rstd * gain (+ bias already in x) -> bf16 into ACT; with t, also xn * t -> HF
+// xn = (x + bias) * rstd * gain -> bf16 into ACT; with t, also xn * t -> HF
 __device__ void row_normed(uint8_t* sm, uint32_t tx, const float* bias, float rstd,
-                           const float* gain, const float* t, int set, int r) {
+                           const float* gain, const float* t, int cg, int r) {
 #pragma unroll 1
-  for (int j = 0; j < 4; ++j) {
-    const int c0 = 128 * set + 32 * j;
+  for (int j = 0; j < 2; ++j) {
+    const int c0 = NF_CW * cg + 32 * j;
     float v[32];
     ld32f(tx + c0, v);
 #pragma unroll
@@ -405,20 +441,15 @@ __device__ void row_normed(uint8_t* sm, uint32_t tx, const float* bias, float rs
   }
 }
 
-// Drain 256 scratch columns: v + bias (+ per-sequence row bias), SiLU -> bf16 into buf.
-__device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, const float* bias2,
-                           int set, int r) {
+// Drain this thread's 64 of 256 scratch columns: v + bias, SiLU -> bf16 into buf.
+__device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, int cg, int r) {
 #pragma unroll 1
-  for (int j = 0; j < 4; ++j) {
-    const int c0 = 128 * set + 32 * j;
+  for (int j = 0; j < 2; ++j) {
+    const int c0 = NF_CW * cg + 32 * j;
     float v[32];
     ld32f(tscr + c0, v);
 #pragma unroll
-    for (int e = 0; e < 32; ++e) {
-      float z = v[e] + bias[c0 + e];
-      if (bias2) z += bias2[c0 + e];
-      v[e] = silu_fast(z);
-    }
+    for (int e = 0; e < 32; ++e) v[e] = silu_fast(v[e] + bias[c0 + e]);
     put32(buf, r, c0, v);
   }
 }
@@ -462,6 +493,10 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_base;
+  if (warp == 0 && lane == 0)      // the weight stream needs nothing from earlier launches
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  else
+    pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -479,10 +514,12 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ row workers
-    const int set = (warp - 2) >> 2;                 // column half / head of the pair
-    const int wi = (warp - 2) & 3;                   // warp inside the set
+    const int cg = (warp - 2) >> 2;                  // column group: columns 64cg .. 64cg+63
+    const int set = cg >> 1;                         // head of the pair in the attention core
+    const int wi = (warp - 2) & 7;                   // warp inside the set: queries 16wi..+15
     const int q = warp & 3;                          // tensor-memory lane quarter
     const int r = q * 32 + lane;                     // node row
+    const int wr = warp - 2;                         // row-worker warp index 0..15
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const uint32_t tx = tmem + lane_off + X_COL, tscr = tmem + lane_off + SCR_COL;
     const int L = a.L, K = a.K, LK = a.LK, nl = a.n_layers;
@@ -523,10 +560,9 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         // node base rows. cp.async brings, all at once, the drafter-state rows W_h h_s + b_h,
         // the slot and rank tables (into ACT, which c1 fills afterwards) and the folded
         // embedding rows of 64 nodes at a time (into HF, 16-byte pieces XOR-swizzled by row);
-        // the thread owning a row then sums its half from shared memory into tensor memory.
+        // the threads owning a row then sum it from shared memory into tensor memory.
         float* tab = reinterpret_cast<float*>(sm + OFF_ACT);     // rows: hproj+slot+b_c2 [L], rank [K]
         uint8_t* stg = sm + OFF_HF;
-        const int wr = warp - 2;
         for (int i = tid; i < (2 * L + K) * (NF_D / 4); i += NF_RW) {
           const int row = i / (NF_D / 4), c = (i % (NF_D / 4)) * 4;
           const float* src = row < L ? a.hproj + ((size_t)b * L + row) * NF_D + c
@@ -565,13 +601,12 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         for (int p = 0; p < 2; ++p) {
           if ((q >> 1) == p) {                      // rows 64p .. 64p+63 belong to quarters 2p, 2p+1
             const int nr = r - 64 * p;
-            const bool okr = r < LK;
             const uint8_t* row = stg + nr * 1024;
-            const float* S = tab + (size_t)(okr ? r / K : 0) * NF_D;
-            const float* R = tab + (size_t)(2 * L + (okr ? r % K : 0)) * NF_D;
+            const float* S = tab + (size_t)(ok ? r / K : 0) * NF_D;
+            const float* R = tab + (size_t)(2 * L + (ok ? r % K : 0)) * NF_D;
 #pragma unroll 1
-            for (int j = 0; j < 4; ++j) {
-              const int c0 = 128 * set + 32 * j;
+            for (int j = 0; j < 2; ++j) {
+              const int c0 = NF_CW * cg + 32 * j;
               float v[32];
 #pragma unroll
               for (int u = 0; u < 8; ++u) {
@@ -579,10 +614,10 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
                     *reinterpret_cast<const float4*>(row + ((((c0 >> 2) + u) ^ (nr & 7)) << 4));
                 const float4 y = *reinterpret_cast<const float4*>(S + c0 + 4 * u);
                 const float4 z = *reinterpret_cast<const float4*>(R + c0 + 4 * u);
-                v[4 * u] = okr ? x.x + y.x + z.x : 0.f;
-                v[4 * u + 1] = okr ? x.y + y.y + z.y : 0.f;
-                v[4 * u + 2] = okr ? x.z + y.z + z.z : 0.f;
-                v[4 * u + 3] = okr ? x.w + y.w + z.w : 0.f;
+                v[4 * u] = ok ? x.x + y.x + z.x : 0.f;
+                v[4 * u + 1] = ok ? x.y + y.y + z.y : 0.f;
+                v[4 * u + 2] = ok ? x.z + y.z + z.z : 0.f;
+                v[4 * u + 3] = ok ? x.w + y.w + z.w : 0.f;
               }
               st32f(tx + c0, v);
             }
@@ -594,10 +629,10 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
             rw_bar();
           }
         }
-        // c1 of this thread's row and column half, 4 columns per step (ACT is free again)
+        // c1 of this thread's row and 64 columns, 4 columns per step (ACT is free again)
 #pragma unroll 1
-        for (int j = 0; j < 4; ++j) {
-          const int c0 = 128 * set + 32 * j;
+        for (int j = 0; j < 2; ++j) {
+          const int c0 = NF_CW * cg + 32 * j;
           float c1[32];
 #pragma unroll
           for (int e = 0; e < 32; e += 4) {
@@ -618,7 +653,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
           put32(sm + OFF_ACT, r, c0, c1);
         }
         tmem_wait_st();
-        if (set == 0) s_slot[r] = (uint8_t)min(r / K, L - 1);   // read after the next rw_bar
+        if (cg == 0) s_slot[r] = (uint8_t)min(r / K, L - 1);   // read after the next rw_bar
         rw_signal(&sh.ready[0], lane);
       }
       // ---- Transformer layers
@@ -639,142 +674,157 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         if (tid < NF_NH) s_same[tid] = a.same[l][tid] * LOG2E;
         // x += b_2 of the previous layer (staged then), RMSNorm statistics
         const float* b2p = l == 0 ? nullptr : vec + V_B2 + ((l - 1) & 1) * NF_D;
-        float rstd = row_rstd(tx, b2p, true, set, r, s_ss);
-        row_normed(sm, tx, nullptr, rstd, vec + V_AN, nullptr, set, r);
+        float rstd = row_rstd(tx, b2p, true, cg, r, s_ss);
+        row_normed(sm, tx, nullptr, rstd, vec + V_AN, nullptr, cg, r);
         rw_signal(&sh.ready[R_XN(l)], lane);
 
         for (int g = 0; g < 4; ++g) {
-          // q | k | v of head 2g+set -> shared memory (bias added, bf16)
+          // q | k (bf16) and v (fp16) of head 2g+set -> shared memory, biases added
           ev_wait(&sh.done[D_QKV(l, g)], par, sh.abort);
           tc_fence_after();
           set_bar(set);                              // the set's previous head is done
           uint8_t* qs = sm + OFF_HF + set * QKV_SET;
           const int hh = 2 * g + set;
 #pragma unroll 1
-          for (int part = 0; part < 3; ++part) {
+          for (int part = (cg & 1) ? 2 : 0; part < ((cg & 1) ? 3 : 2); ++part) {
             float v[32];
             ld32f(tscr + 64 * part + 32 * set, v);
             const float* bq = vec + V_BQKV + part * NF_D + hh * NF_HD;
-            const bool zero = part > 0 && r >= LK;   // padded keys and values
+            const bool zero = part == 2 && r >= LK;  // padded values (their keys are masked)
 #pragma unroll
             for (int e = 0; e < 32; ++e) v[e] = zero ? 0.f : v[e] + bq[e];
             uint8_t* dst = qs + part * 8192;
 #pragma unroll
             for (int p = 0; p < 4; ++p)
-              *reinterpret_cast<uint4*>(dst + qkv_off(r, p)) = pack8(v + 8 * p);
+              *reinterpret_cast<uint4*>(dst + qkv_off(r, p)) =
+                  part == 2 ? pack8h(v + 8 * p) : pack8(v + 8 * p);
           }
           if (g < 3) rw_signal(&sh.ready[R_QKV_DRAINED(l, g)], lane);
           set_bar(set);
-          // attention core of head hh: warp wi takes queries 32wi .. 32wi+31
+          // attention core of head hh, queries 16wi .. 16wi+15: blocks of 32 keys with an
+          // online softmax in log2 units; P = 2^(S - max) in fp16 pairs (one MUFU op per pair)
           const uint32_t qb = smem_u32(qs), kb = qb + 8192, vb = qb + 16384;
           const int g8 = lane >> 2, t4 = lane & 3;
           const float qscale = rsqrtf((float)NF_HD) * LOG2E;
           const float same_l2 = s_same[hh];
           const float* sd = s_dist + hh * nd + (L - 1);
-          uint8_t* att = sm + OFF_ATT;
+          const int q0 = 16 * wi;
+          uint32_t qa[2][4];
+#pragma unroll
+          for (int ks = 0; ks < 2; ++ks)
+            ldsm_x4(qb + qkv_off(q0 + (lane & 15), ks * 2 + (lane >> 4)), qa[ks]);
+          const int i0 = q0 + g8, i1 = i0 + 8;
+          const int si0 = s_slot[i0], si1 = s_slot[i1];
+          float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+          float o[4][4];
+#pragma unroll
+          for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
 #pragma unroll 1
-          for (int mt = 0; mt < 2; ++mt) {
-            const int q0 = 32 * wi + 16 * mt;
-            uint32_t qa[2][4];
+          for (int kb0 = 0; kb0 < LK; kb0 += 32) {
+            float s4[4][4];
 #pragma unroll
-            for (int ks = 0; ks < 2; ++ks)
-              ldsm_x4(qb + qkv_off(q0 + (lane & 15), ks * 2 + (lane >> 4)), qa[ks]);
-            float s[16][4];
-#pragma unroll
-            for (int nb = 0; nb < 16; ++nb) s[nb][0] = s[nb][1] = s[nb][2] = s[nb][3] = 0.f;
+            for (int nb = 0; nb < 4; ++nb) s4[nb][0] = s4[nb][1] = s4[nb][2] = s4[nb][3] = 0.f;
 #pragma unroll
             for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
-              for (int nb = 0; nb < 16; nb += 2) {
+              for (int nb = 0; nb < 4; nb += 2) {
                 uint32_t bf[4];
-                const int key = nb * 8 + (lane & 7) + ((lane >> 4) << 3);
+                const int key = kb0 + nb * 8 + (lane & 7) + ((lane >> 4) << 3);
                 ldsm_x4(kb + qkv_off(key, ks * 2 + ((lane >> 3) & 1)), bf);
-                mma16816(s[nb], qa[ks], bf[0], bf[1]);
-                mma16816(s[nb + 1], qa[ks], bf[2], bf[3]);
+                mma_bf16_16816(s4[nb], qa[ks], bf[0], bf[1]);
+                mma_bf16_16816(s4[nb + 1], qa[ks], bf[2], bf[3]);
               }
-            const int i0 = q0 + g8, i1 = i0 + 8;
-            const int si0 = s_slot[i0], si1 = s_slot[i1];
-            float m0 = -INFINITY, m1 = -INFINITY;
+            float bm0 = -INFINITY, bm1 = -INFINITY;
 #pragma unroll
-            for (int nb = 0; nb < 16; ++nb) {
-              const int j0 = nb * 8 + 2 * t4;
+            for (int nb = 0; nb < 4; ++nb) {
+              const int j0 = kb0 + nb * 8 + 2 * t4;
               const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                const int j = j0 + (e & 1);
+                const int jj = j0 + (e & 1);
                 const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
                 const int si = e < 2 ? si0 : si1;
-                const float v = j < LK ? s[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
-                                       : -INFINITY;
-                s[nb][e] = v;
-                if (e < 2) m0 = fmaxf(m0, v); else m1 = fmaxf(m1, v);
+                const float v = jj < LK
+                                    ? s4[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
+                                    : -INFINITY;
+                s4[nb][e] = v;
+                if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
               }
             }
-            m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 1));
-            m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 2));
-            m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 1));
-            m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 2));
-            float l0 = 0.f, l1 = 0.f;
-            uint32_t pa[8][4];
+            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
+            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
+            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
+            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
+            const float mn0 = fmaxf(m0, bm0), mn1 = fmaxf(m1, bm1);
+            const float c0 = ex2f(m0 - mn0), c1 = ex2f(m1 - mn1);   // 0 on the first block
+            m0 = mn0;
+            m1 = mn1;
+            l0 *= c0;
+            l1 *= c1;
 #pragma unroll
-            for (int nb = 0; nb < 16; ++nb) {
-              const float p0 = ex2f(s[nb][0] - m0), p1 = ex2f(s[nb][1] - m0);
-              const float p2 = ex2f(s[nb][2] - m1), p3 = ex2f(s[nb][3] - m1);
-              l0 += p0 + p1;
-              l1 += p2 + p3;
+            for (int nb = 0; nb < 4; ++nb) {
+              o[nb][0] *= c0; o[nb][1] *= c0;
+              o[nb][2] *= c1; o[nb][3] *= c1;
+            }
+            uint32_t pa[2][4];
+#pragma unroll
+            for (int nb = 0; nb < 4; ++nb) {
+              const uint32_t h01 = ex2_h2(pack_h2(s4[nb][0] - mn0, s4[nb][1] - mn0));
+              const uint32_t h23 = ex2_h2(pack_h2(s4[nb][2] - mn1, s4[nb][3] - mn1));
+              const float2 f01 = h2_to_f2(h01), f23 = h2_to_f2(h23);
+              l0 += f01.x + f01.y;
+              l1 += f23.x + f23.y;
               const int kk = nb >> 1;
               if ((nb & 1) == 0) {
-                pa[kk][0] = pack_bf16x2(p0, p1);
-                pa[kk][1] = pack_bf16x2(p2, p3);
+                pa[kk][0] = h01;
+                pa[kk][1] = h23;
               } else {
-                pa[kk][2] = pack_bf16x2(p0, p1);
-                pa[kk][3] = pack_bf16x2(p2, p3);
+                pa[kk][2] = h01;
+                pa[kk][3] = h23;
               }
             }
-            float o[4][4];
 #pragma unroll
-            for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
+            for (int kk = 0; kk < 2; ++kk)
 #pragma unroll
               for (int nb = 0; nb < 4; nb += 2) {
                 uint32_t vf[4];
-                const int key = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+                const int key = kb0 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
                 ldsm_x4_t(vb + qkv_off(key, nb + (lane >> 4)), vf);
-                mma16816(o[nb], pa[kk], vf[0], vf[1]);
-                mma16816(o[nb + 1], pa[kk], vf[2], vf[3]);
+                mma_f16_16816(o[nb], pa[kk], vf[0], vf[1]);
+                mma_f16_16816(o[nb + 1], pa[kk], vf[2], vf[3]);
               }
-            l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-            l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-            l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-            l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-            const float inv0 = 1.0f / l0, inv1 = 1.0f / l1;
-            // the attention-output buffer is free once the previous pair's W_o product ran
-            if (mt == 0 && g > 0) ev_wait(&sh.done[D_WO(l, g - 1)], par, sh.abort);
+          }
+          l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+          l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+          l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+          l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+          const float inv0 = 1.0f / l0, inv1 = 1.0f / l1;
+          // the attention-output buffer is free once the previous pair's W_o product ran
+          if (g > 0) ev_wait(&sh.done[D_WO(l, g - 1)], par, sh.abort);
+          uint8_t* att = sm + OFF_ATT;
 #pragma unroll
-            for (int nb = 0; nb < 4; ++nb) {
-              const int piece = 4 * set + nb;
-              *reinterpret_cast<uint32_t*>(att + swz(i0, piece) + 4 * t4) =
-                  pack_bf16x2(o[nb][0] * inv0, o[nb][1] * inv0);
-              *reinterpret_cast<uint32_t*>(att + swz(i1, piece) + 4 * t4) =
-                  pack_bf16x2(o[nb][2] * inv1, o[nb][3] * inv1);
-            }
+          for (int nb = 0; nb < 4; ++nb) {
+            const int piece = 4 * set + nb;
+            *reinterpret_cast<uint32_t*>(att + swz(i0, piece) + 4 * t4) =
+                pack_bf16x2(o[nb][0] * inv0, o[nb][1] * inv0);
+            *reinterpret_cast<uint32_t*>(att + swz(i1, piece) + 4 * t4) =
+                pack_bf16x2(o[nb][2] * inv1, o[nb][3] * inv1);
           }
           rw_signal(&sh.ready[R_ATT(l, g)], lane);
         }
         // ---- FFN: x += b_o, xn2 = RMSNorm(x)
         ev_wait(&sh.done[D_WO(l, 3)], par, sh.abort);
         tc_fence_after();
-        rstd = row_rstd(tx, vec + V_BO, true, set, r, s_ss);
-        row_normed(sm, tx, nullptr, rstd, vec + V_FN, nullptr, set, r);
+        rstd = row_rstd(tx, vec + V_BO, true, cg, r, s_ss);
+        row_normed(sm, tx, nullptr, rstd, vec + V_FN, nullptr, cg, r);
         rw_signal(&sh.ready[R_XN2(l)], lane);
         ev_wait(&sh.done[D_FFN(l, 0)], par, sh.abort);
         tc_fence_after();
-        drain_silu(sm + OFF_HF, tscr, vec + V_B1, nullptr, set, r);
+        drain_silu(sm + OFF_HF, tscr, vec + V_B1, cg, r);
         rw_signal(&sh.ready[R_HFA(l)], lane);
         ev_wait(&sh.done[D_FFN(l, 1)], par, sh.abort);
         tc_fence_after();
-        drain_silu(sm + OFF_ACT, tscr, vec + V_B1 + 256, nullptr, set, r);
+        drain_silu(sm + OFF_ACT, tscr, vec + V_B1 + 256, cg, r);
         rw_signal(&sh.ready[R_HFB(l)], lane);
       }
       // ---- fusion: xf = RMSNorm(x + b_2) -> ACT, xf * t -> HF; u = SiLU(. + cb) -> ACT
@@ -782,33 +832,33 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
       tc_fence_after();
       {
         const float* b2l = vec + V_B2 + ((nl - 1) & 1) * NF_D;
-        const float rstd = row_rstd(tx, b2l, false, set, r, s_ss);
-        row_normed(sm, tx, b2l, rstd, vec + V_FIN, vec + V_T, set, r);
+        const float rstd = row_rstd(tx, b2l, false, cg, r, s_ss);
+        row_normed(sm, tx, b2l, rstd, vec + V_FIN, vec + V_T, cg, r);
       }
       rw_signal(&sh.ready[lb(nl)], lane);
       ev_wait(&sh.done[lb(nl)], par, sh.abort);
       tc_fence_after();
-      drain_silu(sm + OFF_ACT, tscr, vec + V_CB, nullptr, set, r);
+      drain_silu(sm + OFF_ACT, tscr, vec + V_CB, cg, r);
       rw_signal(&sh.ready[lb(nl) + 1], lane);
       // ---- out / in heads: 256 columns of [o | i] at a time -> oi (fp32, not yet unit).
-      // Each column half goes through a staging buffer (128 rows x 128 floats, pieces
+      // Each 128-column half goes through a staging buffer (128 rows x 128 floats, pieces
       // swizzled by row) so that the global stores are row-contiguous.
       for (int h = 0; h * 256 < a.d2; ++h) {
         ev_wait(&sh.done[lb(nl) + 1 + h], par, sh.abort);
         tc_fence_after();
         uint8_t* stg = sm + OFF_HF;
-        const int wr = warp - 2;
 #pragma unroll 1
         for (int hs = 0; hs < 2; ++hs) {
-          if (set == hs) {
+          if ((cg >> 1) == hs) {
 #pragma unroll 1
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < 2; ++j) {
+              const int cl = 64 * (cg & 1) + 32 * j;          // column inside the 128 staged
               float v[32];
-              ld32f(tscr + 128 * hs + 32 * j, v);
-              const float* bo = vec + V_BOI + 256 * h + 128 * hs + 32 * j;
+              ld32f(tscr + 128 * hs + cl, v);
+              const float* bo = vec + V_BOI + 256 * h + 128 * hs + cl;
 #pragma unroll
               for (int u = 0; u < 8; ++u)
-                *reinterpret_cast<float4*>(stg + r * 512 + (((8 * j + u) ^ (r & 7)) << 4)) =
+                *reinterpret_cast<float4*>(stg + r * 512 + ((((cl >> 2) + u) ^ (r & 7)) << 4)) =
                     make_float4(v[4 * u] + bo[4 * u], v[4 * u + 1] + bo[4 * u + 1],
                                 v[4 * u + 2] + bo[4 * u + 2], v[4 * u + 3] + bo[4 * u + 3]);
             }
@@ -823,7 +873,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         if ((h + 1) * 256 < a.d2) rw_signal(&sh.ready[lb(nl) + 2 + h], lane);
       }
       tc_fence_before();
-      rw_bar();                                      // s_dist / s_ss reuse by the next sequence
+      rw_bar();                                      // s_dist / s_ss / vectors reuse by the next sequence
     }
   }
 
@@ -936,8 +986,8 @@ lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t*
   static bool configured[64] = {false};
   LL_TRY(allow_max_dynamic_smem(net_fused_kernel, configured));
   const int grid = B < num_sms() ? B : num_sms();
-  net_fused_kernel<<<grid, NF_THREADS, NF_SMEM, st>>>(nm->m, a);
-  return last_launch();
+  LL_TRY(launch_k(net_fused_kernel, grid, NF_THREADS, NF_SMEM, st, nm->m, a));
+  return LILICORR_OK;
 }
 
 }  // namespace lilicorr

@@ -62,6 +62,7 @@ __device__ void walk_sequence(const float* A, const float* P, int b, int L, int 
 }
 
 __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
+  pdl_wait();
   extern __shared__ float sm[];
   __shared__ int s_last;
   const int b = blockIdx.x, j = blockIdx.y;          // j = 0: anchor row; j >= 1: pair (j-1, j)
@@ -129,6 +130,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
 }
 
 __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
+  pdl_wait();
   extern __shared__ float sm[];
   const int b = blockIdx.x, L = a.L, K = a.K;
   const int n_scores = K + (L - 1) * K * K;
@@ -164,12 +166,12 @@ lilicorr_status_t launch_pair_walk(const PairWalkArgs& in, cudaStream_t st) {
     if (a.do_walk && a.scores_in_smem && score_bytes > smem) smem = score_bytes;
     LL_TRY(allow_max_dynamic_smem(pair_rows_kernel, cfg_pair));
     dim3 grid(a.B, a.L);
-    pair_rows_kernel<<<grid, PW_THREADS, smem, st>>>(a);
-    return last_launch();
+    LL_TRY(launch_k(pair_rows_kernel, grid, PW_THREADS, smem, st, a));
+    return LILICORR_OK;
   }
   LL_TRY(allow_max_dynamic_smem(walk_kernel, cfg_walk));
-  walk_kernel<<<a.B, PW_THREADS, a.scores_in_smem ? score_bytes : 0, st>>>(a);
-  return last_launch();
+  LL_TRY(launch_k(walk_kernel, a.B, PW_THREADS, a.scores_in_smem ? score_bytes : 0, st, a));
+  return LILICORR_OK;
 }
 
 }  // namespace lilicorr

@@ -306,6 +306,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
                 size_t rec_bytes, int32_t* __restrict__ ids, float* __restrict__ logp,
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
                 unsigned char* partials) {
+  pdl_wait();
   constexpr int VEC = Vec<T>::N;
   __shared__ uint64_t s_buf[TK_WARPS][TK_CAP];   // the warps' candidates
   __shared__ uint64_t s_tmp[TK_WARPS][LILICORR_MAX_K];
@@ -502,14 +503,14 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
   const TopkPlan p = topk_plan(rows, V, K, dt);
   dim3 grid(p.splits, rows);
   if (dt == LILICORR_BF16)
-    topk_lse_kernel<uint16_t><<<grid, TK_THREADS, 0, st>>>(
+    LL_TRY(launch_k(topk_lse_kernel<uint16_t>, grid, TK_THREADS, 0, st, 
         static_cast<const uint16_t*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials));
+        lse, status, counters, static_cast<unsigned char*>(partials)));
   else
-    topk_lse_kernel<float><<<grid, TK_THREADS, 0, st>>>(
+    LL_TRY(launch_k(topk_lse_kernel<float>, grid, TK_THREADS, 0, st, 
         static_cast<const float*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials));
-  return last_launch();
+        lse, status, counters, static_cast<unsigned char*>(partials)));
+  return LILICORR_OK;
 }
 
 }  // namespace lilicorr

@@ -38,14 +38,14 @@ def _topk(wl, logits):
 
 
 def _run(ll, head, wl, ids, logp, inp, fused):
-    ll.test_fused_path(head, fused)
+    ll.test_fused_path(head, 2 if fused else 0)
     try:
         res = ll.embed_in_out(head, to_dev(ids.astype(np.int32), "f32"),
                               to_dev(logp.astype(np.float32), "f32"),
                               to_dev(inp["hidden"], wl.dtype), to_dev(inp["target"], wl.dtype))
         torch.cuda.synchronize()
     finally:
-        ll.test_fused_path(None, True)
+        ll.test_fused_path(None, 1)
     return [t.cpu().numpy() for t in res]
 
 
@@ -68,7 +68,7 @@ def test_fused_matches_oracle_and_unfused(B, L, K):
     ids, logp = _topk(wl, inp["logits"])
     head = ll.Head.from_workload(wl, W, workloads.embed_table(wl.V, wl.H, wl.dtype))
     try:
-        assert ll.test_fused_path(head, True), "this head shape should take the fused kernel"
+        assert ll.test_fused_path(head, 1), "this head shape should take the fused kernel"
         out, inn, anc = _run(ll, head, wl, ids, logp, inp, True)
         assert np.isfinite(out).all() and np.isfinite(inn).all()
         assert np.allclose(np.linalg.norm(out, axis=-1), 1, atol=1e-5)
@@ -93,7 +93,7 @@ def test_fused_more_sequences_than_sms():
     logp = np.take_along_axis(x.astype(np.float64), ids, -1) - 10.0
     head = ll.Head.from_workload(wl, W, workloads.embed_table(wl.V, wl.H, wl.dtype))
     try:
-        assert ll.test_fused_path(head, True)
+        assert ll.test_fused_path(head, 1)
         out, inn, anc = _run(ll, head, wl, ids, logp, inp, True)
         again = _run(ll, head, wl, ids, logp, inp, True)       # a second call, same head
         assert np.array_equal(out, again[0]) and np.array_equal(inn, again[1])
