@@ -369,6 +369,37 @@ def run_ours(args, world, rank, local):
            + d_target.numel() * d_target.element_size()) * e2e_calls
     d2h = d_tokens.numel() * 4 * e2e_calls
 
+    # ---- the exact best path (App. E) in place of the greedy walk: the same calls on a
+    # sample of the blocks, both walks captured alike and timed back to back
+    nv = min(nblk, 100)
+    walk_ms = {}
+    for walk in ("greedy", "viterbi"):
+        gl = []
+        for i0 in range(0, nv, G):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                for i in range(i0, min(i0 + G, nv)):
+                    ll.select_block(head, logits[i], hidden[i], target[i], ws=ws, tokens=tokens[i],
+                                    walk=walk)
+            gl.append(g)
+        for g in gl:
+            g.replay()
+        torch.cuda.synchronize()
+        best = None
+        for _ in range(3):
+            w0 = torch.cuda.Event(enable_timing=True)
+            w1 = torch.cuda.Event(enable_timing=True)
+            w0.record(stream)
+            for g in gl:
+                g.replay()
+            w1.record(stream)
+            torch.cuda.synchronize()
+            t = w0.elapsed_time(w1)
+            best = t if best is None else min(best, t)
+        walk_ms[walk] = best / nv
+    if ws.status() != 0:
+        raise RuntimeError("device status set by the walk comparison")
+
     # ---- roofline of the top-K pass: its launches back to back in one captured graph,
     # CUDA events on the launching stream around the replay
     rows = B * wl.L
@@ -425,6 +456,10 @@ def run_ours(args, world, rank, local):
                 "d2h_bytes_per_step": d2h,
                 "note": f"pinned host blocks cycled ({nh} distinct), copies captured with each call"},
         "gpu_launches": launches_per_call * (nblk if batch1 else 1) * args.steps,
+        "walk_viterbi": {"us_per_call": round(walk_ms["viterbi"] * 1e3, 2),
+                         "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
+                         "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
+                         "sample": f"{nv} calls of this workload, best of 3"},
         "roofline": roofline,
     }
     if rank == 0 and not args.no_cpu_baseline:

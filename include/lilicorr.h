@@ -64,6 +64,13 @@ typedef enum {
 
 typedef enum { LILICORR_F32 = 0, LILICORR_BF16 = 1 } lilicorr_dtype_t;
 
+/* How the last step picks one candidate per slot: the greedy left-to-right walk of
+ * Sec. 3.5, or the exact maximiser of the path score (App. E, Viterbi). */
+typedef enum { LILICORR_WALK_GREEDY = 0, LILICORR_WALK_VITERBI = 1 } lilicorr_walk_t;
+
+/* The paper's score scale sigma of the pair cosines (App. A "Architecture"). */
+#define LILICORR_SIGMA 8.0f
+
 /* Shapes of a scoring head (App. A; Table "hparams": D = 1024, d = 1024, 8 heads,
  * F = 2048, 2 layers, 5 captured target layers, K = 8, L = 15).
  *   H         drafter/target hidden width (input width of the two projections)
@@ -199,6 +206,18 @@ lilicorr_status_t lilicorr_greedy_walk(int B, int L, int K, const float* anchor_
                                        int32_t* choice, int32_t* tokens, float* margin,
                                        cudaStream_t stream);
 
+/* Exact best path (App. E): the candidates c maximising
+ *   g(c) = sigma * (A[c_0] + sum_{s>=1} P[s-1, c_{s-1}, c_s])
+ * over all K^L paths, by one left-to-right sweep that keeps, per candidate, the best
+ * path ending there and its predecessor (ties to the lower index), then a traceback
+ * from the best final candidate (ties to the lower index). Same layouts as
+ * lilicorr_greedy_walk; path_score [B] receives g of the chosen path (may be NULL).
+ * sigma > 0 does not change the path; it scales path_score. */
+lilicorr_status_t lilicorr_best_path(int B, int L, int K, const float* anchor_scores,
+                                     const float* pair_scores, const int32_t* ids, float sigma,
+                                     int32_t* choice, int32_t* tokens, float* path_score,
+                                     cudaStream_t stream);
+
 /* Steps (1)-(4) fused: raw inputs to the chosen tokens.
  *   logits [B, L, V], drafter_hidden [B, L, H], target_hidden [B, n_tgt, H], all of
  *   head dtype; tokens [B, L] int32. ws: lilicorr_workspace_bytes(head, B). */
@@ -206,6 +225,15 @@ lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const 
                                         const void* drafter_hidden, const void* target_hidden,
                                         int32_t* tokens, void* ws, size_t ws_bytes,
                                         cudaStream_t stream);
+
+/* lilicorr_select_block with the last step chosen by `walk`: LILICORR_WALK_GREEDY (the
+ * same as lilicorr_select_block) or LILICORR_WALK_VITERBI (the exact best path, App. E,
+ * fused into the pair-score kernel like the walk). */
+lilicorr_status_t lilicorr_select_block_walk(const lilicorr_head* head, int B, const void* logits,
+                                             const void* drafter_hidden,
+                                             const void* target_hidden, lilicorr_walk_t walk,
+                                             int32_t* tokens, void* ws, size_t ws_bytes,
+                                             cudaStream_t stream);
 
 /* Device view of a select_block workspace after the call, for inspection:
  * pointers into ws of the intermediates of the last call (ids [B,L,K] int32,

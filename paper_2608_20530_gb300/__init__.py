@@ -25,7 +25,7 @@ F32, BF16 = 0, 1
 STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported or inconsistent shape",
           3: "unsupported dtype", 4: "CUDA error", 5: "non-finite logit row",
           6: "device wait timed out", 7: "workspace too small"}
-ERR_NONFINITE = 5
+ERR_ARG, ERR_SHAPE, ERR_NONFINITE = 1, 2, 5
 MAX_K = 32
 
 
@@ -60,6 +60,8 @@ _SIGS = {
     "lilicorr_pair_scores": (_I, [_I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
     "lilicorr_greedy_walk": (_I, [_I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "lilicorr_select_block": (_I, [_P, _I, _P, _P, _P, _P, _P, _S, _P]),
+    "lilicorr_best_path": (_I, [_I, _I, _I, _P, _P, _P, ctypes.c_float, _P, _P, _P, _P]),
+    "lilicorr_select_block_walk": (_I, [_P, _I, _P, _P, _P, _I, _P, _P, _S, _P]),
     "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
@@ -311,10 +313,32 @@ def greedy_walk(A: torch.Tensor, P: torch.Tensor, ids: torch.Tensor):
     return choice, tokens, margin
 
 
+SIGMA = 8.0
+WALKS = {"greedy": 0, "viterbi": 1}
+
+
+def best_path(A: torch.Tensor, P: torch.Tensor, ids: torch.Tensor, sigma: float = SIGMA):
+    """Exact best path (App. E): choice [B, L], tokens [B, L] (int32) and path score
+    g [B] (fp32, scaled by sigma)."""
+    B, K = A.shape
+    L = P.shape[1] + 1
+    for t, n in ((A, "anchor_scores"), (P, "pair_scores"), (ids, "ids")):
+        _dev(t, n)
+    choice = torch.empty((B, L), dtype=torch.int32, device=A.device)
+    tokens = torch.empty_like(choice)
+    score = torch.empty((B,), dtype=torch.float32, device=A.device)
+    _check(lib().lilicorr_best_path(B, L, K, A.data_ptr(), P.data_ptr() if P.numel() else None,
+                                    ids.data_ptr(), float(sigma), choice.data_ptr(),
+                                    tokens.data_ptr(), score.data_ptr(), _stream()), "best_path")
+    return choice, tokens, score
+
+
 def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target: torch.Tensor,
-                 ws: Optional[Workspace] = None, tokens: Optional[torch.Tensor] = None):
+                 ws: Optional[Workspace] = None, tokens: Optional[torch.Tensor] = None,
+                 walk: str = "greedy"):
     """The fused path: logits [B, L, V], hidden [B, L, H], target [B, n_tgt, H] (head dtype,
-    on the device) -> chosen token ids [B, L] int32."""
+    on the device) -> chosen token ids [B, L] int32. walk: "greedy" (Sec. 3.5) or
+    "viterbi" (the exact best path, App. E)."""
     B = logits.shape[0]
     for t, n in ((logits, "logits"), (hidden, "hidden"), (target, "target")):
         _dev(t, n)
@@ -323,9 +347,14 @@ def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target:
     ws = ws or head.workspace(B)
     if tokens is None:
         tokens = torch.empty((B, head.L), dtype=torch.int32, device=logits.device)
-    _check(lib().lilicorr_select_block(head._h, B, logits.data_ptr(), hidden.data_ptr(),
-                                       target.data_ptr(), tokens.data_ptr(), ws.ptr, ws.nbytes,
-                                       _stream()), "select_block")
+    if walk == "greedy":
+        _check(lib().lilicorr_select_block(head._h, B, logits.data_ptr(), hidden.data_ptr(),
+                                           target.data_ptr(), tokens.data_ptr(), ws.ptr,
+                                           ws.nbytes, _stream()), "select_block")
+    else:
+        _check(lib().lilicorr_select_block_walk(head._h, B, logits.data_ptr(), hidden.data_ptr(),
+                                                target.data_ptr(), WALKS[walk], tokens.data_ptr(),
+                                                ws.ptr, ws.nbytes, _stream()), "select_block_walk")
     return tokens
 
 

@@ -644,10 +644,41 @@ lilicorr_status_t lilicorr_greedy_walk(int B, int L, int K, const float* anchor_
   return launch_pair_walk(a, stream);
 }
 
+lilicorr_status_t lilicorr_best_path(int B, int L, int K, const float* anchor_scores,
+                                     const float* pair_scores, const int32_t* ids, float sigma,
+                                     int32_t* choice, int32_t* tokens, float* path_score,
+                                     cudaStream_t stream) {
+  if (B < 0 || L <= 0 || L > LILICORR_MAX_L || K <= 0 || K > LILICORR_MAX_K)
+    return LILICORR_ERR_SHAPE;
+  if (!(sigma > 0.f) || !isfinite(sigma)) return LILICORR_ERR_ARG;
+  if (B == 0) return LILICORR_OK;
+  if (!anchor_scores || (L > 1 && !pair_scores) || !ids || !choice || !tokens)
+    return LILICORR_ERR_ARG;
+  if (pair_walk_smem_bytes(L, K, 0) > 200 * 1024) return LILICORR_ERR_SHAPE;
+  PairWalkArgs a;
+  memset(&a, 0, sizeof(a));
+  a.B = B; a.L = L; a.K = K; a.d = 0;
+  a.A = const_cast<float*>(anchor_scores); a.P = const_cast<float*>(pair_scores);
+  a.ids = ids; a.choice = choice; a.tokens = tokens;
+  a.walk_mode = LILICORR_WALK_VITERBI; a.sigma = sigma; a.path_score = path_score;
+  a.do_pairs = false; a.do_walk = true;
+  return launch_pair_walk(a, stream);
+}
+
 lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const void* logits,
                                         const void* drafter_hidden, const void* target_hidden,
                                         int32_t* tokens, void* ws, size_t ws_bytes,
                                         cudaStream_t stream) {
+  return lilicorr_select_block_walk(head, B, logits, drafter_hidden, target_hidden,
+                                    LILICORR_WALK_GREEDY, tokens, ws, ws_bytes, stream);
+}
+
+lilicorr_status_t lilicorr_select_block_walk(const lilicorr_head* head, int B, const void* logits,
+                                             const void* drafter_hidden,
+                                             const void* target_hidden, lilicorr_walk_t walk,
+                                             int32_t* tokens, void* ws, size_t ws_bytes,
+                                             cudaStream_t stream) {
+  if (walk != LILICORR_WALK_GREEDY && walk != LILICORR_WALK_VITERBI) return LILICORR_ERR_ARG;
   if (!head || B < 0) return LILICORR_ERR_ARG;
   if (B == 0) return LILICORR_OK;
   if (!logits || !drafter_hidden || !target_hidden || !tokens || !ws) return LILICORR_ERR_ARG;
@@ -679,6 +710,7 @@ lilicorr_status_t lilicorr_select_block(const lilicorr_head* head, int B, const 
   a.A = at<float>(ws, w.A); a.P = at<float>(ws, w.P);
   a.ids = ids; a.choice = at<int32_t>(ws, w.choice); a.tokens = tokens; a.margin = nullptr;
   a.do_pairs = true; a.do_walk = true;
+  a.walk_mode = walk; a.sigma = LILICORR_SIGMA;
   a.counters = at<uint32_t>(ws, w.pw_counters);
   return launch_pair_walk(a, stream);
 }

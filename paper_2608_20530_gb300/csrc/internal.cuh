@@ -268,6 +268,9 @@ struct PairWalkArgs {
   const int32_t* ids;                             // [B, L, K] (walk)
   int32_t* choice; int32_t* tokens; float* margin;
   bool do_pairs, do_walk;
+  int walk_mode;                                  // LILICORR_WALK_GREEDY / _VITERBI
+  float sigma;                                    // score scale of the exact path (Viterbi)
+  float* path_score;                              // [B] g of the chosen path (Viterbi), may be null
   uint32_t* counters;                             // [B] zeroed tickets (pairs + walk fused)
   bool scores_in_smem;                            // set by the launcher
 };

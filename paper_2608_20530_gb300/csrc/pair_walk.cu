@@ -14,7 +14,11 @@
 // scores into shared memory and walks them.
 // walk_kernel: grid B, the walk alone over given scores.
 // The walk is one warp: a warp argmax per step (ties to the lower index) and the
-// best-minus-second margin.
+// best-minus-second margin. In Viterbi mode (App. E) the same warp computes the exact
+// maximiser of the path score g(c) = sigma (A[c_1] + sum_s P[s-1, c_{s-1}, c_s]) instead:
+// lane k keeps the best score of a path ending at candidate k, one sweep over the slots
+// records each lane's best predecessor (ties to the lower index) in shared memory, and
+// lane 0 traces the path back from the best final candidate (ties to the lower index).
 #include "internal.cuh"
 
 namespace lilicorr {
@@ -61,10 +65,56 @@ __device__ void walk_sequence(const float* A, const float* P, int b, int L, int 
   }
 }
 
+// Exact best path of one sequence (one full warp). back: [L * K] bytes of shared memory.
+__device__ void viterbi_sequence(const float* A, const float* P, int b, int L, int K, float sigma,
+                                 const int32_t* ids, int32_t* choice, int32_t* tokens,
+                                 float* score, uint8_t* back) {
+  const int lane = threadIdx.x & 31;
+  float best = lane < K ? sigma * A[lane] : -INFINITY;
+  for (int s = 1; s < L; ++s) {
+    const float* Ps = P + (size_t)(s - 1) * K * K;
+    float bv = -INFINITY;
+    int bk = 0;
+    for (int k = 0; k < K; ++k) {
+      const float pk = __shfl_sync(0xffffffffu, best, k);
+      const float c = pk + sigma * (lane < K ? Ps[k * K + lane] : 0.f);
+      if (c > bv) { bv = c; bk = k; }             // strict: the lower predecessor on ties
+    }
+    if (lane < K) back[s * K + lane] = (uint8_t)bk;
+    best = lane < K ? bv : -INFINITY;
+  }
+  float v = best;
+  int bi = lane < K ? lane : 0x7fffffff;
+  warp_argmax(v, bi);
+  bi = __shfl_sync(0xffffffffu, bi, 0);
+  v = __shfl_sync(0xffffffffu, v, 0);
+  if (bi < 0 || bi >= K) bi = 0;
+  __syncwarp();
+  if (lane == 0) {
+    int c = bi;
+    for (int s = L - 1; s >= 0; --s) {
+      const size_t o = (size_t)b * L + s;
+      if (choice) choice[o] = c;
+      if (tokens) tokens[o] = ids[o * K + c];
+      if (s > 0) c = back[s * K + c];
+    }
+    if (score) score[b] = v;
+  }
+}
+
+__device__ __forceinline__ void run_walk(const PairWalkArgs& a, const float* A, const float* P,
+                                         int b, uint8_t* back) {
+  if (a.walk_mode == LILICORR_WALK_VITERBI)
+    viterbi_sequence(A, P, b, a.L, a.K, a.sigma, a.ids, a.choice, a.tokens, a.path_score, back);
+  else
+    walk_sequence(A, P, b, a.L, a.K, a.ids, a.choice, a.tokens, a.margin);
+}
+
 __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
   pdl_wait();
   extern __shared__ float sm[];
   __shared__ int s_last;
+  __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
   const int b = blockIdx.x, j = blockIdx.y;          // j = 0: anchor row; j >= 1: pair (j-1, j)
   const int L = a.L, K = a.K, d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = PW_THREADS / 32;
@@ -124,7 +174,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
     P = sm + K;
   }
   if (warp == 0) {
-    walk_sequence(A, P, b, L, K, a.ids, a.choice, a.tokens, a.margin);
+    run_walk(a, A, P, b, s_back);
     if (lane == 0) a.counters[b] = 0u;          // leave the workspace reusable
   }
 }
@@ -132,6 +182,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
 __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
   pdl_wait();
   extern __shared__ float sm[];
+  __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
   const int b = blockIdx.x, L = a.L, K = a.K;
   const int n_scores = K + (L - 1) * K * K;
   const float* A = a.A + (size_t)b * K;
@@ -142,7 +193,7 @@ __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
     A = sm;
     P = sm + K;
   }
-  if ((threadIdx.x >> 5) == 0) walk_sequence(A, P, b, L, K, a.ids, a.choice, a.tokens, a.margin);
+  if ((threadIdx.x >> 5) == 0) run_walk(a, A, P, b, s_back);
 }
 
 }  // namespace
