@@ -15,6 +15,9 @@ Everything here is plain, slow and in float64, written from the paper:
   restated step by step with library matmuls, no fusion or reordering.
 * pair scores (Eq. "pair"; Sec. 3.5), the greedy walk (Sec. 3.5), the path score
   (Eq. "pathscore") and the exact Viterbi maximiser (App. E).
+* the local next-candidate distributions (Eq. "localar") and decision gaps
+  (Eq. "margin") along a path; coverage, oracle prefix and prefix acceptance
+  against ground-truth tokens (Sec. 3.3 "Oracle-prefix supervision"; Sec. 3.1).
 
 Pinned by ``tests/test_oracle_*.py`` against closed forms, brute force,
 library routines and the paper's printed parameter counts. The scoring network's
@@ -344,6 +347,58 @@ def brute_force_paths(A: np.ndarray, P: np.ndarray, sigma: float = SIGMA):
     K = A.shape[0]
     for c in itertools.product(range(K), repeat=L):
         yield c, path_score(A, P, c, sigma)
+
+
+# =========================================================================== diagnostics
+def local_softmax(A: np.ndarray, P: np.ndarray, sigma: float = SIGMA) -> Tuple[np.ndarray, np.ndarray]:
+    """Eq. "localar": P(c_s = k | c_{s-1}) = softmax_k(z_s[k]) with node scores
+    z_s[k] = phi(s-1, c_{s-1}, k) = sigma * cos. Returns the anchor row's distribution
+    [K] (predecessor: the anchor) and, for every slot pair and predecessor k, the
+    distribution over successors [L-1, K, K] (last axis sums to 1)."""
+    def softmax(z):
+        z = np.asarray(z, np.float64)
+        e = np.exp(z - z.max())
+        return e / e.sum()
+    A = np.asarray(A, np.float64)
+    P = np.asarray(P, np.float64)
+    pa = softmax(sigma * A)
+    pp = np.zeros_like(P)
+    for s in range(P.shape[0]):
+        for k in range(P.shape[1]):
+            pp[s, k] = softmax(sigma * P[s, k])
+    return pa, pp
+
+
+def path_probs(A: np.ndarray, P: np.ndarray, c: Sequence[int], sigma: float = SIGMA):
+    """Along the path c: prob[s] = P(c_s | c_{s-1}) of Eq. "localar" (the anchor before
+    slot 0), gap[s] = z_s[c_s] - max_{k != c_s} z_s[k] (the decision gap of Eq. "margin";
+    +inf when K = 1) and log_prob = sum_s log prob[s]."""
+    pa, pp = local_softmax(A, P, sigma)
+    L = len(c)
+    prob = np.zeros(L)
+    gap = np.zeros(L)
+    for s in range(L):
+        z = sigma * (np.asarray(A, np.float64) if s == 0 else np.asarray(P[s - 1, c[s - 1]], np.float64))
+        prob[s] = pa[c[0]] if s == 0 else pp[s - 1, c[s - 1], c[s]]
+        others = np.delete(z, c[s])
+        gap[s] = z[c[s]] - others.max() if others.size else np.inf
+    return prob, gap, float(np.sum(np.log(prob)))
+
+
+def block_acceptance(ids: np.ndarray, tokens: np.ndarray, truth: np.ndarray):
+    """Against ground-truth tokens truth [L]: covered[s] = truth[s] is among slot s's K
+    candidates; the oracle prefix is the longest leading run of covered slots; the
+    accepted length is the longest leading run of slots whose chosen token equals the
+    truth (prefix acceptance: the verifier keeps tokens up to the first mismatch)."""
+    L = len(truth)
+    covered = np.array([int(truth[s] in set(int(x) for x in ids[s])) for s in range(L)])
+    oracle_prefix = 0
+    while oracle_prefix < L and covered[oracle_prefix]:
+        oracle_prefix += 1
+    accepted = 0
+    while accepted < L and int(tokens[accepted]) == int(truth[accepted]):
+        accepted += 1
+    return covered, oracle_prefix, accepted
 
 
 # =========================================================================== whole path
