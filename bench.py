@@ -230,13 +230,16 @@ def gen_blocks(wl, seeds, dev, chunk=50):
     logits = torch.empty((n, 1, wl.L, wl.V), dtype=tdt, device=dev)
     hidden = torch.empty((n, 1, wl.L, wl.H), dtype=tdt, device=dev)
     target = torch.empty((n, 1, wl.n_tgt, wl.H), dtype=tdt, device=dev)
+    planted = np.zeros((n, 1, wl.L), np.int32)
     for i in range(0, n, chunk):
         inp = workloads.batch_inputs(wl, seeds[i:i + chunk])
         m = inp["logits"].shape[0]
         logits[i:i + m, 0] = upload(inp["logits"], wl.dtype, dev)
         hidden[i:i + m, 0] = upload(inp["hidden"], wl.dtype, dev)
         target[i:i + m, 0] = upload(inp["target"], wl.dtype, dev)
-    return logits, hidden, target
+        if inp["planted"] is not None:
+            planted[i:i + m, 0] = inp["planted"]
+    return logits, hidden, target, planted
 
 
 def run_ours(args, world, rank, local):
@@ -257,7 +260,7 @@ def run_ours(args, world, rank, local):
         nblk = args.blocks or wl.blocks
         seeds = [s + rank * nblk for s in wl.block_seeds()[:nblk]] if nblk <= wl.blocks else \
             [wl.seed_base + i + rank * nblk for i in range(nblk)]
-        logits, hidden, target = gen_blocks(wl, seeds, dev)
+        logits, hidden, target, planted = gen_blocks(wl, seeds, dev)
         B = 1
     else:
         nblk = 1
@@ -265,6 +268,7 @@ def run_ours(args, world, rank, local):
         logits = upload(inp["logits"], wl.dtype, dev)[None]
         hidden = upload(inp["hidden"], wl.dtype, dev)[None]
         target = upload(inp["target"], wl.dtype, dev)[None]
+        planted = inp["planted"][None].astype(np.int32) if inp["planted"] is not None else None
         B = wl.B
         del inp
     ws = head.workspace(B)
@@ -400,6 +404,45 @@ def run_ours(args, world, rank, local):
     if ws.status() != 0:
         raise RuntimeError("device status set by the walk comparison")
 
+    # ---- diagnostics of the chosen blocks (Eq. "localar" probabilities and gaps along the
+    # walk; coverage / oracle prefix / accepted prefix against the planted tokens)
+    diag = None
+    if planted is not None:
+        nd = min(nblk, 100)
+        prefix_sum = acc_sum = 0
+        for i in range(nd):
+            tok = ll.select_block(head, logits[i], hidden[i], target[i], ws=ws, tokens=tokens[i])
+            inter = ll.select_block_intermediates(head, B, ws)
+            truth = torch.from_numpy(planted[i]).to(dev)
+            _, pre, acc = ll.block_acceptance(inter["ids"], tok, truth)
+            prefix_sum += int(pre.sum())
+            acc_sum += int(acc.sum())
+        inter = ll.select_block_intermediates(head, B, ws)
+        truth = torch.from_numpy(planted[nd - 1]).to(dev)
+
+        def diag_call():
+            ll.path_probs(inter["A"], inter["P"], inter["choice"])
+            ll.block_acceptance(inter["ids"], tokens[nd - 1], truth)
+        diag_call()
+        torch.cuda.synchronize()
+        dg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(dg):
+            for _ in range(50):
+                diag_call()
+        dg.replay()
+        torch.cuda.synchronize()
+        d0 = torch.cuda.Event(enable_timing=True)
+        d1 = torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        dg.replay()
+        d1.record(stream)
+        torch.cuda.synchronize()
+        diag = {"truth": "planted token per slot", "blocks": nd * B,
+                "mean_oracle_prefix": round(prefix_sum / (nd * B), 3),
+                "mean_accepted": round(acc_sum / (nd * B), 3),
+                "us_per_call": round(d0.elapsed_time(d1) * 1e3 / 50, 2),
+                "note": "path_probs + block_acceptance on one call's outputs"}
+
     # ---- roofline of the top-K pass: its launches back to back in one captured graph,
     # CUDA events on the launching stream around the replay
     rows = B * wl.L
@@ -456,6 +499,7 @@ def run_ours(args, world, rank, local):
                 "d2h_bytes_per_step": d2h,
                 "note": f"pinned host blocks cycled ({nh} distinct), copies captured with each call"},
         "gpu_launches": launches_per_call * (nblk if batch1 else 1) * args.steps,
+        "diagnostics": diag,
         "walk_viterbi": {"us_per_call": round(walk_ms["viterbi"] * 1e3, 2),
                          "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
                          "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),

@@ -218,6 +218,37 @@ lilicorr_status_t lilicorr_best_path(int B, int L, int K, const float* anchor_sc
                                      int32_t* choice, int32_t* tokens, float* path_score,
                                      cudaStream_t stream);
 
+/* Local next-candidate distributions (Eq. "localar"): with node scores z = sigma * score,
+ *   anchor_probs[b, k]      = softmax_k(sigma * A[b, :])[k]            (predecessor: the anchor)
+ *   pair_probs[b, s, k, k'] = softmax_k'(sigma * P[b, s, k, :])[k']    (predecessor k at slot s)
+ * anchor_scores [B, K], pair_scores [B, L-1, K, K] fp32 in; the probabilities fp32 out,
+ * same layouts. sigma > 0 (the paper's LILICORR_SIGMA). */
+lilicorr_status_t lilicorr_local_softmax(int B, int L, int K, const float* anchor_scores,
+                                         const float* pair_scores, float sigma,
+                                         float* anchor_probs, float* pair_probs,
+                                         cudaStream_t stream);
+
+/* Along a path choice [B, L] (candidate indices, e.g. a walk's choice or the ground
+ * truth's): prob[b, s] = P(c_s | c_{s-1}) of Eq. "localar" (the anchor precedes slot 0),
+ * gap[b, s] = z_s[c_s] - max_{k != c_s} z_s[k], the decision gap of Eq. "margin" (+inf when
+ * K = 1), log_prob[b] = sum_s log prob[b, s]. A choice outside [0, K) gives NaN for its
+ * step. Any output may be NULL. */
+lilicorr_status_t lilicorr_path_probs(int B, int L, int K, const float* anchor_scores,
+                                      const float* pair_scores, const int32_t* choice,
+                                      float sigma, float* prob, float* gap, float* log_prob,
+                                      cudaStream_t stream);
+
+/* Coverage and prefix acceptance against ground-truth tokens truth [B, L] int32 (Sec. 3.3
+ * "Oracle-prefix supervision"; Sec. 3.1): covered[b, s] = 1 if truth[b, s] is among
+ * ids[b, s, :] (the top-K candidates) else 0; oracle_prefix[b] = the longest leading run of
+ * covered slots; accepted[b] = the longest leading run of slots whose chosen token
+ * tokens[b, s] equals the truth (the verifier keeps tokens up to the first mismatch).
+ * ids [B, L, K], tokens [B, L] int32. Any output may be NULL. */
+lilicorr_status_t lilicorr_block_acceptance(int B, int L, int K, const int32_t* ids,
+                                            const int32_t* tokens, const int32_t* truth,
+                                            int32_t* covered, int32_t* oracle_prefix,
+                                            int32_t* accepted, cudaStream_t stream);
+
 /* Steps (1)-(4) fused: raw inputs to the chosen tokens.
  *   logits [B, L, V], drafter_hidden [B, L, H], target_hidden [B, n_tgt, H], all of
  *   head dtype; tokens [B, L] int32. ws: lilicorr_workspace_bytes(head, B). */

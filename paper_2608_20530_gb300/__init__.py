@@ -62,6 +62,9 @@ _SIGS = {
     "lilicorr_select_block": (_I, [_P, _I, _P, _P, _P, _P, _P, _S, _P]),
     "lilicorr_best_path": (_I, [_I, _I, _I, _P, _P, _P, ctypes.c_float, _P, _P, _P, _P]),
     "lilicorr_select_block_walk": (_I, [_P, _I, _P, _P, _P, _I, _P, _P, _S, _P]),
+    "lilicorr_local_softmax": (_I, [_I, _I, _I, _P, _P, ctypes.c_float, _P, _P, _P]),
+    "lilicorr_path_probs": (_I, [_I, _I, _I, _P, _P, _P, ctypes.c_float, _P, _P, _P, _P]),
+    "lilicorr_block_acceptance": (_I, [_I, _I, _I, _P, _P, _P, _P, _P, _P, _P]),
     "lilicorr_select_block_intermediates": (_I, [_P, _I, _P, _S] + [ctypes.POINTER(_P)] * 6),
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
@@ -331,6 +334,53 @@ def best_path(A: torch.Tensor, P: torch.Tensor, ids: torch.Tensor, sigma: float 
                                     ids.data_ptr(), float(sigma), choice.data_ptr(),
                                     tokens.data_ptr(), score.data_ptr(), _stream()), "best_path")
     return choice, tokens, score
+
+
+def local_softmax(A: torch.Tensor, P: torch.Tensor, sigma: float = SIGMA):
+    """Local next-candidate distributions (Eq. "localar"): anchor [B, K] and, per slot
+    pair and predecessor, over successors [B, L-1, K, K] (fp32)."""
+    B, K = A.shape
+    L = P.shape[1] + 1
+    for t, n in ((A, "anchor_scores"), (P, "pair_scores")):
+        _dev(t, n)
+    pa = torch.empty_like(A)
+    pp = torch.empty_like(P)
+    _check(lib().lilicorr_local_softmax(B, L, K, A.data_ptr(), P.data_ptr() if P.numel() else None,
+                                        float(sigma), pa.data_ptr(),
+                                        pp.data_ptr() if pp.numel() else None, _stream()),
+           "local_softmax")
+    return pa, pp
+
+
+def path_probs(A: torch.Tensor, P: torch.Tensor, choice: torch.Tensor, sigma: float = SIGMA):
+    """Along the path `choice` [B, L]: P(c_s | c_{s-1}) [B, L], decision gaps [B, L] and the
+    path's log-probability [B] (fp32)."""
+    B, K = A.shape
+    L = P.shape[1] + 1
+    for t, n in ((A, "anchor_scores"), (P, "pair_scores"), (choice, "choice")):
+        _dev(t, n)
+    prob = torch.empty((B, L), dtype=torch.float32, device=A.device)
+    gap = torch.empty_like(prob)
+    lp = torch.empty((B,), dtype=torch.float32, device=A.device)
+    _check(lib().lilicorr_path_probs(B, L, K, A.data_ptr(), P.data_ptr() if P.numel() else None,
+                                     choice.data_ptr(), float(sigma), prob.data_ptr(),
+                                     gap.data_ptr(), lp.data_ptr(), _stream()), "path_probs")
+    return prob, gap, lp
+
+
+def block_acceptance(ids: torch.Tensor, tokens: torch.Tensor, truth: torch.Tensor):
+    """Coverage [B, L], oracle prefix [B] and accepted prefix length [B] (int32) of chosen
+    tokens against ground-truth tokens."""
+    B, L, K = ids.shape
+    for t, n in ((ids, "ids"), (tokens, "tokens"), (truth, "truth")):
+        _dev(t, n)
+    covered = torch.empty((B, L), dtype=torch.int32, device=ids.device)
+    prefix = torch.empty((B,), dtype=torch.int32, device=ids.device)
+    acc = torch.empty_like(prefix)
+    _check(lib().lilicorr_block_acceptance(B, L, K, ids.data_ptr(), tokens.data_ptr(),
+                                           truth.data_ptr(), covered.data_ptr(), prefix.data_ptr(),
+                                           acc.data_ptr(), _stream()), "block_acceptance")
+    return covered, prefix, acc
 
 
 def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target: torch.Tensor,
