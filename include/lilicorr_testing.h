@@ -18,7 +18,9 @@ extern "C" {
  * bias and residual (fp32, residual with leading dimension ldc) may be NULL;
  * act 0 = none, 1 = SiLU. path selects the kernel: 0 = the network's own choice,
  * 1 = tiled CUDA-core kernel, 2 = few-row (split-N) CUDA-core kernel,
- * 3 = tensor cores (bf16 A and W only; LILICORR_ERR_DTYPE otherwise).
+ * 3 = tensor cores (bf16 A and W only; LILICORR_ERR_DTYPE otherwise),
+ * 4 = tensor cores for one tile of rows (M <= 128, Kd <= 512 a multiple of 64, N a
+ *     multiple of 32 (fp32 out) or 64 (bf16 out); LILICORR_ERR_SHAPE otherwise).
  * status: a device uint32 word that receives bounded-wait timeouts (may be NULL). */
 lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W,
                                        lilicorr_dtype_t w_dt, int ldw, void* C,

@@ -199,6 +199,7 @@ GemmArgs gemm(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, lili
 // tiled fp32 CUDA-core kernel (the fp32 head keeps fp32 arithmetic throughout).
 lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
   if (g.M <= 64) return launch_gemm_skinny(g, st);
+  if (gemm_small_supported(g)) return launch_gemm_small(g, st);
   if (gemm_tc_supported(g)) return launch_gemm_tc(g, st);
   return launch_gemm_simt(g, st);
 }
@@ -748,6 +749,7 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
     case 1: return launch_gemm_simt(g, stream);
     case 2: return launch_gemm_skinny(g, stream);
     case 3: return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_DTYPE;
+    case 4: return gemm_small_supported(g) ? launch_gemm_small(g, stream) : LILICORR_ERR_SHAPE;
   }
   return LILICORR_ERR_ARG;
 }

@@ -222,6 +222,9 @@ lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
 lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st);   // M <= 64
 bool gemm_tc_supported(const GemmArgs& g);
 lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
+// one tile of rows (M <= 128, Kd <= 512, a multiple of 64): whole-K TMA copies (gemm_small.cu)
+bool gemm_small_supported(const GemmArgs& g);
+lilicorr_status_t launch_gemm_small(const GemmArgs& g, cudaStream_t st);
 
 // scoring-network helpers (head_kernels.cu)
 // fused scoring network (net_fused.cu): one CTA per sequence, bf16 head with D = 256,

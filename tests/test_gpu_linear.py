@@ -1,6 +1,7 @@
 """GPU check of the scoring network's linear-layer kernels (building blocks of step 2)
 against a plain PyTorch fp32 matmul of the same bf16/fp32 operands: the tensor-core
-(tcgen05) kernel, the tiled and the few-row CUDA-core kernels, with bias, SiLU,
+(tcgen05) kernels (tiled, and one tile of rows with whole-K copies), the tiled and the
+few-row CUDA-core kernels, with bias, SiLU,
 residual, bf16 output, ragged M/N and long Kd."""
 import pytest
 import torch
@@ -64,3 +65,44 @@ def test_linear_fp32_operands_use_cuda_cores():
         ll.test_linear(A, W, path=3)
     C = ll.test_linear(A, W, path=0)
     assert (C - A @ W.T).abs().max().item() < 1e-4
+
+
+SMALL_CASES = [  # M, N, Kd: one tile of rows, whole-K copies
+    (128, 256, 256), (128, 768, 256), (128, 512, 512), (100, 256, 512), (65, 64, 64),
+    (1, 32, 128), (128, 1024, 256), (77, 192, 320),
+]
+
+
+@pytest.mark.parametrize("M,N,Kd", SMALL_CASES)
+def test_linear_one_row_tile(M, N, Kd):
+    ll = _ll()
+    g = torch.Generator(device="cuda").manual_seed(M * 5 + N + Kd)
+    A = torch.randn((M, Kd), generator=g, device="cuda").to(torch.bfloat16)
+    W = (0.02 * torch.randn((N, Kd), generator=g, device="cuda")).to(torch.bfloat16)
+    bias = 0.1 * torch.randn(N, generator=g, device="cuda")
+    res = torch.randn((M, N), generator=g, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    combos = [(0, None, None, torch.float32), (1, bias, None, torch.float32),
+              (0, bias, res, torch.float32)]
+    if N % 64 == 0:
+        combos.append((1, bias, None, torch.bfloat16))
+    for act, b, r, odt in combos:
+        C = ll.test_linear(A, W, odt, bias=b, residual=r, act=act, path=4, status=status)
+        torch.cuda.synchronize()
+        want = _ref(A, W, b, r, act)
+        tol = 2e-2 if odt == torch.bfloat16 else 2e-4 * max(1.0, (Kd / 256) ** 0.5)
+        err = (C.float() - want).abs().max().item()
+        assert err <= tol * max(1.0, want.abs().max().item()), (act, odt, err)
+    assert int(status.item()) == 0
+
+
+def test_linear_one_row_tile_rejects_other_shapes():
+    ll = _ll()
+    A = torch.randn((129, 256), device="cuda").to(torch.bfloat16)
+    W = torch.randn((256, 256), device="cuda").to(torch.bfloat16)
+    with pytest.raises(ll.LilicorrError):
+        ll.test_linear(A, W, path=4)                        # more than one tile of rows
+    A = torch.randn((128, 1024), device="cuda").to(torch.bfloat16)
+    W = torch.randn((256, 1024), device="cuda").to(torch.bfloat16)
+    with pytest.raises(ll.LilicorrError):
+        ll.test_linear(A, W, path=4)                        # Kd above 512
