@@ -13,8 +13,9 @@
 // of a sequence to finish (atomic ticket, nobody waits) loads the sequence's
 // scores into shared memory and walks them.
 // walk_kernel: grid B, the walk alone over given scores.
-// The walk is one warp: a warp argmax per step (ties to the lower index) and the
-// best-minus-second margin. In Viterbi mode (App. E) the same warp computes the exact
+// The walk is one warp: per step one butterfly over the candidates' lanes carries the best
+// (ties to the lower index) and the second-best score, for the choice and the
+// best-minus-second margin; the tokens are gathered for all slots after the walk. In Viterbi mode (App. E) the same warp computes the exact
 // maximiser of the path score g(c) = sigma (A[c_1] + sum_s P[s-1, c_{s-1}, c_s]) instead:
 // lane k keeps the best score of a path ending at candidate k, one sweep over the slots
 // records each lane's best predecessor (ties to the lower index) in shared memory, and
@@ -38,37 +39,51 @@ __device__ __forceinline__ void warp_argmax(float& v, int& idx) {
   }
 }
 
-// Walk one sequence (called by one full warp). A [K], P [(L-1)][K][K] in any memory.
-__device__ void walk_sequence(const float* A, const float* P, int b, int L, int K,
-                              const int32_t* ids, int32_t* choice, int32_t* tokens,
-                              float* margin) {
+// Best value (ties to the lower index), its index and the second-best value over the
+// first `width` lanes (a power of two): one butterfly that carries the top two.
+__device__ __forceinline__ void group_top2(float& v1, int& i1, float& v2, int width) {
+  for (int o = width >> 1; o > 0; o >>= 1) {
+    const float ov1 = __shfl_xor_sync(0xffffffffu, v1, o);
+    const int oi1 = __shfl_xor_sync(0xffffffffu, i1, o);
+    const float ov2 = __shfl_xor_sync(0xffffffffu, v2, o);
+    if (ov1 > v1 || (ov1 == v1 && oi1 < i1)) {
+      v2 = fmaxf(v1, ov2);
+      v1 = ov1;
+      i1 = oi1;
+    } else {
+      v2 = fmaxf(v2, ov1);
+    }
+  }
+}
+
+// Walk one sequence (called by one full warp). A [K], P [(L-1)][K][K] in any memory; the
+// choices go to path[L] in shared memory (the tokens are gathered after the walk, so no
+// step waits on a global load).
+__device__ void walk_sequence(const float* A, const float* P, int b, int L, int K, float* margin,
+                              uint8_t* path) {
   const int lane = threadIdx.x & 31;
+  int width = 1;                                 // lanes that hold candidates, rounded up
+  while (width < K) width <<= 1;
   int prev = 0;
   for (int s = 0; s < L; ++s) {
     const float* row = s == 0 ? A : P + ((size_t)(s - 1) * K + prev) * K;
-    const float v = lane < K ? row[lane] : -INFINITY;
-    float best = v;
+    float best = lane < K ? row[lane] : -INFINITY, second = -INFINITY;
     int bi = lane < K ? lane : 0x7fffffff;
-    warp_argmax(best, bi);
+    group_top2(best, bi, second, width);
     bi = __shfl_sync(0xffffffffu, bi, 0);      // one choice for the warp, even on NaN rows
-    best = __shfl_sync(0xffffffffu, best, 0);
     if (bi < 0 || bi >= K) bi = 0;
-    float second = (lane < K && lane != bi) ? v : -INFINITY;
-    second = warp_max(second);
     if (lane == 0) {
-      const size_t o = (size_t)b * L + s;
-      if (choice) choice[o] = bi;
-      if (tokens) tokens[o] = ids[o * K + bi];
-      if (margin) margin[o] = K > 1 ? best - second : INFINITY;
+      path[s] = (uint8_t)bi;
+      if (margin) margin[(size_t)b * L + s] = K > 1 ? best - second : INFINITY;
     }
     prev = bi;
   }
 }
 
-// Exact best path of one sequence (one full warp). back: [L * K] bytes of shared memory.
+// Exact best path of one sequence (one full warp). back: [L * K] bytes of shared memory;
+// the path goes to path[L] in shared memory.
 __device__ void viterbi_sequence(const float* A, const float* P, int b, int L, int K, float sigma,
-                                 const int32_t* ids, int32_t* choice, int32_t* tokens,
-                                 float* score, uint8_t* back) {
+                                 float* score, uint8_t* back, uint8_t* path) {
   const int lane = threadIdx.x & 31;
   float best = lane < K ? sigma * A[lane] : -INFINITY;
   for (int s = 1; s < L; ++s) {
@@ -93,9 +108,7 @@ __device__ void viterbi_sequence(const float* A, const float* P, int b, int L, i
   if (lane == 0) {
     int c = bi;
     for (int s = L - 1; s >= 0; --s) {
-      const size_t o = (size_t)b * L + s;
-      if (choice) choice[o] = c;
-      if (tokens) tokens[o] = ids[o * K + c];
+      path[s] = (uint8_t)c;
       if (s > 0) c = back[s * K + c];
     }
     if (score) score[b] = v;
@@ -103,11 +116,19 @@ __device__ void viterbi_sequence(const float* A, const float* P, int b, int L, i
 }
 
 __device__ __forceinline__ void run_walk(const PairWalkArgs& a, const float* A, const float* P,
-                                         int b, uint8_t* back) {
+                                         int b, uint8_t* back, uint8_t* path) {
   if (a.walk_mode == LILICORR_WALK_VITERBI)
-    viterbi_sequence(A, P, b, a.L, a.K, a.sigma, a.ids, a.choice, a.tokens, a.path_score, back);
+    viterbi_sequence(A, P, b, a.L, a.K, a.sigma, a.path_score, back, path);
   else
-    walk_sequence(A, P, b, a.L, a.K, a.ids, a.choice, a.tokens, a.margin);
+    walk_sequence(A, P, b, a.L, a.K, a.margin, path);
+  __syncwarp();
+  const int lane = threadIdx.x & 31;
+  for (int s = lane; s < a.L; s += 32) {        // choices and tokens, all slots at once
+    const size_t o = (size_t)b * a.L + s;
+    const int c = path[s];
+    if (a.choice) a.choice[o] = c;
+    if (a.tokens) a.tokens[o] = a.ids[o * a.K + c];
+  }
 }
 
 __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
@@ -115,6 +136,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
   extern __shared__ float sm[];
   __shared__ int s_last;
   __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
+  __shared__ uint8_t s_path[LILICORR_MAX_L];
   const int b = blockIdx.x, j = blockIdx.y;          // j = 0: anchor row; j >= 1: pair (j-1, j)
   const int L = a.L, K = a.K, d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = PW_THREADS / 32;
@@ -139,16 +161,27 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
     const float* o = j == 0 ? a.anchor + (size_t)b * d
                             : a.out + ((size_t)(b * L + j - 1) * K + r) * a.ld_vec;
     float oo = 0.f;
-    for (int c = lane; c < d; c += 32) oo += o[c] * o[c];
+    for (int c = lane; c < d; c += 32) oo = fmaf(o[c], o[c], oo);
     const float on = fmaxf(sqrtf(warp_sum(oo)), UNIT_EPS);
-    for (int k2 = 0; k2 < K; ++k2) {
-      float dot = 0.f;
-      for (int c = lane; c < d; c += 32) dot = fmaf(o[c], s_in[k2 * d + c], dot);
-      dot = warp_sum(dot);
+    for (int k0 = 0; k0 < K; k0 += 4) {          // four dot products at a time
+      float dot[4] = {0.f, 0.f, 0.f, 0.f};
+      for (int c = lane; c < d; c += 32) {
+        const float x = o[c];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (k0 + q < K) dot[q] = fmaf(x, s_in[(k0 + q) * d + c], dot[q]);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) dot[q] = warp_sum(dot[q]);
       if (lane == 0) {
-        const float v = dot / (on * s_inn[k2]);
-        if (j == 0) a.A[(size_t)b * K + k2] = v;
-        else a.P[((size_t)b * (L - 1) + (j - 1)) * K * K + (size_t)r * K + k2] = v;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int k2 = k0 + q;
+          if (k2 >= K) break;
+          const float v = dot[q] / (on * s_inn[k2]);
+          if (j == 0) a.A[(size_t)b * K + k2] = v;
+          else a.P[((size_t)b * (L - 1) + (j - 1)) * K * K + (size_t)r * K + k2] = v;
+        }
       }
     }
   }
@@ -174,7 +207,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
     P = sm + K;
   }
   if (warp == 0) {
-    run_walk(a, A, P, b, s_back);
+    run_walk(a, A, P, b, s_back, s_path);
     if (lane == 0) a.counters[b] = 0u;          // leave the workspace reusable
   }
 }
@@ -183,6 +216,7 @@ __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
   pdl_wait();
   extern __shared__ float sm[];
   __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
+  __shared__ uint8_t s_path[LILICORR_MAX_L];
   const int b = blockIdx.x, L = a.L, K = a.K;
   const int n_scores = K + (L - 1) * K * K;
   const float* A = a.A + (size_t)b * K;
@@ -193,7 +227,7 @@ __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
     A = sm;
     P = sm + K;
   }
-  if ((threadIdx.x >> 5) == 0) run_walk(a, A, P, b, s_back);
+  if ((threadIdx.x >> 5) == 0) run_walk(a, A, P, b, s_back, s_path);
 }
 
 }  // namespace

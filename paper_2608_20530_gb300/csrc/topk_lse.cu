@@ -6,15 +6,21 @@
 //   * grid = (splits, rows): each CTA streams one contiguous chunk of one row with
 //     16-byte loads, a batch of 4 per thread in flight;
 //   * every thread keeps an online (max, sum exp) pair, merged by warp shuffles;
-//   * candidates are order-preserving 64-bit keys (value, then lower id first); each
-//     warp keeps its top-K as a sorted list in registers (lane i holds the i-th key).
-//     The hot loop costs one compare per batch: a warp looks at a batch only if some
-//     lane's batch maximum reaches the threshold, the larger of the warp's own K-th
-//     value and the CTA's (shared memory; every warp's K-th value bounds the CTA's
-//     K-th from below). While its list is not full, a warp raises the threshold to
-//     the K-th largest lane maximum of the batch (each lane maximum is a distinct
-//     element, so K elements reach it). Elements that pass are inserted one at a
-//     time with a ballot (position) and a shuffle (shift);
+//   * candidates are order-preserving 64-bit keys (value, then lower id first). Each
+//     warp appends the elements that reach its value bound to a key buffer in shared
+//     memory (a ballot for the slots). The hot loop costs one compare per batch: a warp
+//     looks at a batch only if some lane's batch maximum reaches the bound. The bound
+//     is the largest of three lower bounds on the CTA's K-th value: the K-th largest of
+//     the warp's 32 running lane maxima (each a distinct element; used until the buffer
+//     holds K keys), the K-th key of the buffer (compacted by rank counting whenever it
+//     holds 2K keys), and a CTA-wide bound in shared memory. Every warp publishes its
+//     r-th largest lane maximum (r = ceil(K / warps)); the smallest of those has r
+//     distinct elements at or above it in each of the warps, K in all, so it bounds the
+//     CTA's K-th value from below while each warp alone has seen only a fraction of the
+//     row;
+//   * the arithmetic runs on packed pairs: the batch maxima on raw bf16x2 words, the
+//     exponent arguments and the running sums as f32x2 (one instruction per two
+//     logits), one ex2 per logit;
 //   * the CTA merges its warps' lists by rank counting; with several splits per
 //     row the last CTA to finish (atomic ticket, no waiting) merges the splits'
 //     partial (max, sum, top-K) records and writes ids, logp and lse.
@@ -61,6 +67,32 @@ __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// Packed fp32 pairs (one register pair, one instruction for both halves).
+__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack2(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.ftz.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.ftz.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// larger of two bf16 pairs, per half (exact; a NaN half yields the other operand's half)
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+  uint32_t d;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  return d;
 }
 
 // Rank counting: each key of keys[0..n) (distinct apart from zeros, which mean "empty")
@@ -145,6 +177,12 @@ template <> struct Vec<uint16_t> {        // bf16
     }
   }
   __device__ static float scalar(const uint16_t* p, size_t i) { return bf16_to_f32(p[i]); }
+  // largest of the 8 values (NaN ignored), on the packed words
+  __device__ static float vmax(const uint4& v) {
+    const uint32_t m = max_bf16x2(max_bf16x2(v.x, v.y), max_bf16x2(v.z, v.w));
+    return fmaxf(__uint_as_float(m << 16), __uint_as_float(m & 0xFFFF0000u));
+  }
+  static constexpr uint32_t NEG_INF4 = 0xFF80FF80u;       // two bf16 -inf
 };
 template <> struct Vec<float> {
   static constexpr int N = 4;
@@ -153,6 +191,11 @@ template <> struct Vec<float> {
     x[2] = __uint_as_float(v.z); x[3] = __uint_as_float(v.w);
   }
   __device__ static float scalar(const float* p, size_t i) { return p[i]; }
+  __device__ static float vmax(const uint4& v) {
+    return fmaxf(fmaxf(__uint_as_float(v.x), __uint_as_float(v.y)),
+                 fmaxf(__uint_as_float(v.z), __uint_as_float(v.w)));
+  }
+  static constexpr uint32_t NEG_INF4 = 0xFF800000u;       // fp32 -inf
 };
 
 // K-th largest (K <= 32) of one value per lane, by a bitonic sort across the warp.
@@ -173,9 +216,10 @@ __device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
 //   * the K-th largest running maximum over the warp's lanes (each lane's running maximum
 //     is a distinct element, so K elements reach it), and
 //   * the K-th key of the buffer after a compaction, and the CTA-wide bound (the largest
-//     bound any warp of the CTA has published).
+//     bound any warp of the CTA has published, and the smallest of the warps' published
+//     r-th largest lane maxima).
 // Appending costs a ballot and a store; the buffer is compacted to its K largest keys by
-// rank counting only when it fills.
+// rank counting once it holds 2K keys (or when it would overflow).
 constexpr int TK_CAP = 96;
 
 struct WarpCand {
@@ -236,32 +280,28 @@ __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], ui
 // CHECK = false: every vector is inside the chunk (no predicates). The values stay in
 // registers; the online (max, sum exp) takes one rescale check per batch; the warp looks
 // at the values for candidates only if some lane's batch maximum reaches the bound.
+// s_wtop[warp]: the warps' published r-th largest lane maxima (r = ceil(K / TK_WARPS)).
 template <typename T, bool CHECK>
 __device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int it, int v_end,
                                               uint32_t id_base, int K, int tid, int lane,
                                               float& m, float& s, WarpCand& w,
-                                              uint32_t* s_cta_thr) {
+                                              uint32_t* s_cta_thr, float* s_wtop) {
   constexpr int VEC = Vec<T>::N;
   uint4 raw[TK_UNROLL];
 #pragma unroll
   for (int u = 0; u < TK_UNROLL; ++u) {
     const int v = it + u * TK_THREADS + tid;
-    raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(0, 0, 0, 0);
+    constexpr uint32_t NI = Vec<T>::NEG_INF4;          // outside the chunk: contributes nothing
+    raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(NI, NI, NI, NI);
   }
   float x[TK_UNROLL][VEC];
   float vmx[TK_UNROLL];
   float bmax = -INFINITY;
 #pragma unroll
   for (int u = 0; u < TK_UNROLL; ++u) {
+    vmx[u] = Vec<T>::vmax(raw[u]);
+    bmax = fmaxf(bmax, vmx[u]);
     Vec<T>::unpack(raw[u], x[u]);
-    if (CHECK && it + u * TK_THREADS + tid >= v_end)
-#pragma unroll
-      for (int j = 0; j < VEC; ++j) x[u][j] = -INFINITY;   // contributes nothing
-    float mx = x[u][0];
-#pragma unroll
-    for (int j = 1; j < VEC; ++j) mx = fmaxf(mx, x[u][j]);
-    vmx[u] = mx;
-    bmax = fmaxf(bmax, mx);
   }
   // online log-sum-exp, one rescale per batch (rarely taken after the first batches)
   if (bmax > m) {
@@ -270,28 +310,58 @@ __device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int 
   }
   if (m != -INFINITY) {
     const float ml = m * LOG2E;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint64_t l2 = pack2(LOG2E, LOG2E), nm = pack2(-ml, -ml);
+    uint64_t a0 = pack2(0.f, 0.f), a1 = a0;
 #pragma unroll
     for (int u = 0; u < TK_UNROLL; ++u)
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) acc[j & 3] += ex2(fmaf(x[u][j], LOG2E, -ml));
-    s += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      for (int j = 0; j < VEC; j += 2) {
+        float t0, t1;
+        unpack2(fma2(pack2(x[u][j], x[u][j + 1]), l2, nm), t0, t1);
+        const uint64_t e = pack2(ex2(t0), ex2(t1));
+        if ((j >> 1) & 1) a1 = add2(a1, e); else a0 = add2(a0, e);
+      }
+    float p0, p1, p2, p3;
+    unpack2(a0, p0, p1);
+    unpack2(a1, p2, p3);
+    s += (p0 + p1) + (p2 + p3);
   }
   // candidates: only when some lane's batch maximum reaches the current bound
   w.thr = fmaxf(w.thr, unord32(*(volatile uint32_t*)s_cta_thr));
-  if (__any_sync(FULL, bmax >= w.thr)) {
-    // tighten the bound with the K-th largest running lane maximum first
+  if (!__any_sync(FULL, bmax >= w.thr)) return;
+  {
+    // the CTA-wide bound from the warps' published lane maxima
+    const int r = (K + TK_WARPS - 1) / TK_WARPS;
+    const float mine = r == 1 ? warp_max(m) : warp_kth_largest(m, r, lane);
+    volatile float* wtop = s_wtop;
+    if (lane == 0) wtop[tid >> 5] = mine;             // lane maxima only grow
+    __syncwarp();
+    float cb = INFINITY;
+#pragma unroll
+    for (int i = 0; i < TK_WARPS; ++i) cb = fminf(cb, wtop[i]);
+    if (cb > w.thr) {
+      w.thr = cb;
+      if (lane == 0) atomicMax(s_cta_thr, ord32(cb));
+    }
+  }
+  if (!__any_sync(FULL, bmax >= w.thr)) return;
+  if (w.n < K) {
+    // until the buffer holds K keys: the K-th largest running lane maximum
     const float tb = warp_kth_largest(m, K, lane);
     if (tb > w.thr) {
       w.thr = tb;
       if (lane == 0) atomicMax(s_cta_thr, ord32(tb));
     }
+  }
 #pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u) {
-      if (!__any_sync(FULL, vmx[u] >= w.thr)) continue;
-      const int v = it + u * TK_THREADS + tid;
-      warp_append<VEC>(w, x[u], id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
-    }
+  for (int u = 0; u < TK_UNROLL; ++u) {
+    if (!__any_sync(FULL, vmx[u] >= w.thr)) continue;
+    const int v = it + u * TK_THREADS + tid;
+    warp_append<VEC>(w, x[u], id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
+  }
+  if (w.n >= 2 * K) {                                  // the buffer's K-th key bounds it
+    warp_compact(w, K, lane);
+    if (lane == 0) atomicMax(s_cta_thr, ord32(w.thr));
   }
 }
 
@@ -315,6 +385,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ float s_m[TK_WARPS], s_s[TK_WARPS];
   __shared__ uint32_t s_cta_thr;                // CTA-wide value bound (order image)
+  __shared__ float s_wtop[TK_WARPS];            // the warps' r-th largest lane maxima
   __shared__ int s_last, s_count;
   __shared__ uint64_t s_bound;
 
@@ -336,6 +407,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   w.n = 0;
   w.thr = -INFINITY;
   if (tid == 0) s_cta_thr = ord32(-INFINITY);
+  if (tid < TK_WARPS) s_wtop[tid] = -INFINITY;
   __syncthreads();
 
   float m = -INFINITY, s = 0.f;
@@ -359,9 +431,9 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   constexpr int STEP = TK_UNROLL * TK_THREADS;
   const int full_end = v_begin + (v_end - v_begin) / STEP * STEP;
   for (int it = v_begin; it < full_end; it += STEP)
-    process_batch<T, false>(vp, it, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr);
+    process_batch<T, false>(vp, it, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
   if (full_end < v_end)
-    process_batch<T, true>(vp, full_end, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr);
+    process_batch<T, true>(vp, full_end, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
 
   // (max, sum) of the warp, then of the CTA
   const float wm = warp_max(m);
