@@ -246,6 +246,7 @@ def run_ours(args, world, rank, local):
     import __graft_entry__
     __graft_entry__.build()
     import paper_2608_20530_gb300 as ll
+    from paper_2608_20530_gb300 import shards
 
     dev = torch.device("cuda", torch.cuda.current_device())
     wl = workloads.WORKLOADS[args.workload]
@@ -474,6 +475,44 @@ def run_ours(args, world, rank, local):
                 "traffic": profiled_traffic("topk_lse.cu", wl.name),
                 "alg_bytes_per_launch": alg_bytes, "us_per_launch": round(tk_ms * 1e3, 3)}
 
+    # ---- the vocabulary-sharded pass (a tensor-parallel LM head's logits), simulated on
+    # this GPU: P contiguous vocabulary slices, each summarised into per-row records
+    # (what one rank computes), then the merge of the gathered records
+    P = 4
+    sl = [flat[0][:, a:b].contiguous() for a, b in shards.bounds(wl.V, P)]
+    sws = [ll.Workspace(ll.lib().lilicorr_topk_lse_partial_workspace_bytes(rows, t.shape[1], wl.K))
+           for t in sl]
+    recs = torch.stack([ll.topk_lse_partial(t, wl.K, a, ws=w)
+                        for t, (a, _), w in zip(sl, shards.bounds(wl.V, P), sws)])
+    torch.cuda.synchronize()
+
+    def timed(fn, n=20):
+        fn()
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            for _ in range(n):
+                fn()
+        gr.replay()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        gr.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / n
+
+    part_us = timed(lambda: ll.topk_lse_partial(sl[0], wl.K, 0, ws=sws[0]))
+    merge_us = timed(lambda: ll.topk_lse_merge(recs, wl.K))
+    sharded = {"shards": P, "partial_us_per_rank": round(part_us, 2),
+               "merge_us": round(merge_us, 2),
+               "gather_bytes_per_rank": rows * ll.topk_partial_bytes(wl.K),
+               "note": "one rank's slice (V/%d columns of every row) and the merge of %d "
+                       "ranks' records, both on this GPU; the all-gather itself is not timed"
+                       % (P, P)}
+    del sl, sws, recs
+
     l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
     in_bytes = logits.numel() * es
     if in_bytes > l2_bytes:
@@ -504,6 +543,7 @@ def run_ours(args, world, rank, local):
                          "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
                          "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
                          "sample": f"{nv} calls of this workload, best of 3"},
+        "vocab_sharded": sharded,
         "roofline": roofline,
     }
     if rank == 0 and not args.no_cpu_baseline:

@@ -142,6 +142,37 @@ lilicorr_status_t lilicorr_topk_lse(const void* logits, lilicorr_dtype_t dtype, 
                                     int K, int32_t* ids, float* logp, float* lse, void* ws,
                                     size_t ws_bytes, cudaStream_t stream);
 
+/* Step (1) over a vocabulary split into P shards (the logits of a tensor-parallel LM
+ * head, each rank holding the columns of its vocabulary slice). Each shard emits one
+ * partial record per row; the records of all shards, gathered in shard order, merge into
+ * exactly what lilicorr_topk_lse computes on the whole row (the same ids; the normaliser
+ * up to fp32 rounding of the combination). The log-sum-exp combines associatively:
+ * lse = M + log sum_p s_p exp(m_p - M), M = max_p m_p, and every global top-K element is
+ * in its shard's top-K (the lower-id rule holds across shards through the ids).
+ * Partial record of one row, lilicorr_topk_partial_bytes(K) = 8 + 8K bytes:
+ *   float m;        the shard row's maximum logit (-inf if it has none)
+ *   float s;        sum_v exp(logits[v] - m) over the shard row
+ *   float val[K];   the shard row's K largest logits, descending, ties to the lower id
+ *   int32 id[K];    their vocabulary ids (column + id_offset); -1 (val -inf) when the
+ *                   shard row has fewer than K elements
+ * lilicorr_topk_lse_partial: logits [rows, V] of dtype is the shard (V >= 1, any K <=
+ *   LILICORR_MAX_K, K may exceed V), id_offset the vocabulary id of its column 0 (>= 0),
+ *   partial [rows] records (device, 8-byte aligned), ws a zero-filled workspace of at least
+ *   lilicorr_topk_lse_partial_workspace_bytes(rows, V, K) bytes. A shard row may be all
+ *   -inf; non-finite results are reported by the merge.
+ * lilicorr_topk_lse_merge: partials [P][rows] records (the shards' outputs in any order;
+ *   the ids carry the offsets), 1 <= P and P*K <= 512; ids/logp/lse as lilicorr_topk_lse;
+ *   status: a device uint32 word (may be NULL) that receives LILICORR_ERR_NONFINITE for a
+ *   row whose merged normaliser is not finite. */
+size_t lilicorr_topk_partial_bytes(int K);
+size_t lilicorr_topk_lse_partial_workspace_bytes(int rows, int V, int K);
+lilicorr_status_t lilicorr_topk_lse_partial(const void* logits, lilicorr_dtype_t dtype, int rows,
+                                            int V, int K, int32_t id_offset, void* partial,
+                                            void* ws, size_t ws_bytes, cudaStream_t stream);
+lilicorr_status_t lilicorr_topk_lse_merge(const void* partials, int P, int rows, int K,
+                                          int32_t* ids, float* logp, float* lse, uint32_t* status,
+                                          cudaStream_t stream);
+
 /* Step (1) without a caller workspace. Not from the paper (it has no counterpart
  * there): an addition for callers that cannot allocate device memory at the point
  * where they select a block. Examples: a serving process whose memory pool has claimed

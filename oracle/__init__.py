@@ -115,6 +115,42 @@ def topk_lse(x: np.ndarray, K: int) -> Tuple[np.ndarray, np.ndarray, float]:
     return ids, x[ids] - lse, lse
 
 
+def topk_lse_partial(x: np.ndarray, K: int, id_offset: int):
+    """One vocabulary shard's summary of a slot row (the vocabulary-sharded step (1) of a
+    tensor-parallel LM head): the shard's maximum m, s = sum exp(x - m) over the shard,
+    and its K largest logits with their vocabulary ids (column + id_offset) by the same
+    full stable sort as topk_lse, padded with (-inf, -1) when the shard is narrower than
+    K. m = -inf and s = 0 for a shard holding only -inf. Returns (m, s, vals[K], ids[K])."""
+    x = np.asarray(x, dtype=np.float64)
+    V = x.shape[0]
+    m = float(x.max()) if V else -np.inf
+    s = float(np.sum(np.exp(x - m))) if np.isfinite(m) else 0.0
+    order = np.lexsort((np.arange(V), -x))[:K]
+    vals = np.full(K, -np.inf)
+    ids = np.full(K, -1, dtype=np.int64)
+    vals[:len(order)] = x[order]
+    ids[:len(order)] = order + id_offset
+    return m, s, vals, ids
+
+
+def merge_partials(parts, K: int) -> Tuple[np.ndarray, np.ndarray, float]:
+    """Combine shard summaries (any order) into topk_lse's result for the whole row:
+    lse = M + log sum_p s_p exp(m_p - M) with M = max_p m_p, and the K largest of the
+    union of the shards' candidates by (value descending, id ascending)."""
+    ms = np.array([p[0] for p in parts], dtype=np.float64)
+    ss = np.array([p[1] for p in parts], dtype=np.float64)
+    M = ms.max()
+    if not np.isfinite(M):
+        raise ValueError("row has NaN, +inf, or is all -inf")
+    lse = float(M + np.log(np.sum(ss * np.exp(ms - M))))
+    vals = np.concatenate([p[2] for p in parts])
+    ids = np.concatenate([p[3] for p in parts])
+    keep = ids >= 0
+    vals, ids = vals[keep], ids[keep]
+    order = np.lexsort((ids, -vals))[:K]
+    return ids[order].astype(np.int64), vals[order] - lse, lse
+
+
 # =========================================================================== step a2
 def confidence_features(logp: np.ndarray) -> np.ndarray:
     """Five confidence scalars per candidate of one slot (App. A "Architecture"):

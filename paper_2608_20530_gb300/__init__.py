@@ -70,6 +70,10 @@ _SIGS = {
     "lilicorr_launch_count": (ctypes.c_uint64, []),
     "lilicorr_test_fused_path": (_I, [_P, _I]),
     "lilicorr_topk_lse_noalloc_max_bytes": (_S, []),
+    "lilicorr_topk_partial_bytes": (_S, [_I]),
+    "lilicorr_topk_lse_partial_workspace_bytes": (_S, [_I, _I, _I]),
+    "lilicorr_topk_lse_partial": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _S, _P]),
+    "lilicorr_topk_lse_merge": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _P]),
     "lilicorr_topk_lse_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
     "lilicorr_test_linear": (_I, [_P, _I, _I, _P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I,
                                   _P, _P]),
@@ -264,6 +268,45 @@ def topk_lse_noalloc(logits: torch.Tensor, K: int):
     _check(lib().lilicorr_topk_lse_noalloc(logits.data_ptr(), _dtype_code(logits), rows, V, K,
                                            ids.data_ptr(), logp.data_ptr(), lse.data_ptr(),
                                            _stream()), "topk_lse_noalloc")
+    return ids, logp, lse
+
+
+def topk_partial_bytes(K: int) -> int:
+    """Bytes of one row's partial record of a vocabulary shard (8 + 8K)."""
+    return 8 + 8 * int(K)
+
+
+def topk_lse_partial(logits: torch.Tensor, K: int, id_offset: int,
+                     ws: Optional[Workspace] = None) -> torch.Tensor:
+    """Partial records [rows, 8 + 8K] (uint8) of a vocabulary shard: logits [..., V_shard]
+    whose column 0 is vocabulary id ``id_offset`` (see lilicorr_topk_lse_partial)."""
+    _dev(logits, "logits")
+    V = logits.shape[-1]
+    rows = logits.numel() // V if V else 0
+    need = int(lib().lilicorr_topk_lse_partial_workspace_bytes(rows, V, K))
+    if ws is None:
+        ws = Workspace(need, logits.device)
+    rec = torch.empty((rows, topk_partial_bytes(K)), dtype=torch.uint8, device=logits.device)
+    _check(lib().lilicorr_topk_lse_partial(logits.data_ptr(), _dtype_code(logits), rows, V, K,
+                                           int(id_offset), rec.data_ptr(), ws.ptr, ws.nbytes,
+                                           _stream()), "topk_lse_partial")
+    return rec
+
+
+def topk_lse_merge(partials: torch.Tensor, K: int, status: Optional[torch.Tensor] = None):
+    """Merge the shards' records [P, rows, 8 + 8K] into (ids [rows, K] int32, logp [rows, K],
+    lse [rows]) as topk_lse computes them on whole rows."""
+    _dev(partials, "partials")
+    if partials.dim() != 3 or partials.shape[2] != topk_partial_bytes(K):
+        raise ValueError("partials must be [P, rows, 8 + 8K] bytes")
+    P, rows = partials.shape[0], partials.shape[1]
+    dev = partials.device
+    ids = torch.empty((rows, K), dtype=torch.int32, device=dev)
+    logp = torch.empty((rows, K), dtype=torch.float32, device=dev)
+    lse = torch.empty((rows,), dtype=torch.float32, device=dev)
+    _check(lib().lilicorr_topk_lse_merge(partials.contiguous().data_ptr(), P, rows, K,
+                                         ids.data_ptr(), logp.data_ptr(), lse.data_ptr(),
+                                         _ptr(status), _stream()), "topk_lse_merge")
     return ids, logp, lse
 
 

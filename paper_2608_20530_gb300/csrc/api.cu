@@ -579,6 +579,43 @@ lilicorr_status_t lilicorr_topk_lse(const void* logits, lilicorr_dtype_t dtype, 
                          stream);
 }
 
+size_t lilicorr_topk_partial_bytes(int K) {
+  return K > 0 && K <= LILICORR_MAX_K ? topk_partial_bytes(K) : 0;
+}
+
+size_t lilicorr_topk_lse_partial_workspace_bytes(int rows, int V, int K) {
+  if (rows < 0 || V <= 0 || K <= 0 || K > LILICORR_MAX_K) return 0;
+  size_t a = topk_ws_bytes(rows, V, K, LILICORR_F32), b = topk_ws_bytes(rows, V, K, LILICORR_BF16);
+  return a > b ? a : b;
+}
+
+lilicorr_status_t lilicorr_topk_lse_partial(const void* logits, lilicorr_dtype_t dtype, int rows,
+                                            int V, int K, int32_t id_offset, void* partial,
+                                            void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (dtype != LILICORR_F32 && dtype != LILICORR_BF16) return LILICORR_ERR_DTYPE;
+  if (rows < 0 || V <= 0 || K <= 0 || K > LILICORR_MAX_K) return LILICORR_ERR_SHAPE;
+  if (id_offset < 0 || (int64_t)id_offset + V > INT32_MAX) return LILICORR_ERR_ARG;
+  if (rows == 0) return LILICORR_OK;
+  if (!logits || !partial || !ws) return LILICORR_ERR_ARG;
+  if (!aligned16(logits) || !aligned16(ws) || (reinterpret_cast<uintptr_t>(partial) & 7))
+    return LILICORR_ERR_ARG;
+  if (ws_bytes < lilicorr_topk_lse_partial_workspace_bytes(rows, V, K)) return LILICORR_ERR_WORKSPACE;
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  return launch_topk_lse(logits, dtype, rows, V, K, nullptr, nullptr, nullptr,
+                         reinterpret_cast<uint32_t*>(w), reinterpret_cast<uint32_t*>(w + 256),
+                         w + 256 + align_up((size_t)rows * 4, 256), stream, partial, id_offset);
+}
+
+lilicorr_status_t lilicorr_topk_lse_merge(const void* partials, int P, int rows, int K,
+                                          int32_t* ids, float* logp, float* lse, uint32_t* status,
+                                          cudaStream_t stream) {
+  if (rows < 0 || P < 1 || K <= 0 || K > LILICORR_MAX_K || P * K > 512) return LILICORR_ERR_SHAPE;
+  if (rows == 0) return LILICORR_OK;
+  if (!partials || !ids || !logp || !lse) return LILICORR_ERR_ARG;
+  if (reinterpret_cast<uintptr_t>(partials) & 7) return LILICORR_ERR_ARG;
+  return launch_topk_merge(partials, P, rows, K, ids, logp, lse, status, stream);
+}
+
 size_t lilicorr_workspace_bytes(const lilicorr_head* head, int B) {
   if (!head || B < 0) return 0;
   return ws_layout(head->desc, B).total;

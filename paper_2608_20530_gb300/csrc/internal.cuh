@@ -201,9 +201,17 @@ size_t topk_ws_bytes(int rows, int V, int K, lilicorr_dtype_t dt);
 
 // ----------------------------------------------------------------------------- launchers
 // (1) top-K + log-normaliser. ws: status word at offset 0, then counters, partials.
+// partial_out non-null: write each row's public partial record (see
+// lilicorr_topk_lse_partial) with id_offset added to its ids instead of ids/logp/lse
 lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int rows, int V, int K,
                                   int32_t* ids, float* logp, float* lse, uint32_t* status,
-                                  uint32_t* counters, void* partials, cudaStream_t st);
+                                  uint32_t* counters, void* partials, cudaStream_t st,
+                                  void* partial_out = nullptr, int32_t id_offset = 0);
+// bytes of one row's partial record: max, sum, K values, K ids
+__host__ __device__ constexpr size_t topk_partial_bytes(int K) { return 8 + 8 * (size_t)K; }
+// merge P shards' records [P][rows][topk_partial_bytes(K)] into the final outputs
+lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K, int32_t* ids,
+                                    float* logp, float* lse, uint32_t* status, cudaStream_t st);
 
 // Generic linear layer C = act(A W^T + bias [+ bias_rows[m / rows_per_bias]]) [+ residual].
 enum { ACT_NONE = 0, ACT_SILU = 1 };

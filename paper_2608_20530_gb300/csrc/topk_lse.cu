@@ -370,12 +370,48 @@ struct Rec {            // partial record of one (row, split)
   uint64_t keys[1];     // [K]
 };
 
+// Where a row's result goes: the final outputs (ids, logp, lse), or, for one vocabulary
+// shard, the row's public partial record (running max, sum of exp below it, the shard's
+// top-K values and ids with the shard's id offset added; empty entries -inf / -1).
+struct PartialOut {
+  unsigned char* rec;       // [rows][partial_bytes(K)], or null for the final outputs
+  int32_t id_offset;
+};
+
+// Warp 0 of the CTA that completes row `row`: (m, s) of the row, its top-K keys in s_top.
+__device__ __forceinline__ void write_row(int row, int K, float m, float s, const uint64_t* s_top,
+                                          const PartialOut& pout, int32_t* ids, float* logp,
+                                          float* lse, uint32_t* status, int lane) {
+  if (pout.rec) {
+    unsigned char* r = pout.rec + (size_t)row * topk_partial_bytes(K);
+    float* rf = reinterpret_cast<float*>(r);
+    int32_t* ri = reinterpret_cast<int32_t*>(r + 8 + 4 * (size_t)K);
+    if (lane == 0) { rf[0] = m; rf[1] = s; }
+    if (lane < K) {
+      const uint64_t k = s_top[lane];
+      rf[2 + lane] = k ? key_value(k) : -INFINITY;
+      ri[lane] = k ? key_id(k) + pout.id_offset : -1;
+    }
+    return;
+  }
+  const float l = m + logf(s);
+  if (lane == 0) {
+    lse[row] = l;
+    if (!isfinite(l)) set_status(status, LILICORR_ERR_NONFINITE);
+  }
+  if (lane < K) {
+    const uint64_t k = s_top[lane];
+    ids[(size_t)row * K + lane] = key_id(k);
+    logp[(size_t)row * K + lane] = key_value(k) - l;
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(TK_THREADS, 4)
 topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chunk_vecs,
                 size_t rec_bytes, int32_t* __restrict__ ids, float* __restrict__ logp,
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
-                unsigned char* partials) {
+                unsigned char* partials, PartialOut pout) {
   pdl_wait();
   constexpr int VEC = Vec<T>::N;
   __shared__ uint64_t s_buf[TK_WARPS][TK_CAP];   // the warps' candidates
@@ -479,18 +515,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   }
 
   if (splits == 1) {
-    if (warp == 0) {
-      const float l = cm + logf(cs);
-      if (lane == 0) {
-        lse[row] = l;
-        if (!isfinite(l)) set_status(status, LILICORR_ERR_NONFINITE);
-      }
-      if (lane < K) {
-        const uint64_t k = s_top[lane];
-        ids[(size_t)row * K + lane] = key_id(k);
-        logp[(size_t)row * K + lane] = key_value(k) - l;
-      }
-    }
+    if (warp == 0) write_row(row, K, cm, cs, s_top, pout, ids, logp, lse, status, lane);
     return;
   }
 
@@ -529,17 +554,47 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
     }
     const float gm = warp_max(pm);
     const float gs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - gm) * LOG2E));
-    const float l = gm + logf(gs);
-    if (lane == 0) {
-      lse[row] = l;
-      if (!isfinite(l)) set_status(status, LILICORR_ERR_NONFINITE);
-      counters[row] = 0u;             // leave the workspace reusable
+    if (lane == 0) counters[row] = 0u;             // leave the workspace reusable
+    write_row(row, K, gm, gs, s_top, pout, ids, logp, lse, status, lane);
+  }
+}
+
+// Merge of P vocabulary shards' partial records of one row (one CTA per row): the union
+// of the shards' top-K lists holds the row's top-K, and (m, s) pairs combine as in the
+// split merge above.
+__global__ void __launch_bounds__(TK_THREADS)
+topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K,
+                  int32_t* __restrict__ ids, float* __restrict__ logp, float* __restrict__ lse,
+                  uint32_t* status) {
+  pdl_wait();
+  __shared__ uint64_t s_keys[TK_MERGE_MAX];
+  __shared__ uint64_t s_merge[TK_MERGE_MAX];
+  __shared__ uint64_t s_top[LILICORR_MAX_K];
+  __shared__ int s_count;
+  __shared__ uint64_t s_bound;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, row = blockIdx.x;
+  const size_t rb = topk_partial_bytes(K);
+  for (int i = tid; i < P * K; i += TK_THREADS) {
+    const unsigned char* r = recs + ((size_t)(i / K) * rows + row) * rb;
+    const float v = reinterpret_cast<const float*>(r)[2 + i % K];
+    const int32_t id = reinterpret_cast<const int32_t*>(r + 8 + 4 * (size_t)K)[i % K];
+    s_keys[i] = id < 0 ? 0ull : make_key(v, (uint32_t)id);
+  }
+  __syncthreads();
+  cta_select(s_keys, P, K, K, s_merge, &s_count, &s_bound, s_top);
+  if (warp == 0) {
+    float pm = -INFINITY, ps = 0.f;
+    for (int p = lane; p < P; p += 32) {
+      const float* r = reinterpret_cast<const float*>(recs + ((size_t)p * rows + row) * rb);
+      const float rm = r[0], rs = r[1];
+      if (rm == -INFINITY) continue;
+      if (rm > pm) { ps = ps * ex2((pm - rm) * LOG2E) + rs; pm = rm; }
+      else ps += rs * ex2((rm - pm) * LOG2E);
     }
-    if (lane < K) {
-      const uint64_t k = s_top[lane];
-      ids[(size_t)row * K + lane] = key_id(k);
-      logp[(size_t)row * K + lane] = key_value(k) - l;
-    }
+    const float gm = warp_max(pm);
+    const float gs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - gm) * LOG2E));
+    const PartialOut none{nullptr, 0};
+    write_row(row, K, gm, gs, s_top, none, ids, logp, lse, status, lane);
   }
 }
 
@@ -570,18 +625,29 @@ size_t topk_ws_bytes(int rows, int V, int K, lilicorr_dtype_t dt) {
 
 lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int rows, int V, int K,
                                   int32_t* ids, float* logp, float* lse, uint32_t* status,
-                                  uint32_t* counters, void* partials, cudaStream_t st) {
+                                  uint32_t* counters, void* partials, cudaStream_t st,
+                                  void* partial_out, int32_t id_offset) {
+  const PartialOut pout{static_cast<unsigned char*>(partial_out), id_offset};
   if (rows == 0) return LILICORR_OK;
   const TopkPlan p = topk_plan(rows, V, K, dt);
   dim3 grid(p.splits, rows);
   if (dt == LILICORR_BF16)
     LL_TRY(launch_k(topk_lse_kernel<uint16_t>, grid, TK_THREADS, 0, st, 
         static_cast<const uint16_t*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials)));
+        lse, status, counters, static_cast<unsigned char*>(partials), pout));
   else
     LL_TRY(launch_k(topk_lse_kernel<float>, grid, TK_THREADS, 0, st, 
         static_cast<const float*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials)));
+        lse, status, counters, static_cast<unsigned char*>(partials), pout));
+  return LILICORR_OK;
+}
+
+lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K, int32_t* ids,
+                                    float* logp, float* lse, uint32_t* status, cudaStream_t st) {
+  if (rows == 0) return LILICORR_OK;
+  if (P < 1 || P * K > TK_MERGE_MAX) return LILICORR_ERR_SHAPE;
+  LL_TRY(launch_k(topk_merge_kernel, rows, TK_THREADS, 0, st,
+                  static_cast<const unsigned char*>(partials), P, rows, K, ids, logp, lse, status));
   return LILICORR_OK;
 }
 
