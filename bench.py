@@ -513,6 +513,39 @@ def run_ours(args, world, rank, local):
                        % (P, P)}
     del sl, sws, recs
 
+    # ---- the LM-head projection fused with the top-K pass (logits never written): this
+    # workload's drafter hidden states against a random bf16 vocabulary projection of the
+    # workload's shape, next to the unfused pair (cuBLAS bf16 product writing the logits,
+    # then the top-K pass)
+    lm_head = None
+    if wl.dtype == "bf16":
+        gW = torch.Generator(device=dev).manual_seed(1_000_033)
+        Wv = (0.02 * torch.randn((wl.V, wl.H), generator=gW, device=dev)).to(torch.bfloat16)
+        hrows = hidden[0].reshape(rows, wl.H)
+        lws = ll.Workspace(ll.lib().lilicorr_lm_head_topk_workspace_bytes(rows, wl.H, wl.V, wl.K))
+        fused_us = timed(lambda: ll.lm_head_topk(hrows, Wv, wl.K, ws=lws), n=5)
+        if ws.status() != 0 or lws.status() != 0:
+            raise RuntimeError("device status set by the fused LM head")
+        logits_tmp = torch.empty((rows, wl.V), dtype=torch.bfloat16, device=dev)
+
+        def unfused():
+            torch.matmul(hrows, Wv.t(), out=logits_tmp)
+            ll.topk_lse(logits_tmp, wl.K, ws=tk_ws)
+        unfused_us = timed(unfused, n=5)
+        flops = 2.0 * rows * wl.H * wl.V
+        w_bytes = wl.V * wl.H * 2
+        bf16_peak = float(pk.get("bf16_tflops", 1900.0))
+        lm_head = {"rows": rows, "H": wl.H, "V": wl.V, "us_per_call": round(fused_us, 2),
+                   "tflops": round(flops / (fused_us * 1e-6) / 1e12, 1),
+                   "tensor_frac": round(flops / (fused_us * 1e-6) / 1e12 / bf16_peak, 4),
+                   "weight_gbs": round(w_bytes / (fused_us * 1e-6) / 1e9, 1),
+                   "hbm_frac": round(w_bytes / (fused_us * 1e-6) / 1e9 / hbm, 4),
+                   "unfused_us_per_call": round(unfused_us, 2),
+                   "note": "hidden[rows, H] @ W_vocab[V, H]^T reduced to top-K + lse in one "
+                           "tcgen05 pass; unfused = cuBLAS bf16 GEMM writing the logits, then "
+                           "topk_lse; fractions of the measured bf16 and copy peaks"}
+        del Wv, logits_tmp, lws
+
     l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
     in_bytes = logits.numel() * es
     if in_bytes > l2_bytes:
@@ -544,6 +577,7 @@ def run_ours(args, world, rank, local):
                          "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
                          "sample": f"{nv} calls of this workload, best of 3"},
         "vocab_sharded": sharded,
+        "lm_head_fused": lm_head,
         "roofline": roofline,
     }
     if rank == 0 and not args.no_cpu_baseline:

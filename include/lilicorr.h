@@ -161,7 +161,7 @@ lilicorr_status_t lilicorr_topk_lse(const void* logits, lilicorr_dtype_t dtype, 
  *   lilicorr_topk_lse_partial_workspace_bytes(rows, V, K) bytes. A shard row may be all
  *   -inf; non-finite results are reported by the merge.
  * lilicorr_topk_lse_merge: partials [P][rows] records (the shards' outputs in any order;
- *   the ids carry the offsets), 1 <= P and P*K <= 512; ids/logp/lse as lilicorr_topk_lse;
+ *   the ids carry the offsets), 1 <= P and P*K <= 8192; ids/logp/lse as lilicorr_topk_lse;
  *   status: a device uint32 word (may be NULL) that receives LILICORR_ERR_NONFINITE for a
  *   row whose merged normaliser is not finite. */
 size_t lilicorr_topk_partial_bytes(int K);
@@ -172,6 +172,25 @@ lilicorr_status_t lilicorr_topk_lse_partial(const void* logits, lilicorr_dtype_t
 lilicorr_status_t lilicorr_topk_lse_merge(const void* partials, int P, int rows, int K,
                                           int32_t* ids, float* logp, float* lse, uint32_t* status,
                                           cudaStream_t stream);
+
+/* Step (1) with the LM-head projection in front of it, fused: the logits
+ * logits[r, v] = sum_h hidden[r, h] * w_vocab[v, h] (fp32 accumulation of bf16 products)
+ * are formed tile by tile on the tensor cores and reduced in place to what
+ * lilicorr_topk_lse returns for them (top-K ids by descending logit, ties to the lower id;
+ * logp = logit - lse; lse = log sum_v exp(logit)), so the [rows, V] logits never reach
+ * memory (the projection that produces the drafter's logits, Table "cost"; Sec. 3.2).
+ *   hidden    [rows, H] bf16, the final hidden states of the rows (row-major)
+ *   w_vocab   [V, H] bf16, the LM-head weight (row v produces logit v)
+ *   ids, logp [rows, K]; lse [rows]
+ *   ws        zero-filled workspace of at least lilicorr_lm_head_topk_workspace_bytes(rows,
+ *             H, V, K) bytes (0: unsupported shape); its first word is the device status
+ * H a multiple of 64, 1 <= K <= min(V, LILICORR_MAX_K); hidden, w_vocab and ws 16-byte
+ * aligned. A non-finite normaliser (NaN or inf in the inputs) sets LILICORR_ERR_NONFINITE
+ * in the device status. */
+size_t lilicorr_lm_head_topk_workspace_bytes(int rows, int H, int V, int K);
+lilicorr_status_t lilicorr_lm_head_topk(const void* hidden, const void* w_vocab, int rows, int H,
+                                        int V, int K, int32_t* ids, float* logp, float* lse,
+                                        void* ws, size_t ws_bytes, cudaStream_t stream);
 
 /* Step (1) without a caller workspace. Not from the paper (it has no counterpart
  * there): an addition for callers that cannot allocate device memory at the point

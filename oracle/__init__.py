@@ -151,6 +151,16 @@ def merge_partials(parts, K: int) -> Tuple[np.ndarray, np.ndarray, float]:
     return ids[order].astype(np.int64), vals[order] - lse, lse
 
 
+def lm_head_topk(hidden: np.ndarray, w_vocab: np.ndarray, K: int):
+    """The LM-head projection followed by step (1) (the projection that produces the
+    drafter's logits, Table "cost"): logits = w_vocab @ hidden in fp64 (a library matmul),
+    then topk_lse of those logits. hidden [H], w_vocab [V, H]. Returns topk_lse's
+    (ids, logp, lse) and the logits."""
+    x = np.asarray(w_vocab, dtype=np.float64) @ np.asarray(hidden, dtype=np.float64)
+    ids, logp, lse = topk_lse(x, K)
+    return ids, logp, lse, x
+
+
 # =========================================================================== step a2
 def confidence_features(logp: np.ndarray) -> np.ndarray:
     """Five confidence scalars per candidate of one slot (App. A "Architecture"):

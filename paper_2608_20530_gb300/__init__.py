@@ -71,6 +71,8 @@ _SIGS = {
     "lilicorr_test_fused_path": (_I, [_P, _I]),
     "lilicorr_topk_lse_noalloc_max_bytes": (_S, []),
     "lilicorr_topk_partial_bytes": (_S, [_I]),
+    "lilicorr_lm_head_topk_workspace_bytes": (_S, [_I, _I, _I, _I]),
+    "lilicorr_lm_head_topk": (_I, [_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _S, _P]),
     "lilicorr_topk_lse_partial_workspace_bytes": (_S, [_I, _I, _I]),
     "lilicorr_topk_lse_partial": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _S, _P]),
     "lilicorr_topk_lse_merge": (_I, [_P, _I, _I, _I, _P, _P, _P, _P, _P]),
@@ -268,6 +270,31 @@ def topk_lse_noalloc(logits: torch.Tensor, K: int):
     _check(lib().lilicorr_topk_lse_noalloc(logits.data_ptr(), _dtype_code(logits), rows, V, K,
                                            ids.data_ptr(), logp.data_ptr(), lse.data_ptr(),
                                            _stream()), "topk_lse_noalloc")
+    return ids, logp, lse
+
+
+def lm_head_topk(hidden: torch.Tensor, w_vocab: torch.Tensor, K: int,
+                 ws: Optional[Workspace] = None):
+    """Top-K ids [rows, K] int32, log-probs [rows, K] and log-normaliser [rows] of the
+    logits hidden [rows, H] @ w_vocab[V, H]^T (bf16), which are never written out."""
+    _dev(hidden, "hidden")
+    _dev(w_vocab, "w_vocab")
+    if hidden.dtype != torch.bfloat16 or w_vocab.dtype != torch.bfloat16:
+        raise ValueError("hidden and w_vocab must be bf16")
+    rows, H = hidden.shape
+    V = w_vocab.shape[0]
+    need = int(lib().lilicorr_lm_head_topk_workspace_bytes(rows, H, V, K))
+    if need == 0 and rows > 0:
+        raise LilicorrError(ERR_SHAPE, "lm_head_topk")
+    if ws is None:
+        ws = Workspace(need, hidden.device)
+    dev = hidden.device
+    ids = torch.empty((rows, K), dtype=torch.int32, device=dev)
+    logp = torch.empty((rows, K), dtype=torch.float32, device=dev)
+    lse = torch.empty((rows,), dtype=torch.float32, device=dev)
+    _check(lib().lilicorr_lm_head_topk(hidden.data_ptr(), w_vocab.data_ptr(), rows, H, V, K,
+                                       ids.data_ptr(), logp.data_ptr(), lse.data_ptr(), ws.ptr,
+                                       ws.nbytes, _stream()), "lm_head_topk")
     return ids, logp, lse
 
 

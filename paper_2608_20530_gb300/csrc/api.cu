@@ -609,11 +609,32 @@ lilicorr_status_t lilicorr_topk_lse_partial(const void* logits, lilicorr_dtype_t
 lilicorr_status_t lilicorr_topk_lse_merge(const void* partials, int P, int rows, int K,
                                           int32_t* ids, float* logp, float* lse, uint32_t* status,
                                           cudaStream_t stream) {
-  if (rows < 0 || P < 1 || K <= 0 || K > LILICORR_MAX_K || P * K > 512) return LILICORR_ERR_SHAPE;
+  if (rows < 0 || P < 1 || K <= 0 || K > LILICORR_MAX_K || P * K > TOPK_MERGE_KEYS_MAX)
+    return LILICORR_ERR_SHAPE;
   if (rows == 0) return LILICORR_OK;
   if (!partials || !ids || !logp || !lse) return LILICORR_ERR_ARG;
   if (reinterpret_cast<uintptr_t>(partials) & 7) return LILICORR_ERR_ARG;
   return launch_topk_merge(partials, P, rows, K, ids, logp, lse, status, stream);
+}
+
+size_t lilicorr_lm_head_topk_workspace_bytes(int rows, int H, int V, int K) {
+  if (!lm_head_supported(rows, H, V, K)) return 0;
+  return 256 + align_up(lm_head_records_bytes(rows, V, K), 256);
+}
+
+lilicorr_status_t lilicorr_lm_head_topk(const void* hidden, const void* w_vocab, int rows, int H,
+                                        int V, int K, int32_t* ids, float* logp, float* lse,
+                                        void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (rows < 0 || H <= 0 || V <= 0 || K <= 0 || K > LILICORR_MAX_K || K > V)
+    return LILICORR_ERR_SHAPE;
+  if (rows == 0) return LILICORR_OK;
+  if (!lm_head_supported(rows, H, V, K)) return LILICORR_ERR_SHAPE;
+  if (!hidden || !w_vocab || !ids || !logp || !lse || !ws) return LILICORR_ERR_ARG;
+  if (!aligned16(hidden) || !aligned16(w_vocab) || !aligned16(ws)) return LILICORR_ERR_ARG;
+  if (ws_bytes < lilicorr_lm_head_topk_workspace_bytes(rows, H, V, K)) return LILICORR_ERR_WORKSPACE;
+  unsigned char* w = static_cast<unsigned char*>(ws);
+  return launch_lm_head_topk(hidden, w_vocab, rows, H, V, K, w + 256, ids, logp, lse,
+                             reinterpret_cast<uint32_t*>(w), stream);
 }
 
 size_t lilicorr_workspace_bytes(const lilicorr_head* head, int B) {

@@ -209,6 +209,30 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
                                   void* partial_out = nullptr, int32_t id_offset = 0);
 // bytes of one row's partial record: max, sum, K values, K ids
 __host__ __device__ constexpr size_t topk_partial_bytes(int K) { return 8 + 8 * (size_t)K; }
+// the merge holds P*K keys (and as many survivors) in shared memory
+constexpr int TOPK_MERGE_KEYS_MAX = 8192;
+
+// Order-preserving 64-bit candidate key: larger value first, equal values by lower id;
+// -0.0 == +0.0. Key 0 never occurs for a real element and marks an empty slot.
+__device__ __forceinline__ uint64_t make_key(float v, uint32_t id) {
+  uint32_t b = __float_as_uint(v);
+  if ((b << 1) == 0u) b = 0u;
+  const uint32_t o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+  return ((uint64_t)o << 32) | (uint64_t)(0xFFFFFFFFu - id);
+}
+__device__ __forceinline__ float key_value(uint64_t k) {
+  const uint32_t o = (uint32_t)(k >> 32);
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+__device__ __forceinline__ int32_t key_id(uint64_t k) {
+  return (int32_t)(0xFFFFFFFFu - (uint32_t)k);
+}
+// LM-head projection fused with step (1) (lm_head.cu): records [P][rows] in ws, then merged
+bool lm_head_supported(int rows, int H, int V, int K);
+size_t lm_head_records_bytes(int rows, int V, int K);
+lilicorr_status_t launch_lm_head_topk(const void* hidden, const void* w_vocab, int rows, int H,
+                                      int V, int K, void* recs, int32_t* ids, float* logp,
+                                      float* lse, uint32_t* status, cudaStream_t st);
 // merge P shards' records [P][rows][topk_partial_bytes(K)] into the final outputs
 lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K, int32_t* ids,
                                     float* logp, float* lse, uint32_t* status, cudaStream_t st);

@@ -40,20 +40,6 @@ constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr unsigned FULL = 0xffffffffu;
 
-// Order-preserving key: larger value first, equal values by lower id; -0.0 == +0.0.
-__device__ __forceinline__ uint64_t make_key(float v, uint32_t id) {
-  uint32_t b = __float_as_uint(v);
-  if ((b << 1) == 0u) b = 0u;
-  const uint32_t o = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-  return ((uint64_t)o << 32) | (uint64_t)(0xFFFFFFFFu - id);
-}
-__device__ __forceinline__ float key_value(uint64_t k) {
-  const uint32_t o = (uint32_t)(k >> 32);
-  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
-}
-__device__ __forceinline__ int32_t key_id(uint64_t k) {
-  return (int32_t)(0xFFFFFFFFu - (uint32_t)k);
-}
 // order-preserving 32-bit image of a float (for atomicMax on a threshold)
 __device__ __forceinline__ uint32_t ord32(float v) {
   const uint32_t b = __float_as_uint(v);
@@ -567,8 +553,9 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
                   int32_t* __restrict__ ids, float* __restrict__ logp, float* __restrict__ lse,
                   uint32_t* status) {
   pdl_wait();
-  __shared__ uint64_t s_keys[TK_MERGE_MAX];
-  __shared__ uint64_t s_merge[TK_MERGE_MAX];
+  extern __shared__ uint64_t s_dyn[];            // [P*K] keys, then [P*K] survivors
+  uint64_t* s_keys = s_dyn;
+  uint64_t* s_merge = s_dyn + (size_t)P * K;
   __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ int s_count;
   __shared__ uint64_t s_bound;
@@ -645,8 +632,10 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
 lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K, int32_t* ids,
                                     float* logp, float* lse, uint32_t* status, cudaStream_t st) {
   if (rows == 0) return LILICORR_OK;
-  if (P < 1 || P * K > TK_MERGE_MAX) return LILICORR_ERR_SHAPE;
-  LL_TRY(launch_k(topk_merge_kernel, rows, TK_THREADS, 0, st,
+  if (P < 1 || K < 1 || P * K > TOPK_MERGE_KEYS_MAX) return LILICORR_ERR_SHAPE;
+  static bool configured[64] = {false};
+  LL_TRY(allow_max_dynamic_smem(topk_merge_kernel, configured));
+  LL_TRY(launch_k(topk_merge_kernel, rows, TK_THREADS, 2 * (size_t)P * K * sizeof(uint64_t), st,
                   static_cast<const unsigned char*>(partials), P, rows, K, ids, logp, lse, status));
   return LILICORR_OK;
 }

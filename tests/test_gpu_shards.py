@@ -38,7 +38,8 @@ def _sharded(ll, xd, K, P):
 @pytest.mark.parametrize("rows,V,K,P,dtype,quant", [
     (16, 151936, 8, 2, "bf16", None), (16, 151936, 8, 8, "bf16", None),
     (8, 151936, 16, 3, "bf16", 0.25), (4, 32000, 4, 5, "f32", None),
-    (33, 4099, 32, 7, "bf16", 0.5), (3, 300, 8, 64, "f32", None)])
+    (33, 4099, 32, 7, "bf16", 0.5), (3, 300, 8, 64, "f32", None),
+    (5, 151936, 8, 152, "bf16", None)])
 def test_merged_shards_match_the_whole_row(rows, V, K, P, dtype, quant):
     ll = _ll()
     x = _logits(rows, V, rows * 7 + P, quant)
@@ -95,6 +96,6 @@ def test_merge_flags_a_nan_row_and_rejects_too_many_shards():
     ll.topk_lse_merge(torch.stack(recs), 8, status=status)
     torch.cuda.synchronize()
     assert int(status.item()) == ll.ERR_NONFINITE
-    many = torch.zeros((65, 3, ll.topk_partial_bytes(8)), dtype=torch.uint8, device="cuda")
+    many = torch.zeros((257, 3, ll.topk_partial_bytes(32)), dtype=torch.uint8, device="cuda")
     with pytest.raises(ll.LilicorrError):
-        ll.topk_lse_merge(many, 8)                     # 65 x 8 keys exceed the merge area
+        ll.topk_lse_merge(many, 32)                    # 257 x 32 keys exceed the merge area
