@@ -83,7 +83,8 @@ constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [4][128] f
 constexpr uint32_t OFF_DIST = OFF_SS + NF_CG * NF_M * 4;           // [8][127] float
 constexpr uint32_t OFF_SAME = OFF_DIST + NF_NH * (2 * NF_MAX_L - 1) * 4;
 constexpr uint32_t OFF_SLOT = OFF_SAME + NF_NH * 4;                // [128] slot of each node
-constexpr uint32_t OFF_BAR = (OFF_SLOT + NF_M + 63) & ~63u;
+constexpr uint32_t OFF_IDS = OFF_SLOT + NF_M;                      // [128] token id of each node
+constexpr uint32_t OFF_BAR = (OFF_IDS + NF_M * 4 + 63) & ~63u;
 constexpr int N_EV = 52;                                           // per direction
 constexpr uint32_t NF_SMEM_USED = OFF_BAR + (2 * NF_STAGES + 2 * N_EV) * 8;
 constexpr size_t NF_SMEM = 1024 + NF_SMEM_USED;
@@ -326,11 +327,15 @@ __device__ __forceinline__ uint32_t ex2_h2(uint32_t x) {
 __device__ __forceinline__ float2 h2_to_f2(uint32_t x) {
   return __half22float2(*reinterpret_cast<const __half2*>(&x));
 }
-// SiLU(z) = z sigmoid(z) = z (1 + tanh(z / 2)) / 2, one MUFU operation
-__device__ __forceinline__ float silu_fast(float z) {
-  float t;
-  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * z));
-  return 0.5f * z * (1.0f + t);
+// SiLU(z) = z sigmoid(z) = z (1 + tanh(z / 2)) / 2 for two values with one packed fp16
+// tanh (one MUFU operation per pair; the result feeds a bf16 operand, whose rounding is
+// coarser than the fp16 tanh)
+__device__ __forceinline__ void silu2(float& z0, float& z1) {
+  uint32_t t;
+  asm("tanh.approx.f16x2 %0, %1;" : "=r"(t) : "r"(pack_h2(0.5f * z0, 0.5f * z1)));
+  const float2 tf = h2_to_f2(t);
+  z0 = 0.5f * z0 * (1.0f + tf.x);
+  z1 = 0.5f * z1 * (1.0f + tf.y);
 }
 __device__ __forceinline__ void rw_bar() { named_bar(1, NF_RW); }
 __device__ __forceinline__ void set_bar(int set) { named_bar(2 + set, NF_RW / 2); }
@@ -449,7 +454,11 @@ __device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, int c
     float v[32];
     ld32f(tscr + c0, v);
 #pragma unroll
-    for (int e = 0; e < 32; ++e) v[e] = silu_fast(v[e] + bias[c0 + e]);
+    for (int e = 0; e < 32; e += 2) {
+      v[e] += bias[c0 + e];
+      v[e + 1] += bias[c0 + e + 1];
+      silu2(v[e], v[e + 1]);
+    }
     put32(buf, r, c0, v);
   }
 }
@@ -473,6 +482,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
   float* s_dist = reinterpret_cast<float*>(sm + OFF_DIST);
   float* s_same = reinterpret_cast<float*>(sm + OFF_SAME);
   uint8_t* s_slot = sm + OFF_SLOT;
+  int32_t* s_ids = reinterpret_cast<int32_t*>(sm + OFF_IDS);
   float* vec = reinterpret_cast<float*>(sm + OFF_VEC);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -550,6 +560,14 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         if (ok) {
           const int s = r / K, k = r % K;
           const size_t rk = ((size_t)b * L + s) * K;
+          if (cg == 0) {                            // the node's token, read once per row
+            int id = a.ids[rk + k];
+            if (id < 0 || id >= a.V) {              // an id outside the vocabulary: flag, read row 0
+              set_status(a.status, LILICORR_ERR_ARG);
+              id = 0;
+            }
+            s_ids[r] = id;
+          }
           const float lp = a.logp[rk + k], lp0 = a.logp[rk];
           f[0] = lp;
           f[1] = expf(lp);
@@ -561,25 +579,26 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         // the slot and rank tables (into ACT, which c1 fills afterwards) and the folded
         // embedding rows of 64 nodes at a time (into HF, 16-byte pieces XOR-swizzled by row);
         // the threads owning a row then sum it from shared memory into tensor memory.
-        float* tab = reinterpret_cast<float*>(sm + OFF_ACT);     // rows: hproj+slot+b_c2 [L], rank [K]
+        // rows: hproj+slot+b_c2 [L], rank [K]; the 16-byte pieces of row i XOR-swizzled by
+        // i & 7, so rows read side by side (a warp's slots, its ranks) hit distinct banks
+        float* tab = reinterpret_cast<float*>(sm + OFF_ACT);
+        auto tab_at = [&](int row, int c) {         // c: a multiple of 4
+          return tab + (size_t)row * NF_D + (((c >> 2) ^ (row & 7)) << 2);
+        };
         uint8_t* stg = sm + OFF_HF;
         for (int i = tid; i < (2 * L + K) * (NF_D / 4); i += NF_RW) {
           const int row = i / (NF_D / 4), c = (i % (NF_D / 4)) * 4;
           const float* src = row < L ? a.hproj + ((size_t)b * L + row) * NF_D + c
                            : row < 2 * L ? a.slot + (size_t)(row - L) * NF_D + c
                                          : a.rank + (size_t)(row - 2 * L) * NF_D + c;
-          cp_async16(tab + (size_t)row * NF_D + c, src);
+          cp_async16(tab_at(row, c), src);
         }
+        rw_bar();                                   // s_ids complete
         auto fetch_fold = [&](int p) {
           for (int nloc = wr; nloc < 64; nloc += NF_RW / 32) {
             const int n = 64 * p + nloc;
             if (n >= LK) break;
-            int id = a.ids[((size_t)b * L + n / K) * K + n % K];
-            if (id < 0 || id >= a.V) {              // an id outside the vocabulary: flag, read row 0
-              if (lane == 0) set_status(a.status, LILICORR_ERR_ARG);
-              id = 0;
-            }
-            const float* src = a.fold + (size_t)id * NF_D + 8 * lane;
+            const float* src = a.fold + (size_t)s_ids[n] * NF_D + 8 * lane;
             uint8_t* row = stg + nloc * 1024;
             cp_async16(row + (((2 * lane) ^ (nloc & 7)) << 4), src);
             cp_async16(row + (((2 * lane + 1) ^ (nloc & 7)) << 4), src + 4);
@@ -590,11 +609,11 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
         rw_bar();
         for (int i = tid; i < L * (NF_D / 4); i += NF_RW) {   // S[s] = hproj + slot + b_c2
           const int row = i / (NF_D / 4), c = (i % (NF_D / 4)) * 4;
-          float4 x = *reinterpret_cast<float4*>(tab + (size_t)row * NF_D + c);
-          const float4 y = *reinterpret_cast<const float4*>(tab + (size_t)(L + row) * NF_D + c);
+          float4 x = *reinterpret_cast<float4*>(tab_at(row, c));
+          const float4 y = *reinterpret_cast<const float4*>(tab_at(L + row, c));
           const float4 z = *reinterpret_cast<const float4*>(vec + V_C2B + c);
           x.x += y.x + z.x; x.y += y.y + z.y; x.z += y.z + z.z; x.w += y.w + z.w;
-          *reinterpret_cast<float4*>(tab + (size_t)row * NF_D + c) = x;
+          *reinterpret_cast<float4*>(tab_at(row, c)) = x;
         }
         rw_bar();
 #pragma unroll 1
@@ -602,8 +621,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
           if ((q >> 1) == p) {                      // rows 64p .. 64p+63 belong to quarters 2p, 2p+1
             const int nr = r - 64 * p;
             const uint8_t* row = stg + nr * 1024;
-            const float* S = tab + (size_t)(ok ? r / K : 0) * NF_D;
-            const float* R = tab + (size_t)(2 * L + (ok ? r % K : 0)) * NF_D;
+            const int srow = ok ? r / K : 0, rrow = 2 * L + (ok ? r % K : 0);
 #pragma unroll 1
             for (int j = 0; j < 2; ++j) {
               const int c0 = NF_CW * cg + 32 * j;
@@ -612,8 +630,8 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
               for (int u = 0; u < 8; ++u) {
                 const float4 x =
                     *reinterpret_cast<const float4*>(row + ((((c0 >> 2) + u) ^ (nr & 7)) << 4));
-                const float4 y = *reinterpret_cast<const float4*>(S + c0 + 4 * u);
-                const float4 z = *reinterpret_cast<const float4*>(R + c0 + 4 * u);
+                const float4 y = *reinterpret_cast<const float4*>(tab_at(srow, c0 + 4 * u));
+                const float4 z = *reinterpret_cast<const float4*>(tab_at(rrow, c0 + 4 * u));
                 v[4 * u] = ok ? x.x + y.x + z.x : 0.f;
                 v[4 * u + 1] = ok ? x.y + y.y + z.y : 0.f;
                 v[4 * u + 2] = ok ? x.z + y.z + z.z : 0.f;
@@ -645,10 +663,12 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
               z.z = fmaf(w.z, f[i], z.z);
               z.w = fmaf(w.w, f[i], z.w);
             }
-            c1[e] = ok ? silu_fast(z.x) : 0.f;
-            c1[e + 1] = ok ? silu_fast(z.y) : 0.f;
-            c1[e + 2] = ok ? silu_fast(z.z) : 0.f;
-            c1[e + 3] = ok ? silu_fast(z.w) : 0.f;
+            silu2(z.x, z.y);
+            silu2(z.z, z.w);
+            c1[e] = ok ? z.x : 0.f;
+            c1[e + 1] = ok ? z.y : 0.f;
+            c1[e + 2] = ok ? z.z : 0.f;
+            c1[e + 3] = ok ? z.w : 0.f;
           }
           put32(sm + OFF_ACT, r, c0, c1);
         }
@@ -709,6 +729,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
           const float same_l2 = s_same[hh];
           const float* sd = s_dist + hh * nd + (L - 1);
           const int q0 = 16 * wi;
+          const bool k8 = (K & 7) == 0;
           uint32_t qa[2][4];
 #pragma unroll
           for (int ks = 0; ks < 2; ++ks)
@@ -735,20 +756,38 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
                 mma_bf16_16816(s4[nb + 1], qa[ks], bf[2], bf[3]);
               }
             float bm0 = -INFINITY, bm1 = -INFINITY;
+            if (k8) {
+              // K % 8 == 0: the 8 keys of a tile share one slot, so one bias per query row
 #pragma unroll
-            for (int nb = 0; nb < 4; ++nb) {
-              const int j0 = kb0 + nb * 8 + 2 * t4;
-              const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
+              for (int nb = 0; nb < 4; ++nb) {
+                const int jt = kb0 + nb * 8;
+                const bool in = jt < LK;
+                const int sj = s_slot[in ? jt : 0];
+                const float b0 = sd[sj - si0] + (si0 == sj ? same_l2 : 0.f);
+                const float b1 = sd[sj - si1] + (si1 == sj ? same_l2 : 0.f);
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const int jj = j0 + (e & 1);
-                const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
-                const int si = e < 2 ? si0 : si1;
-                const float v = jj < LK
-                                    ? s4[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
-                                    : -INFINITY;
-                s4[nb][e] = v;
-                if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+                for (int e = 0; e < 4; ++e) {
+                  const float v = in ? fmaf(s4[nb][e], qscale, e < 2 ? b0 : b1) : -INFINITY;
+                  s4[nb][e] = v;
+                  if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+                }
+              }
+            } else {
+#pragma unroll
+              for (int nb = 0; nb < 4; ++nb) {
+                const int j0 = kb0 + nb * 8 + 2 * t4;
+                const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const int jj = j0 + (e & 1);
+                  const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
+                  const int si = e < 2 ? si0 : si1;
+                  const float v = jj < LK
+                                      ? s4[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
+                                      : -INFINITY;
+                  s4[nb][e] = v;
+                  if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+                }
               }
             }
             bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
