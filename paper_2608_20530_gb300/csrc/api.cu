@@ -310,8 +310,14 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   const lilicorr_head_desc& d = c.d;
   const lilicorr_dtype_t F32 = LILICORR_F32, adt = c.adt;
   const int D = c.D, F = c.F, N = c.N;
-  // the fused kernel puts a sequence on one SM: it wins once several sequences share the
-  // GPU; a lone sequence runs faster as the chain of kernels below, each spread over SMs
+  // Network kernels: a cluster of four SMs per sequence while every sequence's cluster
+  // fits on the GPU at once; beyond that one SM per sequence (fewer waves); the chain of
+  // kernels below, each spread over SMs, for heads neither kernel takes.
+  const bool cluster = h->cluster_maps &&
+                       (g_fused_enabled == 3 ||
+                        (g_fused_enabled == 1 && c.B <= net_cluster_capacity()));
+  if (cluster)
+    return launch_net_cluster(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   if (h->net_maps && (g_fused_enabled == 2 || (g_fused_enabled == 1 && c.B >= FUSED_MIN_B)))
     return launch_net_fused(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
@@ -527,6 +533,7 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
   cudaFree(embed_dev);
   embed_dev = nullptr;
   h->net_maps = net_fused_maps_create(h);
+  h->cluster_maps = net_cluster_maps_create(h);
   *out = h;
   return LILICORR_OK;
 }
@@ -538,6 +545,7 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   if (cur != h->device) cudaSetDevice(h->device);
   cudaError_t e = cudaFree(h->pool);
   net_fused_maps_free(h->net_maps);
+  net_cluster_maps_free(h->cluster_maps);
   if (h->side) cudaStreamDestroy(h->side);
   if (h->side2) cudaStreamDestroy(h->side2);
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
@@ -813,8 +821,9 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
 }
 
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode) {
-  g_fused_enabled = mode < 0 ? 0 : mode > 2 ? 2 : mode;
-  return head && head->net_maps ? 1 : 0;
+  g_fused_enabled = mode < 0 ? 0 : mode > 3 ? 3 : mode;
+  if (!head) return 0;
+  return (mode == 3 ? head->cluster_maps : head->net_maps) ? 1 : 0;
 }
 
 uint64_t lilicorr_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }

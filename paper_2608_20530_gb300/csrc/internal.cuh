@@ -176,6 +176,7 @@ struct lilicorr_head {
   const float* boi;           // [2d]
   const void* anc_w; const float* anc_b;
   void* net_maps;             // tensor maps of the fused scoring network, or null
+  void* cluster_maps;         // tensor maps of the cluster scoring network, or null
 };
 
 namespace lilicorr {
@@ -267,7 +268,16 @@ void net_fused_maps_free(void* maps);
 lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t* ids,
                                    const float* logp, const float* hproj, const float* t,
                                    const float* cb, float* oi, uint32_t* status, cudaStream_t st);
-extern int g_fused_enabled;   // 0 never, 1 from FUSED_MIN_B sequences on (default), 2 always
+// the same network on a cluster of four CTAs per sequence (net_cluster.cu)
+bool net_cluster_supported(const lilicorr_head_desc& d);
+void* net_cluster_maps_create(const lilicorr_head* h);
+void net_cluster_maps_free(void* p);
+int net_cluster_capacity();   // clusters that fit on the device at once
+lilicorr_status_t launch_net_cluster(const lilicorr_head* h, int B, const int32_t* ids,
+                                     const float* logp, const float* hproj, const float* t,
+                                     const float* cb, float* oi, uint32_t* status, cudaStream_t st);
+extern int g_fused_enabled;   // 0 never, 1 by batch size (default), 2 the one-CTA kernel
+                              // always, 3 the cluster kernel always
 constexpr int FUSED_MIN_B = 8;
 
 lilicorr_status_t launch_target_norm(const void* T, lilicorr_dtype_t dt, int B, int n_tgt, int H,

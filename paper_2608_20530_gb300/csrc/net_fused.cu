@@ -41,12 +41,13 @@
 // copies and products, runs its remaining barriers through and frees tensor memory.
 #include <new>
 
-#include "tc_ptx.cuh"
+#include "net_common.cuh"
 
 namespace lilicorr {
 
 namespace {
 using namespace tc;
+using namespace net;
 
 constexpr int NF_D = 256;                 // node width
 constexpr int NF_F = 512;                 // FFN width
@@ -277,76 +278,8 @@ struct Issuer {
 __device__ __forceinline__ uint32_t swz(int r, int j) {     // 16-byte piece j of row r
   return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
 }
-// q / k / v of one head: [128 rows][32] 16-bit values, 64-byte rows, pieces XOR-swizzled
-// by row pair so that ldmatrix over 8 consecutive rows touches 8 distinct bank groups
-__device__ __forceinline__ uint32_t qkv_off(int row, int piece) {
-  return (uint32_t)(row * 64 + ((piece ^ ((row >> 1) & 3)) << 4));
-}
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-// warp-level products: S = Q K^T with bf16 operands, O += P V with fp16 operands
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                               uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
-      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void mma_f16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                              uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
-      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ float ex2f(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-// two fp32 -> fp16x2 (round to nearest), and 2^x on both halves in one instruction
-__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
-  const __half2 v = __floats2half2_rn(lo, hi);
-  return *reinterpret_cast<const uint32_t*>(&v);
-}
-__device__ __forceinline__ uint32_t ex2_h2(uint32_t x) {
-  uint32_t y;
-  asm("ex2.approx.f16x2 %0, %1;" : "=r"(y) : "r"(x));
-  return y;
-}
-__device__ __forceinline__ float2 h2_to_f2(uint32_t x) {
-  return __half22float2(*reinterpret_cast<const __half2*>(&x));
-}
-// SiLU(z) = z sigmoid(z) = z (1 + tanh(z / 2)) / 2 for two values with one packed fp16
-// tanh (one MUFU operation per pair; the result feeds a bf16 operand, whose rounding is
-// coarser than the fp16 tanh)
-__device__ __forceinline__ void silu2(float& z0, float& z1) {
-  uint32_t t;
-  asm("tanh.approx.f16x2 %0, %1;" : "=r"(t) : "r"(pack_h2(0.5f * z0, 0.5f * z1)));
-  const float2 tf = h2_to_f2(t);
-  z0 = 0.5f * z0 * (1.0f + tf.x);
-  z1 = 0.5f * z1 * (1.0f + tf.y);
-}
 __device__ __forceinline__ void rw_bar() { named_bar(1, NF_RW); }
 __device__ __forceinline__ void set_bar(int set) { named_bar(2 + set, NF_RW / 2); }
-// 16-byte asynchronous global -> shared copies (L2 only), many in flight per thread
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
-}
-
 // One warp's arrival on a row-worker -> MMA event, after its shared-memory writes
 // (generic proxy, read by the tensor cores through the async proxy) and tensor-memory
 // stores.
@@ -355,46 +288,6 @@ __device__ __forceinline__ void rw_signal(uint64_t* bar, int lane) {
   tc_fence_before();
   __syncwarp();
   if (lane == 0) mbar_arrive(bar);
-}
-
-// 8 bf16 / fp16 of v[0..7] as one 16-byte piece
-__device__ __forceinline__ uint4 pack8(const float* v) {
-  uint4 w;
-  w.x = pack_bf16x2(v[0], v[1]);
-  w.y = pack_bf16x2(v[2], v[3]);
-  w.z = pack_bf16x2(v[4], v[5]);
-  w.w = pack_bf16x2(v[6], v[7]);
-  return w;
-}
-__device__ __forceinline__ uint4 pack8h(const float* v) {
-  uint4 w;
-  w.x = pack_h2(v[0], v[1]);
-  w.y = pack_h2(v[2], v[3]);
-  w.z = pack_h2(v[4], v[5]);
-  w.w = pack_h2(v[6], v[7]);
-  return w;
-}
-
-// Write 32 values (columns c0..c0+31 of row r) as bf16 into a swizzled operand buffer
-// holding 64-column chunks.
-__device__ __forceinline__ void put32(uint8_t* buf, int r, int c0, const float (&v)[32]) {
-  uint8_t* ch = buf + (c0 >> 6) * CHUNK;
-  const int p0 = (c0 & 63) >> 3;
-#pragma unroll
-  for (int p = 0; p < 4; ++p) *reinterpret_cast<uint4*>(ch + swz(r, p0 + p)) = pack8(v + 8 * p);
-}
-
-__device__ __forceinline__ void ld32f(uint32_t taddr, float (&v)[32]) {
-  uint32_t u[32];
-  tmem_ld32(taddr, u);
-#pragma unroll
-  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(u[j]);
-}
-__device__ __forceinline__ void st32f(uint32_t taddr, const float (&v)[32]) {
-  uint32_t u[32];
-#pragma unroll
-  for (int j = 0; j < 32; ++j) u[j] = __float_as_uint(v[j]);
-  tmem_st32(taddr, u);
 }
 
 // RMSNorm statistics of row r over the 256 columns of x (4 threads, 64 columns each):
@@ -723,121 +616,11 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
           set_bar(set);
           // attention core of head hh, queries 16wi .. 16wi+15: blocks of 32 keys with an
           // online softmax in log2 units; P = 2^(S - max) in fp16 pairs (one MUFU op per pair)
-          const uint32_t qb = smem_u32(qs), kb = qb + 8192, vb = qb + 16384;
-          const int g8 = lane >> 2, t4 = lane & 3;
-          const float qscale = rsqrtf((float)NF_HD) * LOG2E;
-          const float same_l2 = s_same[hh];
-          const float* sd = s_dist + hh * nd + (L - 1);
           const int q0 = 16 * wi;
-          const bool k8 = (K & 7) == 0;
-          uint32_t qa[2][4];
-#pragma unroll
-          for (int ks = 0; ks < 2; ++ks)
-            ldsm_x4(qb + qkv_off(q0 + (lane & 15), ks * 2 + (lane >> 4)), qa[ks]);
-          const int i0 = q0 + g8, i1 = i0 + 8;
-          const int si0 = s_slot[i0], si1 = s_slot[i1];
-          float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-          float o[4][4];
-#pragma unroll
-          for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
-#pragma unroll 1
-          for (int kb0 = 0; kb0 < LK; kb0 += 32) {
-            float s4[4][4];
-#pragma unroll
-            for (int nb = 0; nb < 4; ++nb) s4[nb][0] = s4[nb][1] = s4[nb][2] = s4[nb][3] = 0.f;
-#pragma unroll
-            for (int ks = 0; ks < 2; ++ks)
-#pragma unroll
-              for (int nb = 0; nb < 4; nb += 2) {
-                uint32_t bf[4];
-                const int key = kb0 + nb * 8 + (lane & 7) + ((lane >> 4) << 3);
-                ldsm_x4(kb + qkv_off(key, ks * 2 + ((lane >> 3) & 1)), bf);
-                mma_bf16_16816(s4[nb], qa[ks], bf[0], bf[1]);
-                mma_bf16_16816(s4[nb + 1], qa[ks], bf[2], bf[3]);
-              }
-            float bm0 = -INFINITY, bm1 = -INFINITY;
-            if (k8) {
-              // K % 8 == 0: the 8 keys of a tile share one slot, so one bias per query row
-#pragma unroll
-              for (int nb = 0; nb < 4; ++nb) {
-                const int jt = kb0 + nb * 8;
-                const bool in = jt < LK;
-                const int sj = s_slot[in ? jt : 0];
-                const float b0 = sd[sj - si0] + (si0 == sj ? same_l2 : 0.f);
-                const float b1 = sd[sj - si1] + (si1 == sj ? same_l2 : 0.f);
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  const float v = in ? fmaf(s4[nb][e], qscale, e < 2 ? b0 : b1) : -INFINITY;
-                  s4[nb][e] = v;
-                  if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
-                }
-              }
-            } else {
-#pragma unroll
-              for (int nb = 0; nb < 4; ++nb) {
-                const int j0 = kb0 + nb * 8 + 2 * t4;
-                const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  const int jj = j0 + (e & 1);
-                  const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
-                  const int si = e < 2 ? si0 : si1;
-                  const float v = jj < LK
-                                      ? s4[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
-                                      : -INFINITY;
-                  s4[nb][e] = v;
-                  if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
-                }
-              }
-            }
-            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
-            bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
-            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
-            bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
-            const float mn0 = fmaxf(m0, bm0), mn1 = fmaxf(m1, bm1);
-            const float c0 = ex2f(m0 - mn0), c1 = ex2f(m1 - mn1);   // 0 on the first block
-            m0 = mn0;
-            m1 = mn1;
-            l0 *= c0;
-            l1 *= c1;
-#pragma unroll
-            for (int nb = 0; nb < 4; ++nb) {
-              o[nb][0] *= c0; o[nb][1] *= c0;
-              o[nb][2] *= c1; o[nb][3] *= c1;
-            }
-            uint32_t pa[2][4];
-#pragma unroll
-            for (int nb = 0; nb < 4; ++nb) {
-              const uint32_t h01 = ex2_h2(pack_h2(s4[nb][0] - mn0, s4[nb][1] - mn0));
-              const uint32_t h23 = ex2_h2(pack_h2(s4[nb][2] - mn1, s4[nb][3] - mn1));
-              const float2 f01 = h2_to_f2(h01), f23 = h2_to_f2(h23);
-              l0 += f01.x + f01.y;
-              l1 += f23.x + f23.y;
-              const int kk = nb >> 1;
-              if ((nb & 1) == 0) {
-                pa[kk][0] = h01;
-                pa[kk][1] = h23;
-              } else {
-                pa[kk][2] = h01;
-                pa[kk][3] = h23;
-              }
-            }
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk)
-#pragma unroll
-              for (int nb = 0; nb < 4; nb += 2) {
-                uint32_t vf[4];
-                const int key = kb0 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-                ldsm_x4_t(vb + qkv_off(key, nb + (lane >> 4)), vf);
-                mma_f16_16816(o[nb], pa[kk], vf[0], vf[1]);
-                mma_f16_16816(o[nb + 1], pa[kk], vf[2], vf[3]);
-              }
-          }
-          l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-          l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-          l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-          l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-          const float inv0 = 1.0f / l0, inv1 = 1.0f / l1;
+          const int i0 = q0 + (lane >> 2), i1 = i0 + 8, t4 = lane & 3;
+          float o[4][4], inv0, inv1;
+          head_attention(smem_u32(qs), LK, K, s_slot, s_dist + hh * nd + (L - 1), s_same[hh], q0,
+                         lane, o, inv0, inv1);
           // the attention-output buffer is free once the previous pair's W_o product ran
           if (g > 0) ev_wait(&sh.done[D_WO(l, g - 1)], par, sh.abort);
           uint8_t* att = sm + OFF_ATT;
