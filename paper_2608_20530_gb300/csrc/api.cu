@@ -198,7 +198,9 @@ GemmArgs gemm(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, lili
 // Few rows: split-N CUDA-core kernel. bf16 operands: tensor cores. Otherwise the
 // tiled fp32 CUDA-core kernel (the fp32 head keeps fp32 arithmetic throughout).
 lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
-  if (g.M <= 64) return launch_gemm_skinny(g, st);
+  // few rows, or fp32 activations (the tensor-core kernels take bf16) at per-sequence row
+  // counts: the split-N kernel spreads the weights over many CTAs
+  if (g.M <= 64 || (g.a_dt == LILICORR_F32 && g.M <= 1024)) return launch_gemm_skinny(g, st);
   if (gemm_small_supported(g)) return launch_gemm_small(g, st);
   if (gemm_tc_supported(g)) return launch_gemm_tc(g, st);
   return launch_gemm_simt(g, st);

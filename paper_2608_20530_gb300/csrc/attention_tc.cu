@@ -15,8 +15,6 @@ namespace lilicorr {
 
 namespace {
 
-constexpr int AT_WARPS = 4;
-constexpr int AT_QROWS = 16 * AT_WARPS;      // queries per CTA
 constexpr int AT_KBLK = 64;                  // keys per softmax block
 constexpr float LOG2E = 1.4426950408889634f;
 
@@ -51,12 +49,17 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-template <int HD>
-__global__ void __launch_bounds__(AT_WARPS * 32)
+// WARPS warps (16 queries each) share one staging of K and V: 4 when CTAs are scarce,
+// 8 when there are plenty (twice the queries per staged key, and at 64-wide heads the
+// shared memory of two CTAs then fills the register file's 16 warps per SM).
+template <int HD, int WARPS>
+__global__ void __launch_bounds__(WARPS * 32, HD <= 64 ? 16 / WARPS : 1)   // 16 warps per SM
 attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D, int n_heads,
                      const float* __restrict__ dist, const float* __restrict__ same,
                      __nv_bfloat16* __restrict__ out) {
   pdl_wait();
+  constexpr int AT_WARPS = WARPS;
+  constexpr int AT_QROWS = 16 * WARPS;       // queries per CTA
   constexpr int HP = HD + 8;                 // padded row, elements
   constexpr int KS = HD / 16;                // k-steps of Q K^T
   constexpr int NB = HD / 8;                 // 8-wide dim blocks of O
@@ -212,27 +215,37 @@ attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D,
   }
 }
 
+template <int HD, int WARPS>
+lilicorr_status_t launch_hdw(const __nv_bfloat16* qkv, int B, int L, int K, int D, int n_heads,
+                             const float* dist, const float* same, __nv_bfloat16* out,
+                             cudaStream_t st) {
+  static bool configured[64] = {false};
+  LL_TRY(allow_max_dynamic_smem(attention_mma_kernel<HD, WARPS>, configured));
+  const int LK = L * K;
+  const int LKp = (LK + AT_KBLK - 1) / AT_KBLK * AT_KBLK;
+  const size_t smem = sizeof(__nv_bfloat16) * (size_t)(2 * LKp + 16 * WARPS) * (HD + 8) +
+                      sizeof(float) * (2 * L - 1);
+  dim3 grid(B * n_heads, ceil_div(LK, 16 * WARPS));
+  LL_TRY(launch_k(attention_mma_kernel<HD, WARPS>, grid, WARPS * 32, smem, st, qkv, L, K, D,
+                  n_heads, dist, same, out));
+  return LILICORR_OK;
+}
+
 template <int HD>
 lilicorr_status_t launch_hd(const __nv_bfloat16* qkv, int B, int L, int K, int D, int n_heads,
                             const float* dist, const float* same, __nv_bfloat16* out,
                             cudaStream_t st) {
-  static bool configured[64] = {false};
-  LL_TRY(allow_max_dynamic_smem(attention_mma_kernel<HD>, configured));
-  const int LK = L * K;
-  const int LKp = (LK + AT_KBLK - 1) / AT_KBLK * AT_KBLK;
-  const size_t smem = sizeof(__nv_bfloat16) * (size_t)(2 * LKp + AT_QROWS) * (HD + 8) +
-                      sizeof(float) * (2 * L - 1);
-  dim3 grid(B * n_heads, ceil_div(LK, AT_QROWS));
-  LL_TRY(launch_k(attention_mma_kernel<HD>, grid, AT_WARPS * 32, smem, st, qkv, L, K, D, n_heads, dist, same,
-                                                               out));
-  return LILICORR_OK;
+  const long long ctas8 = (long long)B * n_heads * ceil_div(L * K, 128);
+  if (L * K > 64 && ctas8 >= 2LL * num_sms())
+    return launch_hdw<HD, 8>(qkv, B, L, K, D, n_heads, dist, same, out, st);
+  return launch_hdw<HD, 4>(qkv, B, L, K, D, n_heads, dist, same, out, st);
 }
 
 }  // namespace
 
-size_t attention_tc_smem_bytes(int LK, int hd, int L) {
+size_t attention_tc_smem_bytes(int LK, int hd, int L) {     // the larger (8-warp) layout
   const int LKp = (LK + AT_KBLK - 1) / AT_KBLK * AT_KBLK;
-  return sizeof(__nv_bfloat16) * (size_t)(2 * LKp + AT_QROWS) * (hd + 8) + sizeof(float) * (2 * L - 1);
+  return sizeof(__nv_bfloat16) * (size_t)(2 * LKp + 128) * (hd + 8) + sizeof(float) * (2 * L - 1);
 }
 
 bool attention_tc_supported(int hd) { return hd == 16 || hd == 32 || hd == 64 || hd == 128; }
