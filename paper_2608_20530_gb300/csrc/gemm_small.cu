@@ -121,7 +121,11 @@ __global__ void __launch_bounds__(SG_THREADS, 1)
           x.x += br.x; x.y += br.y; x.z += br.z; x.w += br.w;
         }
         if (ep.act == ACT_SILU) {
-          x.x = silu_f(x.x); x.y = silu_f(x.y); x.z = silu_f(x.z); x.w = silu_f(x.w);
+          if (OUT_BF16) {
+            x.x = silu_tanh(x.x); x.y = silu_tanh(x.y); x.z = silu_tanh(x.z); x.w = silu_tanh(x.w);
+          } else {
+            x.x = silu_f(x.x); x.y = silu_f(x.y); x.z = silu_f(x.z); x.w = silu_f(x.w);
+          }
         }
         if (RES) {                                   // fp32 output: 4 columns = 16 bytes
           const int col = c * CH + j;

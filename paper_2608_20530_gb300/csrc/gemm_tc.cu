@@ -9,8 +9,9 @@
 //   * warp 1 allocates two accumulators of BN tensor-memory columns and its lane 0
 //     issues tcgen05.mma (M = 128, N = BN, K = 16), four per stage, releasing stages
 //     with tcgen05.commit and handing finished accumulators to the epilogue;
-//   * warps 2-5 drain an accumulator with tcgen05.ld while the next tile's products
-//     run on the other one. Per chunk of 128 rows x 128 bytes they add bias /
+//   * warps 2-9 drain an accumulator with tcgen05.ld while the next tile's products
+//     run on the other one: two warps per tensor-memory lane quarter, each taking half
+//     of every chunk's columns. Per chunk of 128 rows x 128 bytes they add bias /
 //     per-sequence bias / SiLU / the residual (brought in by a TMA load), write the
 //     chunk into a 128-byte-swizzled staging buffer and store it with one TMA bulk
 //     tensor store (double-buffered staging and residual buffers).
@@ -26,14 +27,26 @@ using namespace tc;
 
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;                  // 64 bf16 = 128 bytes: one swizzle atom row
-constexpr int TC_THREADS = 192;            // producer, MMA, 4 epilogue warps
-constexpr int EPI_THREADS = 128;
+constexpr int TC_THREADS = 320;            // producer, MMA, 8 epilogue warps
+constexpr int EPI_THREADS = 256;
 constexpr uint32_t CHUNK_BYTES = 128 * 128;   // staging chunk: 128 rows x 128 bytes
 constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s at the SM clock
 
-__device__ __forceinline__ void epi_bar() {   // the 4 epilogue warps only
+__device__ __forceinline__ void epi_bar() {   // the 8 epilogue warps only
   asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
 }
+// tcgen05.ld of 16 columns (lane = row of the calling warp's quarter), with the wait
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32"
+      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
 
 struct TcEpilogue {
   const float* bias;
@@ -157,8 +170,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       }
     }
   } else {
-    // ---- epilogue warps 2..5: warp w reads tensor-memory lanes 32*(w%4)..+31
+    // ---- epilogue warps 2..9: warp w reads tensor-memory lanes 32*(w%4)..+31 and takes
+    //      columns HC*half .. HC*half + HC - 1 of every chunk
+    constexpr int HC = CH / 2;
     const int q = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int row = q * 32 + lane;               // row inside the tile
     const bool leader = (warp == 2 && lane == 0);
     uint32_t cc = 0, lt = 0;                     // chunks and tiles handled so far
@@ -191,13 +207,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           if (c + 1 < NCH) issue_res(t, c + 1, cc + 1);
           else if (t + (int)gridDim.x < tiles) issue_res(t + gridDim.x, 0, cc + 1);
         }
-        float v[CH];
+        const int cl = c * CH + half * HC;         // first column of this thread's part
+        float v[HC];
+        {
+          const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + acc * BN + cl;
+          if constexpr (HC == 32) {
+            uint32_t r[32];
+            tmem_ld32(ta, r);
 #pragma unroll
-        for (int h = 0; h < CH / 32; ++h) {
-          uint32_t r[32];
-          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + acc * BN + c * CH + h * 32, r);
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+          } else {
+            uint32_t r[16];
+            tmem_ld16(ta, r);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[h * 32 + j] = __uint_as_float(r[j]);
+            for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+          }
         }
         if (c == NCH - 1) {
           // accumulator drained: hand it back to the MMA warp
@@ -209,20 +233,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             !mbar_wait(&res_full[b], (cc >> 1) & 1u, WAIT_LIMIT_CYCLES))
           abort_flag = 1;
 #pragma unroll
-        for (int j = 0; j < CH; j += 4) {
+        for (int j = 0; j < HC; j += 4) {
           float4 x = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-          const float4 bb = *reinterpret_cast<const float4*>(s_bias + c * CH + j);
+          const float4 bb = *reinterpret_cast<const float4*>(s_bias + cl + j);
           x.x += bb.x; x.y += bb.y; x.z += bb.z; x.w += bb.w;
-          if (brow && n0 + c * CH + j < N) {
-            const float4 br = *reinterpret_cast<const float4*>(brow + n0 + c * CH + j);
+          if (brow && n0 + cl + j < N) {
+            const float4 br = *reinterpret_cast<const float4*>(brow + n0 + cl + j);
             x.x += br.x; x.y += br.y; x.z += br.z; x.w += br.w;
           }
           if (ep.act == ACT_SILU) {
-            x.x = silu_f(x.x); x.y = silu_f(x.y); x.z = silu_f(x.z); x.w = silu_f(x.w);
+            if (OUT_BF16) {
+              x.x = silu_tanh(x.x); x.y = silu_tanh(x.y); x.z = silu_tanh(x.z); x.w = silu_tanh(x.w);
+            } else {
+              x.x = silu_f(x.x); x.y = silu_f(x.y); x.z = silu_f(x.z); x.w = silu_f(x.w);
+            }
           }
           if (ep.has_residual) {            // fp32 output only: 4 columns = 16 bytes
-            const float4 rr =
-                *reinterpret_cast<const float4*>(s_res + b * CHUNK_BYTES + swz(row, j >> 2));
+            const float4 rr = *reinterpret_cast<const float4*>(
+                s_res + b * CHUNK_BYTES + swz(row, (half * HC + j) >> 2));
             x.x += rr.x; x.y += rr.y; x.z += rr.z; x.w += rr.w;
           }
           v[j] = x.x; v[j + 1] = x.y; v[j + 2] = x.z; v[j + 3] = x.w;
@@ -231,18 +259,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         uint8_t* stg = s_out + b * CHUNK_BYTES;
         if (OUT_BF16) {
 #pragma unroll
-          for (int p = 0; p < 8; ++p) {     // 8 pieces of 8 bf16
+          for (int p = 0; p < 4; ++p) {     // 4 pieces of 8 bf16
             uint4 w;
             w.x = pack_bf16x2(v[8 * p + 0], v[8 * p + 1]);
             w.y = pack_bf16x2(v[8 * p + 2], v[8 * p + 3]);
             w.z = pack_bf16x2(v[8 * p + 4], v[8 * p + 5]);
             w.w = pack_bf16x2(v[8 * p + 6], v[8 * p + 7]);
-            *reinterpret_cast<uint4*>(stg + swz(row, p)) = w;
+            *reinterpret_cast<uint4*>(stg + swz(row, 4 * half + p)) = w;
           }
         } else {
 #pragma unroll
-          for (int p = 0; p < 8; ++p)       // 8 pieces of 4 floats
-            *reinterpret_cast<float4*>(stg + swz(row, p)) =
+          for (int p = 0; p < 4; ++p)       // 4 pieces of 4 floats
+            *reinterpret_cast<float4*>(stg + swz(row, 4 * half + p)) =
                 make_float4(v[4 * p], v[4 * p + 1], v[4 * p + 2], v[4 * p + 3]);
         }
         fence_async_shared();

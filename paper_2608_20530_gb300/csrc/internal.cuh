@@ -126,6 +126,13 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 __device__ __forceinline__ float silu_f(float z) { return z / (1.0f + __expf(-z)); }
+// SiLU(z) = z (1 + tanh(z / 2)) / 2 with one MUFU operation, for outputs rounded to bf16
+// (tanh.approx's error is below the bf16 rounding that follows)
+__device__ __forceinline__ float silu_tanh(float z) {
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * z));
+  return 0.5f * z * (1.0f + t);
+}
 
 // Record the first device-detected error in the workspace status word.
 __device__ __forceinline__ void set_status(uint32_t* status, uint32_t code) {
