@@ -70,6 +70,7 @@ attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D,
   __nv_bfloat16* Vs = Ks + (size_t)LKp * HP;
   __nv_bfloat16* Qs = Vs + (size_t)LKp * HP;
   float* s_dist = reinterpret_cast<float*>(Qs + (size_t)AT_QROWS * HP);
+  uint8_t* s_slot = reinterpret_cast<uint8_t*>(s_dist + 2 * L - 1);   // slot of each key
 
   const int b = blockIdx.x / n_heads, h = blockIdx.x % n_heads;
   const int q0 = blockIdx.y * AT_QROWS;
@@ -99,6 +100,9 @@ attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D,
   }
   for (int i = threadIdx.x; i < 2 * L - 1; i += AT_WARPS * 32)
     s_dist[i] = dist[(size_t)h * (2 * L - 1) + i] * LOG2E;
+  const bool k8 = (K & 7) == 0;
+  if (!k8)
+    for (int i = threadIdx.x; i < LK; i += AT_WARPS * 32) s_slot[i] = (uint8_t)(i / K);
   __syncthreads();
 
   const int g = lane >> 2, t = lane & 3;
@@ -137,22 +141,40 @@ attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D,
       }
     // scale, biases (log2 units), mask padded keys; block row maxima
     float bm0 = -INFINITY, bm1 = -INFINITY;
+    if (k8) {
+      // K % 8 == 0: the 8 keys of a tile share one slot, so one bias per query row
 #pragma unroll
-    for (int nb = 0; nb < 8; ++nb)
+      for (int nb = 0; nb < 8; ++nb) {
+        const int jt = kb + nb * 8;
+        const bool in = jt < LK;
+        const int sj = jt / K;
+        const float b0 = s_dist[sj - si0 + L - 1] + (si0 == sj ? same_l2 : 0.f);
+        const float b1 = s_dist[sj - si1 + L - 1] + (si1 == sj ? same_l2 : 0.f);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int j = kb + nb * 8 + 2 * t + (e & 1);
-        const int si = e < 2 ? si0 : si1;
-        float v;
-        if (j < LK) {
-          const int sj = j / K;
-          v = s[nb][e] * qscale + s_dist[sj - si + L - 1] + (si == sj ? same_l2 : 0.f);
-        } else {
-          v = -INFINITY;
+        for (int e = 0; e < 4; ++e) {
+          const float v = in ? fmaf(s[nb][e], qscale, e < 2 ? b0 : b1) : -INFINITY;
+          s[nb][e] = v;
+          if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
         }
-        s[nb][e] = v;
-        if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
       }
+    } else {
+#pragma unroll
+      for (int nb = 0; nb < 8; ++nb)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int j = kb + nb * 8 + 2 * t + (e & 1);
+          const int si = e < 2 ? si0 : si1;
+          float v;
+          if (j < LK) {
+            const int sj = s_slot[j];
+            v = s[nb][e] * qscale + s_dist[sj - si + L - 1] + (si == sj ? same_l2 : 0.f);
+          } else {
+            v = -INFINITY;
+          }
+          s[nb][e] = v;
+          if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+        }
+    }
     bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
     bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
     bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
@@ -224,7 +246,7 @@ lilicorr_status_t launch_hdw(const __nv_bfloat16* qkv, int B, int L, int K, int 
   const int LK = L * K;
   const int LKp = (LK + AT_KBLK - 1) / AT_KBLK * AT_KBLK;
   const size_t smem = sizeof(__nv_bfloat16) * (size_t)(2 * LKp + 16 * WARPS) * (HD + 8) +
-                      sizeof(float) * (2 * L - 1);
+                      sizeof(float) * (2 * L - 1) + LKp;
   dim3 grid(B * n_heads, ceil_div(LK, 16 * WARPS));
   LL_TRY(launch_k(attention_mma_kernel<HD, WARPS>, grid, WARPS * 32, smem, st, qkv, L, K, D,
                   n_heads, dist, same, out));
@@ -245,7 +267,8 @@ lilicorr_status_t launch_hd(const __nv_bfloat16* qkv, int B, int L, int K, int D
 
 size_t attention_tc_smem_bytes(int LK, int hd, int L) {     // the larger (8-warp) layout
   const int LKp = (LK + AT_KBLK - 1) / AT_KBLK * AT_KBLK;
-  return sizeof(__nv_bfloat16) * (size_t)(2 * LKp + 128) * (hd + 8) + sizeof(float) * (2 * L - 1);
+  return sizeof(__nv_bfloat16) * (size_t)(2 * LKp + 128) * (hd + 8) + sizeof(float) * (2 * L - 1) +
+         LKp;
 }
 
 bool attention_tc_supported(int hd) { return hd == 16 || hd == 32 || hd == 64 || hd == 128; }

@@ -144,9 +144,22 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
   float* s_inn = s_in + (size_t)K * d;               // [K]
 
   const float* inb = a.in + (size_t)(b * L + j) * K * a.ld_vec;
-  for (int i = threadIdx.x; i < K * d; i += PW_THREADS) {
-    const int k = i / d, c = i % d;
-    s_in[i] = inb[(size_t)k * a.ld_vec + c];
+  // 16-byte vectors when every row starts 16-byte aligned (d and the row stride multiples
+  // of 4 floats)
+  const bool v4 = ((d | a.ld_vec) & 3) == 0 && (reinterpret_cast<uintptr_t>(a.in) & 15) == 0 &&
+                  (reinterpret_cast<uintptr_t>(a.out) & 15) == 0 &&
+                  (reinterpret_cast<uintptr_t>(a.anchor) & 15) == 0;
+  if (v4) {
+    const int dv = d >> 2;
+    for (int k = 0; k < K; ++k)
+      for (int c = threadIdx.x; c < dv; c += PW_THREADS)
+        reinterpret_cast<float4*>(s_in + (size_t)k * d)[c] =
+            __ldcg(reinterpret_cast<const float4*>(inb + (size_t)k * a.ld_vec) + c);
+  } else {
+    for (int i = threadIdx.x; i < K * d; i += PW_THREADS) {
+      const int k = i / d, c = i % d;
+      s_in[i] = inb[(size_t)k * a.ld_vec + c];
+    }
   }
   __syncthreads();
   for (int k = warp; k < K; k += nw) {
@@ -160,6 +173,45 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
   for (int r = warp; r < nrows; r += nw) {
     const float* o = j == 0 ? a.anchor + (size_t)b * d
                             : a.out + ((size_t)(b * L + j - 1) * K + r) * a.ld_vec;
+    if (v4 && d <= 512) {
+      // the row in registers (up to 4 vectors per lane), four dot products at a time
+      float4 ov[4];
+      float oo = 0.f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = 4 * (lane + 32 * u);
+        ov[u] = c < d ? __ldcg(reinterpret_cast<const float4*>(o + c)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        oo = fmaf(ov[u].x, ov[u].x, fmaf(ov[u].y, ov[u].y, fmaf(ov[u].z, ov[u].z, fmaf(ov[u].w, ov[u].w, oo))));
+      }
+      const float on = fmaxf(sqrtf(warp_sum(oo)), UNIT_EPS);
+      for (int k0 = 0; k0 < K; k0 += 4) {
+        float dot[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int c = 4 * (lane + 32 * u);
+          if (c >= d) break;
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq)
+            if (k0 + qq < K) {
+              const float4 w = *reinterpret_cast<const float4*>(s_in + (size_t)(k0 + qq) * d + c);
+              dot[qq] = fmaf(ov[u].x, w.x, fmaf(ov[u].y, w.y, fmaf(ov[u].z, w.z, fmaf(ov[u].w, w.w, dot[qq]))));
+            }
+        }
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) dot[qq] = warp_sum(dot[qq]);
+        if (lane == 0) {
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) {
+            const int k2 = k0 + qq;
+            if (k2 >= K) break;
+            const float v = dot[qq] / (on * s_inn[k2]);
+            if (j == 0) a.A[(size_t)b * K + k2] = v;
+            else a.P[((size_t)b * (L - 1) + (j - 1)) * K * K + (size_t)r * K + k2] = v;
+          }
+        }
+      }
+      continue;
+    }
     float oo = 0.f;
     for (int c = lane; c < d; c += 32) oo = fmaf(o[c], o[c], oo);
     const float on = fmaxf(sqrtf(warp_sum(oo)), UNIT_EPS);
