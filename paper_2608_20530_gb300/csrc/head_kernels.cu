@@ -282,8 +282,14 @@ __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __r
   pdl_wait();
   __shared__ float f[LILICORR_MAX_K][LILICORR_N_CONF];
   __shared__ int sid[LILICORR_MAX_K];
+  extern __shared__ __align__(16) float s_w[];     // [N_CONF][D] = W_c1^T, then b_c1 [D]
   const int r = blockIdx.x;
   const int s = r % L;
+  for (int i = threadIdx.x; i < D; i += blockDim.x) {
+#pragma unroll
+    for (int j = 0; j < LILICORR_N_CONF; ++j) s_w[j * D + i] = w1[i * LILICORR_N_CONF + j];
+    s_w[LILICORR_N_CONF * D + i] = b1[i];
+  }
   if (threadIdx.x < K) {
     const int k = threadIdx.x;
     const float lp = logp[(size_t)r * K + k];
@@ -316,13 +322,24 @@ __global__ void node_build_kernel(int L, int K, int D, int V, const int32_t* __r
     o.z = fo.z + hp.z + sl.z + rk.z;
     o.w = fo.w + hp.w + sl.w + rk.w;
     *reinterpret_cast<float4*>(x + node * D + n) = o;
+    float4 z = *reinterpret_cast<const float4*>(s_w + LILICORR_N_CONF * D + n);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      float z = b1[n + q];
-#pragma unroll
-      for (int j = 0; j < LILICORR_N_CONF; ++j)
-        z = fmaf(w1[(n + q) * LILICORR_N_CONF + j], f[k][j], z);
-      st_elem(c1, node * D + n + q, silu_f(z));
+    for (int j = 0; j < LILICORR_N_CONF; ++j) {
+      const float4 w = *reinterpret_cast<const float4*>(s_w + j * D + n);
+      const float fj = f[k][j];
+      z.x = fmaf(w.x, fj, z.x);
+      z.y = fmaf(w.y, fj, z.y);
+      z.z = fmaf(w.z, fj, z.z);
+      z.w = fmaf(w.w, fj, z.w);
+    }
+    if constexpr (sizeof(TC1) == 2) {          // bf16 operand: tanh-based SiLU, 8-byte store
+      uint2 u;
+      u.x = bf16_pack2(silu_tanh(z.x), silu_tanh(z.y));
+      u.y = bf16_pack2(silu_tanh(z.z), silu_tanh(z.w));
+      *reinterpret_cast<uint2*>(c1 + node * D + n) = u;
+    } else {
+      *reinterpret_cast<float4*>(c1 + node * D + n) =
+          make_float4(silu_f(z.x), silu_f(z.y), silu_f(z.z), silu_f(z.w));
     }
   }
 }
@@ -498,11 +515,11 @@ lilicorr_status_t launch_node_build(const lilicorr_head* h, int B, const int32_t
   if (B == 0) return LILICORR_OK;
   const float* fold = static_cast<const float*>(h->fold);
   if (c1_dt == LILICORR_F32)
-    LL_TRY(launch_k(node_build_kernel<float>, B * d.L, 256, 0, st, d.L, d.K, d.D, d.V, ids, logp, fold, hproj,
+    LL_TRY(launch_k(node_build_kernel<float>, B * d.L, 256, sizeof(float) * (LILICORR_N_CONF + 1) * d.D, st, d.L, d.K, d.D, d.V, ids, logp, fold, hproj,
                                                       h->slot, h->rank, h->conf1_w, h->conf1_b,
                                                       static_cast<float*>(c1), x, status));
   else
-    LL_TRY(launch_k(node_build_kernel<__nv_bfloat16>, B * d.L, 256, 0, st, 
+    LL_TRY(launch_k(node_build_kernel<__nv_bfloat16>, B * d.L, 256, sizeof(float) * (LILICORR_N_CONF + 1) * d.D, st, 
         d.L, d.K, d.D, d.V, ids, logp, fold, hproj, h->slot, h->rank, h->conf1_w, h->conf1_b,
         static_cast<__nv_bfloat16*>(c1), x, status));
   return LILICORR_OK;

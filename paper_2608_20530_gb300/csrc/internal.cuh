@@ -126,6 +126,11 @@ __device__ __forceinline__ float warp_max(float v) {
 }
 
 __device__ __forceinline__ float silu_f(float z) { return z / (1.0f + __expf(-z)); }
+// two floats as a bf16 pair (round to nearest even), lo in the low half
+__device__ __forceinline__ uint32_t bf16_pack2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
 // SiLU(z) = z (1 + tanh(z / 2)) / 2 with one MUFU operation, for outputs rounded to bf16
 // (tanh.approx's error is below the bf16 rounding that follows)
 __device__ __forceinline__ float silu_tanh(float z) {
