@@ -265,9 +265,9 @@ lilicorr_status_t run_drafter_proj(const HeadCall& c, const void* hidden, cudaSt
   g.bias = h->hid_b;
   return run_gemm(g, st);
 }
-// (b) the target state t = W_t RMSNorm(mean of the captured layers) + b_t, the anchor out
-// vector W_a t + b_a (its consumers normalise it) and the fusion layer's t block, constant
-// per sequence: cb = W_f[:, t] t + b_f.
+// (b) the target state t = W_t RMSNorm(mean of the captured layers) + b_t, then two
+// independent products of t: the anchor out vector W_a t + b_a (its consumers normalise
+// it) and the fusion layer's t block, constant per sequence: cb = W_f[:, t] t + b_f.
 lilicorr_status_t run_target(const HeadCall& c, const void* target, cudaStream_t st) {
   const lilicorr_head* h = c.h;
   const lilicorr_head_desc& d = c.d;
@@ -276,12 +276,18 @@ lilicorr_status_t run_target(const HeadCall& c, const void* target, cudaStream_t
   LL_TRY(launch_target_norm(target, c.wdt, c.B, d.n_tgt, d.H, h->tgt_norm, c.tn, c.tn_dt, st));
   GemmArgs g = c.G(c.tn, c.tn_dt, d.H, h->tgt_w, d.H, c.t, F32, D, c.B, D, d.H);
   g.bias = h->tgt_b;
-  LL_TRY(run_gemm(g, st));
-  g = c.G(c.t, F32, D, h->anc_w, D, c.anc, F32, d.d, c.B, d.d, D);
-  g.bias = h->anc_b;
-  LL_TRY(run_gemm(g, st));
-  g = c.G(c.t, F32, D, h->fuse_t, D, c.cb, F32, D, c.B, D, D);
-  g.bias = h->fuse_b;
+  return run_gemm(g, st);
+}
+lilicorr_status_t run_anchor(const HeadCall& c, cudaStream_t st) {
+  GemmArgs g = c.G(c.t, LILICORR_F32, c.D, c.h->anc_w, c.D, c.anc, LILICORR_F32, c.d.d, c.B,
+                   c.d.d, c.D);
+  g.bias = c.h->anc_b;
+  return run_gemm(g, st);
+}
+lilicorr_status_t run_fusion_t(const HeadCall& c, cudaStream_t st) {
+  GemmArgs g = c.G(c.t, LILICORR_F32, c.D, c.h->fuse_t, c.D, c.cb, LILICORR_F32, c.D, c.B, c.D,
+                   c.D);
+  g.bias = c.h->fuse_b;
   return run_gemm(g, st);
 }
 // Fork both chains from `st` onto the head's side streams; join_prologue makes `st` wait
@@ -292,8 +298,14 @@ lilicorr_status_t fork_prologue(const HeadCall& c, const void* hidden, const voi
   LL_CUDA_TRY(cudaEventRecord(hm->ev_fork, st));
   LL_CUDA_TRY(cudaStreamWaitEvent(hm->side, hm->ev_fork, 0));
   LL_CUDA_TRY(cudaStreamWaitEvent(hm->side2, hm->ev_fork, 0));
-  const lilicorr_status_t s1 = run_drafter_proj(c, hidden, hm->side);
-  const lilicorr_status_t s2 = run_target(c, target, hm->side2);
+  // side: drafter-state projection, then (once t exists) the fusion layer's t block;
+  // side2: the target state, then the anchor vector
+  lilicorr_status_t s1 = run_drafter_proj(c, hidden, hm->side);
+  lilicorr_status_t s2 = run_target(c, target, hm->side2);
+  LL_CUDA_TRY(cudaEventRecord(hm->ev_t, hm->side2));
+  LL_CUDA_TRY(cudaStreamWaitEvent(hm->side, hm->ev_t, 0));
+  if (s1 == LILICORR_OK) s1 = run_fusion_t(c, hm->side);
+  if (s2 == LILICORR_OK) s2 = run_anchor(c, hm->side2);
   LL_CUDA_TRY(cudaEventRecord(hm->ev_join, hm->side));
   LL_CUDA_TRY(cudaEventRecord(hm->ev_join2, hm->side2));
   return s1 != LILICORR_OK ? s1 : s2;
@@ -484,6 +496,7 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
     if (h->ev_fork) cudaEventDestroy(h->ev_fork);
     if (h->ev_join) cudaEventDestroy(h->ev_join);
     if (h->ev_join2) cudaEventDestroy(h->ev_join2);
+    if (h->ev_t) cudaEventDestroy(h->ev_t);
     free(h);
     return s;
   };
@@ -491,7 +504,8 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
       cudaStreamCreateWithFlags(&h->side2, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join2, cudaEventDisableTiming) != cudaSuccess)
+      cudaEventCreateWithFlags(&h->ev_join2, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_t, cudaEventDisableTiming) != cudaSuccess)
     return fail(LILICORR_ERR_CUDA);
   if (cudaMalloc(&h->pool, pool_bytes) != cudaSuccess) return fail(LILICORR_ERR_CUDA);
   h->pool_bytes = pool_bytes;
@@ -553,6 +567,7 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
   if (h->ev_join) cudaEventDestroy(h->ev_join);
   if (h->ev_join2) cudaEventDestroy(h->ev_join2);
+  if (h->ev_t) cudaEventDestroy(h->ev_t);
   if (cur != h->device) cudaSetDevice(cur);
   free(h);
   return e == cudaSuccess ? LILICORR_OK : LILICORR_ERR_CUDA;

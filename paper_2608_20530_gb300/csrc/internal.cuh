@@ -168,7 +168,7 @@ struct lilicorr_head {
   // the projections that do not depend on the top-K pass run on two side streams that
   // fork from and join the caller's stream (fork/join nodes under graph capture)
   cudaStream_t side, side2;
-  cudaEvent_t ev_fork, ev_join, ev_join2;
+  cudaEvent_t ev_fork, ev_join, ev_join2, ev_t;   // ev_t: the target state t is ready
   void* pool;                 // one device allocation holding everything below
   size_t pool_bytes;
   // matrices in head dtype; vectors and tables in fp32
