@@ -8,13 +8,13 @@
 // and heads 2c, 2c+1. Each product computes only the CTA's output slice:
 //   conf2, W_o, W_2     x[:, slice] += A W[slice, :]^T            (N = 64)
 //   q|k|v               the q, k, v rows of head pair c            (N = 192)
+//   W_1                 FFN hidden units 128c..128c+127            (N = 128)
 //   heads               [o | i][:, 128c..128c+127]                 (N = 128)
-// while W_1 (both halves) and the fusion layer run in full on every CTA (their outputs
-// are consumed locally: the FFN hidden state by W_2's K, u by the heads), so the FFN
-// hidden state and u never travel.
+// while the fusion layer runs in full on every CTA (u is consumed locally by the heads).
 // The operands that need every CTA's slice are all-gathered through distributed shared
 // memory: each CTA writes its slice of RMSNorm(x) (before q|k|v and before W_1), of the
-// attention output (before W_o) and of the fusion input [xf | xf*t] into the same place
+// attention output (before W_o), of the FFN hidden state (before W_2; it fills both
+// operand buffers) and of the fusion input [xf | xf*t] into the same place
 // in all four CTAs' operand buffers with st.async, whose bytes complete the transaction
 // count of the receiving CTA's mbarrier for that exchange; the receiving MMA thread waits
 // on it (acquire, cluster scope). RMSNorm statistics travel the same way: each CTA sends
@@ -75,8 +75,9 @@ constexpr uint32_t OFF_SAME = OFF_DIST + NC_NH * (2 * NC_MAX_L - 1) * 4;
 constexpr uint32_t OFF_SLOT = OFF_SAME + NC_NH * 4;                // [128]
 constexpr uint32_t OFF_IDS = OFF_SLOT + NC_M;                      // [128]
 constexpr uint32_t OFF_BAR = (OFF_IDS + NC_M * 4 + 63) & ~63u;
-constexpr int N_DONE = 2 + 5 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 2 + 5 * NC_MAX_LAYERS;
-constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_STAGES + N_DONE + N_READY + N_XG) * 8;
+constexpr int N_DONE = 2 + 4 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 2 + 6 * NC_MAX_LAYERS;
+constexpr int N_W1F = NC_MAX_LAYERS;
+constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_STAGES + N_DONE + N_READY + N_XG + N_W1F) * 8;
 constexpr size_t NC_SMEM = 1024 + NC_SMEM_USED;
 static_assert(NC_SMEM <= 227 * 1024, "shared memory of the cluster network kernel");
 static_assert(OFF_ACT % 1024 == 0 && OFF_HF % 1024 == 0, "swizzle atoms");
@@ -84,30 +85,33 @@ static_assert(OFF_ACT % 1024 == 0 && OFF_HF % 1024 == 0, "swizzle atoms");
 // bytes a CTA receives from its three peers per exchange
 constexpr uint32_t XB_SS = (NC_CC - 1) * NC_M * 4;
 constexpr uint32_t XB_SLICE = (NC_CC - 1) * NC_M * NC_SL * 2;
+constexpr uint32_t XB_H = (NC_CC - 1) * NC_M * (NC_F / NC_CC) * 2;   // 128 hidden units each
 
 enum { G_CONF2, G_QKV, G_WO, G_W1, G_W2, G_FUSE, G_WOI };
 
-// events: MMA -> row workers (done), row workers -> MMA (ready, 16 warp arrivals), and
-// exchanges (xg: the peers' bytes). One sequence per cluster: every event completes once.
-__device__ __forceinline__ int lb(int l) { return 1 + 5 * l; }
-__device__ __forceinline__ int xb(int l) { return 5 * l; }
+// events: MMA -> row workers (done), row workers -> MMA (ready, 16 warp arrivals),
+// exchanges (xg: the peers' bytes) and the hand-shake of the FFN hidden state (w1f: the
+// three peers' W_1 products are done, so their ACT buffers may be overwritten). One
+// sequence per cluster: every event completes once.
+__device__ __forceinline__ int lb(int l) { return 1 + 4 * l; }
+__device__ __forceinline__ int xb(int l) { return 6 * l; }
 // done
 __device__ __forceinline__ int D_QKV(int l) { return lb(l); }
 __device__ __forceinline__ int D_WO(int l) { return lb(l) + 1; }
-__device__ __forceinline__ int D_FFN(int l, int h) { return lb(l) + 2 + h; }
-__device__ __forceinline__ int D_LAYER(int l) { return lb(l) + 4; }
+__device__ __forceinline__ int D_W1(int l) { return lb(l) + 2; }
+__device__ __forceinline__ int D_LAYER(int l) { return lb(l) + 3; }
 // ready
 __device__ __forceinline__ int R_XN(int l) { return lb(l); }
 __device__ __forceinline__ int R_ATT(int l) { return lb(l) + 1; }
 __device__ __forceinline__ int R_XN2(int l) { return lb(l) + 2; }
-__device__ __forceinline__ int R_HFA(int l) { return lb(l) + 3; }
-__device__ __forceinline__ int R_HFB(int l) { return lb(l) + 4; }
+__device__ __forceinline__ int R_H(int l) { return lb(l) + 3; }
 // exchanges
 __device__ __forceinline__ int X_SS(int l) { return xb(l); }
 __device__ __forceinline__ int X_XN(int l) { return xb(l) + 1; }
 __device__ __forceinline__ int X_ATT(int l) { return xb(l) + 2; }
 __device__ __forceinline__ int X_SS2(int l) { return xb(l) + 3; }
 __device__ __forceinline__ int X_XN2(int l) { return xb(l) + 4; }
+__device__ __forceinline__ int X_H(int l) { return xb(l) + 5; }
 
 struct ClusterMaps {
   CUtensorMap conf2, fuse, woi;
@@ -144,8 +148,8 @@ __device__ __forceinline__ int n_chunks(int kind) {
 __device__ __forceinline__ int tile_rows(int kind) {
   switch (kind) {
     case G_QKV: return 192;
-    case G_W1: case G_FUSE: return 256;
-    case G_WOI: return 128;
+    case G_FUSE: return 256;
+    case G_W1: case G_WOI: return 128;
     default: return NC_SL;
   }
 }
@@ -156,7 +160,7 @@ __device__ __forceinline__ void load_chunk(const ClusterMaps& m, int kind, int l
     case G_CONF2: tma_load_3d(dst, &m.conf2, bar, 0, NC_SL * me, kc); break;
     case G_QKV: tma_load_5d(dst, &m.wqkv[l], bar, 0, 0, me, 0, kc); break;
     case G_WO: tma_load_3d(dst, &m.wo[l], bar, 0, NC_SL * me, kc); break;
-    case G_W1: tma_load_3d(dst, &m.w1[l], bar, 0, 256 * h, kc); break;
+    case G_W1: tma_load_3d(dst, &m.w1[l], bar, 0, 128 * me, kc); break;
     case G_W2: tma_load_3d(dst, &m.w2[l], bar, 0, NC_SL * me, kc); break;
     case G_FUSE: tma_load_3d(dst, &m.fuse, bar, 0, 0, kc); break;
     default: tma_load_3d(dst, &m.woi, bar, 0, 128 * me, kc); break;
@@ -170,7 +174,6 @@ __device__ __forceinline__ void schedule(const ClusterArgs& a, Op& op) {
     op.gemm(G_QKV, l, 0);
     op.gemm(G_WO, l, 0);
     op.gemm(G_W1, l, 0);
-    op.gemm(G_W1, l, 1);
     op.gemm(G_W2, l, 0);
   }
   op.gemm(G_FUSE, 0, 0);
@@ -179,7 +182,7 @@ __device__ __forceinline__ void schedule(const ClusterArgs& a, Op& op) {
 
 struct Shared {
   uint8_t* base;
-  uint64_t *full, *empty, *done, *ready, *xg;
+  uint64_t *full, *empty, *done, *ready, *xg, *w1f;
   volatile int* abort;
 };
 
@@ -235,11 +238,8 @@ struct Issuer {
       case G_CONF2: rd = 0; dn = 0; break;
       case G_QKV: rd = R_XN(l); xw = X_XN(l); dn = D_QKV(l); break;
       case G_WO: rd = R_ATT(l); xw = X_ATT(l); dn = D_WO(l); break;
-      case G_W1:
-        if (h == 0) { rd = R_XN2(l); xw = X_XN2(l); } else { rd = R_HFA(l); }
-        dn = D_FFN(l, h);
-        break;
-      case G_W2: rd = R_HFB(l); dn = D_LAYER(l); break;
+      case G_W1: rd = R_XN2(l); xw = X_XN2(l); dn = D_W1(l); break;
+      case G_W2: rd = R_H(l); xw = X_H(l); dn = D_LAYER(l); break;
       case G_FUSE: rd = lb(nl); xw = xb(nl) + 1; dn = lb(nl); break;
       default: rd = lb(nl) + 1; dn = lb(nl) + 1; break;
     }
@@ -305,18 +305,23 @@ struct Peers {
 };
 
 // 16 values (row r, columns 16cg.. of this CTA's slice) as bf16 into chunk `me` of an
-// operand buffer here and in the three peers (two 16-byte pieces each); the peers' copies
-// count toward their exchange barrier `xbar` (same offset in every CTA).
-__device__ __forceinline__ void put16_all(uint8_t* buf, int me, int r, int cg, const float (&v)[16],
-                                          uint64_t* xbar, const Peers& pe) {
+// operand buffer (two 16-byte pieces).
+__device__ __forceinline__ void put16(uint8_t* buf, int me, int r, int cg, const float (&v)[16]) {
   uint8_t* ch = buf + (size_t)me * CHUNK;
 #pragma unroll
-  for (int p = 0; p < 2; ++p) {
-    const uint4 w = pack8(v + 8 * p);
-    uint8_t* dst = ch + swz(r, 2 * cg + p);
-    *reinterpret_cast<uint4*>(dst) = w;
+  for (int p = 0; p < 2; ++p) *reinterpret_cast<uint4*>(ch + swz(r, 2 * cg + p)) = pack8(v + 8 * p);
+}
+// After every row worker wrote its part of `bytes` at src here: the same bytes into the
+// same place in the three peers by the bulk-copy engine, counted on their exchange barrier
+// `xbar` (one thread issues; it waits until the source has been read).
+__device__ __forceinline__ void send_all(const void* src, uint32_t bytes, uint64_t* xbar, int tid,
+                                         const Peers& pe) {
+  fence_async_shared();
+  rw_bar();
+  if (tid == 0) {
 #pragma unroll
-    for (int q = 1; q < NC_CC; ++q) st_peer16(pe.at(q, dst), w, pe.at(q, xbar));
+    for (int q = 1; q < NC_CC; ++q) bulk_to_peer(pe.at(q, src), src, bytes, pe.at(q, xbar));
+    bulk_wait_read();
   }
 }
 
@@ -357,15 +362,25 @@ __device__ void norm_stats(uint32_t tx, const float* bias, bool write_back, int 
 // norm_operand: v * gain into chunk me of `buf` everywhere (exchange `xop`), and with t,
 // v * gain * t into chunk me of `buf2`.
 __device__ void norm_operand(float (&v)[16], const float* gain, uint8_t* buf, const float* t,
-                             uint8_t* buf2, uint64_t* xop, int cg, int r, int me,
+                             uint8_t* buf2, uint64_t* xop, int cg, int r, int me, int tid,
                              const Peers& pe) {
 #pragma unroll
   for (int e = 0; e < 16; ++e) v[e] *= gain[16 * cg + e];
-  put16_all(buf, me, r, cg, v, xop, pe);
+  put16(buf, me, r, cg, v);
   if (t) {
 #pragma unroll
     for (int e = 0; e < 16; ++e) v[e] *= t[16 * cg + e];
-    put16_all(buf2, me, r, cg, v, xop, pe);
+    put16(buf2, me, r, cg, v);
+  }
+  fence_async_shared();
+  rw_bar();
+  if (tid == 0) {
+#pragma unroll
+    for (int q = 1; q < NC_CC; ++q) {
+      bulk_to_peer(pe.at(q, buf + (size_t)me * CHUNK), buf + (size_t)me * CHUNK, CHUNK, pe.at(q, xop));
+      if (t) bulk_to_peer(pe.at(q, buf2 + (size_t)me * CHUNK), buf2 + (size_t)me * CHUNK, CHUNK, pe.at(q, xop));
+    }
+    bulk_wait_read();
   }
 }
 // norm_recv: 1 / rms of row r over the 256 columns, once every CTA's partial is here.
@@ -409,6 +424,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
   sh.done = sh.empty + NC_STAGES;
   sh.ready = sh.done + N_DONE;
   sh.xg = sh.ready + N_READY;
+  sh.w1f = sh.xg + N_XG;
   sh.abort = &abort_flag;
   float* s_ss = reinterpret_cast<float*>(sm + OFF_SS);
   float* s_ssx = reinterpret_cast<float*>(sm + OFF_SSX);
@@ -432,6 +448,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       mbar_init(&sh.ready[e], NC_RW / 32);
     }
     for (int e = 0; e < N_XG; ++e) mbar_init(&sh.xg[e], 1);
+    for (int e = 0; e < N_W1F; ++e) mbar_init(&sh.w1f[e], NC_CC - 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // every exchange barrier: this CTA's own arrival now, the peers' bytes later
@@ -441,6 +458,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       mbar_expect_tx(&sh.xg[X_ATT(l)], XB_SLICE);
       mbar_expect_tx(&sh.xg[X_SS2(l)], XB_SS);
       mbar_expect_tx(&sh.xg[X_XN2(l)], XB_SLICE);
+      mbar_expect_tx(&sh.xg[X_H(l)], XB_H);
     }
     mbar_expect_tx(&sh.xg[xb(nl)], XB_SS);
     mbar_expect_tx(&sh.xg[xb(nl) + 1], 2 * XB_SLICE);
@@ -625,7 +643,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         norm_stats(tx, l == 0 ? nullptr : vec + V_B2 + ((l - 1) & 1) * NC_SL, true, cg, r, me,
                    s_ss, s_ssx, &sh.xg[X_SS(l)], pe, v);
         rs1 = norm_recv(r, s_ssx, &sh.xg[X_SS(l)], sh.abort);
-        norm_operand(v, vec + V_AN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[X_XN(l)], cg, r, me, pe);
+        norm_operand(v, vec + V_AN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[X_XN(l)], cg, r, me, tid,
+                     pe);
       }
       rw_signal(&sh.ready[R_XN(l)], lane);
 
@@ -656,8 +675,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         float o[4][4], inv0, inv1;
         head_attention(smem_u32(qs), LK, K, s_slot, s_dist + hh * nd + (L - 1), s_same[hh], q0,
                        lane, o, inv0, inv1);
-        // the pair's 64 attention-output columns: chunk me of HF here, then the warp's 16
-        // rows x 4 pieces of 16 bytes to the peers, two pieces per lane
+        // the pair's 64 attention-output columns: chunk me of HF, here and in the peers
         uint8_t* att = sm + OFF_HF + (size_t)me * CHUNK;
 #pragma unroll
         for (int nb = 0; nb < 4; ++nb) {
@@ -667,16 +685,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
           *reinterpret_cast<uint32_t*>(att + swz(i1, piece) + 4 * t4) =
               pack_bf16x2(o[nb][2] * inv1, o[nb][3] * inv1);
         }
-        __syncwarp();
-        uint64_t* xbar = &sh.xg[X_ATT(l)];
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-          const int pi = 2 * lane + k;
-          const uint8_t* src = att + swz(q0 + (pi >> 2), 4 * set + (pi & 3));
-          const uint4 w = *reinterpret_cast<const uint4*>(src);
-#pragma unroll
-          for (int qq = 1; qq < NC_CC; ++qq) st_peer16(pe.at(qq, src), w, pe.at(qq, xbar));
-        }
+        send_all(att, CHUNK, &sh.xg[X_ATT(l)], tid, pe);
       }
       rw_signal(&sh.ready[R_ATT(l)], lane);
 
@@ -688,19 +697,51 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         norm_stats(tx, vec + V_BO, true, cg, r, me, s_ss, s_ssx + NC_CC * NC_M, &sh.xg[X_SS2(l)],
                    pe, v);
         norm_operand(v, vec + V_FN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[X_XN2(l)], cg, r, me,
-                     pe);
+                     tid, pe);
       }
       rw_signal(&sh.ready[R_XN2(l)], lane);
       const float rs2 = norm_recv(r, s_ssx + NC_CC * NC_M, &sh.xg[X_SS2(l)], sh.abort);
-      // FFN hidden state, both halves in full on every CTA
-      ev_wait(&sh.done[D_FFN(l, 0)], sh.abort);
+      // FFN hidden units 128me..128me+127: SiLU(rs2 * acc + b_1) -> bf16, gathered into
+      // the W_2 operand (units 0-255 in HF, 256-511 in ACT) here and in every peer. ACT
+      // still holds the W_1 operand until each CTA's W_1 product is done: CTAs that write
+      // there wait for the three peers' word (the W_1 products' completion, signalled as
+      // soon as this CTA sees its own).
+      ev_wait(&sh.done[D_W1(l)], sh.abort);
       tc_fence_after();
-      drain_silu(sm + OFF_HF, tscr, vec + V_B1, rs2, cg, r);
-      rw_signal(&sh.ready[R_HFA(l)], lane);
-      ev_wait(&sh.done[D_FFN(l, 1)], sh.abort);
-      tc_fence_after();
-      drain_silu(sm + OFF_ACT, tscr, vec + V_B1 + 256, rs2, cg, r);
-      rw_signal(&sh.ready[R_HFB(l)], lane);
+      if (tid == 0) {
+        uint64_t* wf = &sh.w1f[l];
+#pragma unroll
+        for (int qq = 1; qq < NC_CC; ++qq) mbar_arrive_peer(pe.at(qq, wf));
+      }
+      {
+        uint8_t* hbuf = me < 2 ? sm + OFF_HF : sm + OFF_ACT;
+        const int ch0 = 2 * (me & 1);              // the two chunks of this CTA's units
+        float v[32];
+        ld32f(tscr + 32 * cg, v);
+        const float* b1 = vec + V_B1 + 128 * me + 32 * cg;
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          v[e] = fmaf(rs2, v[e], b1[e]);
+          v[e + 1] = fmaf(rs2, v[e + 1], b1[e + 1]);
+          silu2(v[e], v[e + 1]);
+        }
+        // columns 32cg..32cg+31 of the 128: chunk ch0 + (cg >> 1), pieces 4(cg & 1)..+3
+        uint8_t* ch = hbuf + (size_t)(ch0 + (cg >> 1)) * CHUNK;
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+          *reinterpret_cast<uint4*>(ch + swz(r, 4 * (cg & 1) + p)) = pack8(v + 8 * p);
+        fence_async_shared();
+        rw_bar();
+        if (tid == 0) {
+          if (me >= 2) xg_wait(&sh.w1f[l], sh.abort);   // the peers' ACT is free
+          uint8_t* src = hbuf + (size_t)ch0 * CHUNK;
+#pragma unroll
+          for (int qq = 1; qq < NC_CC; ++qq)
+            bulk_to_peer(pe.at(qq, src), src, 2 * CHUNK, pe.at(qq, &sh.xg[X_H(l)]));
+          bulk_wait_read();
+        }
+      }
+      rw_signal(&sh.ready[R_H(l)], lane);
     }
 
     // ---- fusion: xf = RMSNorm(x + b_2) -> ACT, xf * t -> HF (slices everywhere);
@@ -714,7 +755,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
                  &sh.xg[xb(nl)], pe, v);
       rsf = norm_recv(r, s_ssx, &sh.xg[xb(nl)], sh.abort);
       norm_operand(v, vec + V_FIN, sm + OFF_ACT, vec + V_T, sm + OFF_HF, &sh.xg[xb(nl) + 1], cg, r,
-                   me, pe);
+                   me, tid, pe);
     }
     rw_signal(&sh.ready[lb(nl)], lane);
     ev_wait(&sh.done[lb(nl)], sh.abort);
@@ -803,7 +844,7 @@ void* net_cluster_maps_create(const lilicorr_head* h) {
   for (int l = 0; l < d.n_layers && ok; ++l) {
     const HeadW& w = h->layer[l];
     ok = nc_qkv_map(&m->wqkv[l], w.wqkv) && nc_chunk_map(&m->wo[l], w.wo, NC_D, NC_D, NC_SL) &&
-         nc_chunk_map(&m->w1[l], w.w1, NC_F, NC_D, 256) &&
+         nc_chunk_map(&m->w1[l], w.w1, NC_F, NC_D, 128) &&
          nc_chunk_map(&m->w2[l], w.w2, NC_D, NC_F, NC_SL);
   }
   for (int l = d.n_layers; l < NC_MAX_LAYERS && ok; ++l) {   // unused slots: valid maps

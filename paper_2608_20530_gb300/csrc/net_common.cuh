@@ -60,6 +60,24 @@ __device__ __forceinline__ void st_peer4(uint32_t raddr, uint32_t v, uint32_t rb
   asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];"
                ::"r"(raddr), "r"(v), "r"(rbar) : "memory");
 }
+// `bytes` (a multiple of 16) of this CTA's shared memory at src into a peer's shared memory
+// at dst (peer address) by the bulk-copy engine, counted on the peer's mbarrier rbar (peer
+// address); the writers of src must have fenced their generic-proxy writes (and synced)
+__device__ __forceinline__ void bulk_to_peer(uint32_t dst, const void* src, uint32_t bytes,
+                                             uint32_t rbar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "r"(smem_u32(src)), "r"(bytes), "r"(rbar) : "memory");
+}
+// wait until this thread's bulk copies have read their sources
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.commit_group;\n cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// one arrival on a peer's mbarrier (peer address), releasing this thread's prior writes
+__device__ __forceinline__ void mbar_arrive_peer(uint32_t rbar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(rbar)
+               : "memory");
+}
 // wait for a phase whose completion was signalled by other CTAs of the cluster (bounded)
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
