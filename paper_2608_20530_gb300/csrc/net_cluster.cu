@@ -44,12 +44,12 @@ using namespace net;
 constexpr int NC_CC = 4;                  // CTAs per sequence
 constexpr int NC_D = 256, NC_F = 512, NC_NH = 8, NC_HD = 32, NC_M = 128;
 constexpr int NC_SL = NC_D / NC_CC;       // 64 columns of x per CTA
-constexpr int NC_STAGES = 2;
+constexpr int NC_SLOTS = 8;               // weight ring: 8 slots of 64 rows x 64 k
 constexpr int NC_MAX_LAYERS = 4;
 constexpr int NC_MAX_L = 64;
 constexpr int NC_RW = 512;                // row-worker threads
 constexpr int NC_THREADS = 64 + NC_RW;
-constexpr uint32_t NC_STAGE = 256 * 128;  // one K chunk of up to 256 weight rows
+constexpr uint32_t NC_SLOT = 64 * 128;
 constexpr uint32_t NC_TMEM = 512;
 constexpr uint32_t X_COL = 0, SCR_COL = 256;
 constexpr long long NC_WAIT = 4000000000ll;
@@ -59,7 +59,7 @@ constexpr uint32_t QKV_SET = 3 * 8192;    // q, k, v of one head
 
 // shared memory (offsets from the 1024-aligned base)
 constexpr uint32_t OFF_RING = 0;
-constexpr uint32_t OFF_ACT = OFF_RING + NC_STAGES * NC_STAGE;      // 4 chunks
+constexpr uint32_t OFF_ACT = OFF_RING + NC_SLOTS * NC_SLOT;        // 4 chunks
 constexpr uint32_t OFF_HF = OFF_ACT + 4 * CHUNK;                   // 4 chunks
 constexpr uint32_t OFF_VEC = OFF_HF + 4 * CHUNK;
 constexpr int V_AN = 0, V_FN = 64, V_BO = 128, V_B2 = 192, V_FIN = 320, V_C2B = 384, V_T = 448,
@@ -77,7 +77,7 @@ constexpr uint32_t OFF_IDS = OFF_SLOT + NC_M;                      // [128]
 constexpr uint32_t OFF_BAR = (OFF_IDS + NC_M * 4 + 63) & ~63u;
 constexpr int N_DONE = 2 + 4 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 2 + 6 * NC_MAX_LAYERS;
 constexpr int N_W1F = NC_MAX_LAYERS;
-constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_STAGES + N_DONE + N_READY + N_XG + N_W1F) * 8;
+constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_SLOTS + N_DONE + N_READY + N_XG + N_W1F) * 8;
 constexpr size_t NC_SMEM = 1024 + NC_SMEM_USED;
 static_assert(NC_SMEM <= 227 * 1024, "shared memory of the cluster network kernel");
 static_assert(OFF_ACT % 1024 == 0 && OFF_HF % 1024 == 0, "swizzle atoms");
@@ -188,7 +188,7 @@ struct Shared {
 
 __device__ __forceinline__ bool ev_wait(uint64_t* bar, volatile int* abort) {
   if (*abort) return false;
-  if (!mbar_wait(bar, 0, NC_WAIT)) {
+  if (!mbar_wait_sleep(bar, 0, NC_WAIT)) {
     *abort = 1;
     return false;
   }
@@ -196,31 +196,45 @@ __device__ __forceinline__ bool ev_wait(uint64_t* bar, volatile int* abort) {
 }
 __device__ __forceinline__ bool xg_wait(uint64_t* bar, volatile int* abort) {
   if (*abort) return false;
-  if (!mbar_wait_cluster(bar, 0, NC_WAIT)) {
+  if (!mbar_wait_cluster_sleep(bar, 0, NC_WAIT)) {
     *abort = 1;
     return false;
   }
   return true;
 }
 
+// The weight ring: a K chunk of a product slice (64 rows per slot) sits in consecutive
+// slots, starting over at slot 0 where it would run past the last one; producer and
+// issuer walk the same schedule, so they skip the same slots. Each slot has its own
+// phase (bit `slot` of a mask): full is armed on a chunk's first slot, empty is signalled
+// for every slot of it.
+__device__ __forceinline__ int ring_place(uint32_t& pos, int slots) {
+  int first = (int)(pos % NC_SLOTS);
+  if (first + slots > NC_SLOTS) {
+    pos += NC_SLOTS - first;
+    first = 0;
+  }
+  pos += slots;
+  return first;
+}
+
 struct Producer {
   const ClusterMaps* m;
   Shared sh;
   int me;
-  uint32_t n;
+  uint32_t pos, ph;
   __device__ void gemm(int kind, int l, int h) {
-    const int nk = n_chunks(kind);
+    const int nk = n_chunks(kind), ns = tile_rows(kind) / 64;
     const uint32_t bytes = (uint32_t)tile_rows(kind) * 128u;
-    for (int kc = 0; kc < nk; ++kc, ++n) {
-      const int s = (int)(n % NC_STAGES);
-      const uint32_t ph = (n / NC_STAGES) & 1u;
-      if (!mbar_wait(&sh.empty[s], ph ^ 1u, NC_WAIT)) {
-        *sh.abort = 1;
-        continue;
+    for (int kc = 0; kc < nk; ++kc) {
+      const int s0 = ring_place(pos, ns);
+      for (int i = s0; i < s0 + ns; ++i) {
+        if (!mbar_wait(&sh.empty[i], ((ph >> i) & 1u) ^ 1u, NC_WAIT)) *sh.abort = 1;
+        ph ^= 1u << i;
       }
       if (*sh.abort) continue;
-      mbar_expect_tx(&sh.full[s], bytes);
-      load_chunk(*m, kind, l, h, kc, me, sh.base + OFF_RING + (size_t)s * NC_STAGE, &sh.full[s]);
+      mbar_expect_tx(&sh.full[s0], bytes);
+      load_chunk(*m, kind, l, h, kc, me, sh.base + OFF_RING + (size_t)s0 * NC_SLOT, &sh.full[s0]);
     }
   }
 };
@@ -228,7 +242,7 @@ struct Producer {
 struct Issuer {
   const ClusterArgs* a;
   Shared sh;
-  uint32_t n, tmem;
+  uint32_t pos, ph, tmem;
   __device__ void gemm(int kind, int l, int h) {
     const int nl = a->n_layers;
     // what the product waits for: the row workers' part, and for gathered operands the
@@ -243,15 +257,17 @@ struct Issuer {
       case G_FUSE: rd = lb(nl); xw = xb(nl) + 1; dn = lb(nl); break;
       default: rd = lb(nl) + 1; dn = lb(nl) + 1; break;
     }
+    const bool lead = (threadIdx.x & 31) == 0;     // the lane that issues and commits
     ev_wait(&sh.ready[rd], sh.abort);
     if (xw >= 0) xg_wait(&sh.xg[xw], sh.abort);
+    __syncwarp();
     tc_fence_after();
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // peers' st.async data
-    const int nk = n_chunks(kind);
+    const int nk = n_chunks(kind), ns = tile_rows(kind) / 64;
     const bool onto_x = kind == G_CONF2 || kind == G_WO || kind == G_W2;
     const uint32_t d = tmem + (onto_x ? X_COL : SCR_COL);
     const uint32_t idesc = instr_desc(128, tile_rows(kind));
-    for (int kc = 0; kc < nk; ++kc, ++n) {
+    for (int kc = 0; kc < nk; ++kc) {
       uint32_t a_off;                               // the A operand's K chunk
       switch (kind) {
         case G_WO: a_off = OFF_HF + kc * CHUNK; break;                  // attention output
@@ -259,18 +275,25 @@ struct Issuer {
         case G_FUSE: a_off = kc < 4 ? OFF_ACT + kc * CHUNK : OFF_HF + (kc - 4) * CHUNK; break;
         default: a_off = OFF_ACT + kc * CHUNK; break;
       }
-      const int s = (int)(n % NC_STAGES);
-      const uint32_t ph = (n / NC_STAGES) & 1u;
-      if (!ev_wait_full(s, ph)) continue;
+      const int s0 = ring_place(pos, ns);
+      const uint32_t par = (ph >> s0) & 1u;
+      ph ^= 1u << s0;
+      const bool full = ev_wait_full(s0, par);
+      __syncwarp();
+      if (!full) continue;
       tc_fence_after();
       const uint64_t ad = smem_desc(sh.base + a_off);
-      const uint64_t bd = smem_desc(sh.base + OFF_RING + (size_t)s * NC_STAGE);
+      const uint64_t bd = smem_desc(sh.base + OFF_RING + (size_t)s0 * NC_SLOT);
+      if (lead) {
 #pragma unroll
-      for (int k = 0; k < 4; ++k)
-        mma_bf16(d, ad + 2ull * k, bd + 2ull * k, idesc, (onto_x || kc > 0 || k > 0) ? 1u : 0u);
-      mma_commit(&sh.empty[s]);
+        for (int k = 0; k < 4; ++k)
+          mma_bf16(d, ad + 2ull * k, bd + 2ull * k, idesc, (onto_x || kc > 0 || k > 0) ? 1u : 0u);
+        for (int i = s0; i < s0 + ns; ++i) mma_commit(&sh.empty[i]);
+      }
+      __syncwarp();
     }
-    if (!*sh.abort) mma_commit(&sh.done[dn]);
+    if (!*sh.abort && lead) mma_commit(&sh.done[dn]);
+    __syncwarp();
   }
   __device__ bool ev_wait_full(int s, uint32_t ph) {
     if (*sh.abort) return false;
@@ -410,6 +433,39 @@ __device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, float
   }
 }
 
+// The drafter-state, slot and rank table rows of this CTA's slice in ACT: 256-byte rows
+// (64 fp32) whose 16-byte pieces are XOR-swizzled by row; c is a multiple of 4 below 64.
+__device__ __forceinline__ float* tab_at(uint8_t* sm, int row, int c) {
+  return reinterpret_cast<float*>(sm + OFF_ACT) + (size_t)row * NC_SL + ((((c >> 2) ^ (row & 7))) << 2);
+}
+
+// Layer l's vectors (this CTA's slices of the norm gains, b_o and b_2; b_1, the q|k|v
+// biases, the relative-position and same-slot biases) into shared memory by asynchronous
+// copies: issued once the previous readers are past a barrier, completed (and the biases
+// scaled by log2 e) by layer_vectors_finish from the same thread before a barrier.
+__device__ void layer_vectors_issue(const ClusterArgs& a, int l, float* vec, float* s_dist,
+                                    float* s_same, int tid, int c0s, int nd) {
+  for (int i = tid; i < 4 * (NC_SL / 4); i += NC_RW) {
+    const int part = i / (NC_SL / 4), c = 4 * (i % (NC_SL / 4));
+    const float* src = part == 0 ? a.an[l] : part == 1 ? a.fn[l] : part == 2 ? a.bo[l] : a.b2[l];
+    float* dst = vec + (part == 0 ? V_AN : part == 1 ? V_FN : part == 2 ? V_BO : V_B2 + (l & 1) * NC_SL);
+    cp_async16(dst + c, src + c0s + c);
+  }
+  for (int i = tid; i < NC_F / 4; i += NC_RW) cp_async16(vec + V_B1 + 4 * i, a.b1[l] + 4 * i);
+  for (int i = tid; i < 3 * NC_D / 4; i += NC_RW) cp_async16(vec + V_BQKV + 4 * i, a.bqkv[l] + 4 * i);
+  for (int i = tid; i < NC_NH * nd / 4; i += NC_RW) cp_async16(s_dist + 4 * i, a.dist[l] + 4 * i);
+  if (tid < NC_NH / 4) cp_async16(s_same + 4 * tid, a.same[l] + 4 * tid);
+}
+__device__ void layer_vectors_finish(float* s_dist, float* s_same, int tid, int nd) {
+  cp_async_wait_all();
+  for (int i = tid; i < NC_NH * nd / 4; i += NC_RW)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) s_dist[4 * i + e] *= NC_LOG2E;
+  if (tid < NC_NH / 4)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) s_same[4 * tid + e] *= NC_LOG2E;
+}
+
 __global__ void __launch_bounds__(NC_THREADS, 1)
     net_cluster_kernel(const __grid_constant__ ClusterMaps maps, const __grid_constant__ ClusterArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -420,8 +476,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
   Shared sh;
   sh.base = sm;
   sh.full = reinterpret_cast<uint64_t*>(sm + OFF_BAR);
-  sh.empty = sh.full + NC_STAGES;
-  sh.done = sh.empty + NC_STAGES;
+  sh.empty = sh.full + NC_SLOTS;
+  sh.done = sh.empty + NC_SLOTS;
   sh.ready = sh.done + N_DONE;
   sh.xg = sh.ready + N_READY;
   sh.w1f = sh.xg + N_XG;
@@ -439,7 +495,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
   const int b = blockIdx.x / NC_CC;                  // the cluster's sequence
   const int nl = a.n_layers;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < NC_STAGES; ++s) {
+    for (int s = 0; s < NC_SLOTS; ++s) {
       mbar_init(&sh.full[s], 1);
       mbar_init(&sh.empty[s], 1);
     }
@@ -463,6 +519,29 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     mbar_expect_tx(&sh.xg[xb(nl)], XB_SS);
     mbar_expect_tx(&sh.xg[xb(nl) + 1], 2 * XB_SLICE);
   }
+  const int c0s = NC_SL * me;                        // first column of this CTA's slice
+  const int nd = 2 * a.L - 1;
+  if (warp >= 2) {
+    // weights only, before the wait on earlier launches: the confidence network
+    // (W_c1 transposed to [5][D]) and biases, the slice parts of b_c2, the final gain and
+    // the out / in head biases, the slot and rank tables, the first layer's vectors
+    const int tid = threadIdx.x - 64;
+    for (int i = tid; i < NC_D * LILICORR_N_CONF; i += NC_RW)
+      cp_async4(vec + V_C1W + (i % LILICORR_N_CONF) * NC_D + i / LILICORR_N_CONF, a.conf1_w + i);
+    for (int i = tid; i < NC_D / 4; i += NC_RW) cp_async16(vec + V_C1B + 4 * i, a.conf1_b + 4 * i);
+    for (int i = tid; i < NC_SL / 4; i += NC_RW) {
+      cp_async16(vec + V_C2B + 4 * i, a.conf2_b + c0s + 4 * i);
+      cp_async16(vec + V_FIN + 4 * i, a.final_norm + c0s + 4 * i);
+    }
+    for (int i = tid; i < 128 / 4; i += NC_RW) cp_async16(vec + V_BOI + 4 * i, a.boi + 128 * me + 4 * i);
+    for (int i = tid; i < (a.L + a.K) * (NC_SL / 4); i += NC_RW) {
+      const int row = a.L + i / (NC_SL / 4), c = (i % (NC_SL / 4)) * 4;
+      const float* src = row < 2 * a.L ? a.slot + (size_t)(row - a.L) * NC_D + c0s + c
+                                       : a.rank + (size_t)(row - 2 * a.L) * NC_D + c0s + c;
+      cp_async16(tab_at(sm, row, c), src);
+    }
+    layer_vectors_issue(a, 0, vec, s_dist, s_same, tid, c0s, nd);
+  }
   if (warp == 1) tmem_alloc(&tmem_base, NC_TMEM);
   tc_fence_before();
   cluster_sync();                  // every CTA's barriers exist before any peer signals them
@@ -475,14 +554,12 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      Producer p{&maps, sh, me, 0u};
+      Producer p{&maps, sh, me, 0u, 0u};
       schedule(a, p);
     }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      Issuer is{&a, sh, 0u, tmem};
-      schedule(a, is);
-    }
+  } else if (warp == 1) {       // the whole warp walks the schedule (warp-uniform
+    Issuer is{&a, sh, 0u, 0u, tmem};   // descriptors); one lane issues
+    schedule(a, is);
   } else {
     // ------------------------------------------------------------ row workers
     const int cg = (warp - 2) >> 2;
@@ -494,29 +571,16 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const uint32_t tx = tmem + lane_off + X_COL, tscr = tmem + lane_off + SCR_COL;
     const int L = a.L, K = a.K, LK = a.LK;
-    const int nd = 2 * L - 1;
     const int tid = threadIdx.x - 64;
-    const int c0s = NC_SL * me;                      // first column of this CTA's slice
     const bool ok = r < LK;
     Peers pe;
     pe.local = smem_u32(sm);
 #pragma unroll
     for (int qq = 1; qq < NC_CC; ++qq) pe.base[qq - 1] = peer_addr(pe.local, (uint32_t)((me + qq) % NC_CC));
-    // vectors: confidence-network weights (transposed to [5][D]) and biases, the slice
-    // parts of b_c2, the final gain, t and the out / in head biases
-    for (int i = tid; i < NC_D; i += NC_RW) {
-#pragma unroll
-      for (int j = 0; j < LILICORR_N_CONF; ++j)
-        vec[V_C1W + j * NC_D + i] = a.conf1_w[i * LILICORR_N_CONF + j];
-      vec[V_C1B + i] = a.conf1_b[i];
-      vec[V_CB + i] = a.cb[(size_t)b * NC_D + i];
-    }
-    for (int i = tid; i < NC_SL; i += NC_RW) {
-      vec[V_C2B + i] = a.conf2_b[c0s + i];
-      vec[V_FIN + i] = a.final_norm[c0s + i];
-      vec[V_T + i] = a.t[(size_t)b * NC_D + c0s + i];
-    }
-    for (int i = tid; i < 128; i += NC_RW) vec[V_BOI + i] = a.boi[128 * me + i];
+    // the sequence's vectors from earlier launches: the fusion layer's t block and t
+    for (int i = tid; i < NC_D / 4; i += NC_RW) cp_async16(vec + V_CB + 4 * i, a.cb + (size_t)b * NC_D + 4 * i);
+    for (int i = tid; i < NC_SL / 4; i += NC_RW)
+      cp_async16(vec + V_T + 4 * i, a.t + (size_t)b * NC_D + c0s + 4 * i);
 
     // ---- nodes: x[:, slice] = fold[id] + W_h h_s + b_h + slot[s] + rank[k] + b_c2, and
     //      c1 = SiLU(W_c1 f + b_c1) over all 256 columns (the conf2 operand)
@@ -542,20 +606,13 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       }
       // slice rows of the drafter state, slot and rank tables (ACT, 256-byte rows whose
       // 16-byte pieces are XOR-swizzled by row) and of the folded embedding (HF)
-      float* tab = reinterpret_cast<float*>(sm + OFF_ACT);
-      auto tab_at = [&](int row, int c) {            // c: a multiple of 4 below 64
-        return tab + (size_t)row * NC_SL + ((((c >> 2) ^ (row & 7))) << 2);
-      };
       float* fold_s = reinterpret_cast<float*>(sm + OFF_HF);
       auto fold_at = [&](int row, int c) {
         return fold_s + (size_t)row * NC_SL + ((((c >> 2) ^ (row & 7))) << 2);
       };
-      for (int i = tid; i < (2 * L + K) * (NC_SL / 4); i += NC_RW) {
+      for (int i = tid; i < L * (NC_SL / 4); i += NC_RW) {
         const int row = i / (NC_SL / 4), c = (i % (NC_SL / 4)) * 4;
-        const float* src = row < L ? a.hproj + ((size_t)b * L + row) * NC_D + c0s + c
-                         : row < 2 * L ? a.slot + (size_t)(row - L) * NC_D + c0s + c
-                                       : a.rank + (size_t)(row - 2 * L) * NC_D + c0s + c;
-        cp_async16(tab_at(row, c), src);
+        cp_async16(tab_at(sm, row, c), a.hproj + ((size_t)b * L + row) * NC_D + c0s + c);
       }
       rw_bar();                                      // s_ids complete
       for (int i = tid; i < LK * (NC_SL / 4); i += NC_RW) {
@@ -566,11 +623,11 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       rw_bar();
       for (int i = tid; i < L * (NC_SL / 4); i += NC_RW) {   // S[s] = hproj + slot + b_c2
         const int row = i / (NC_SL / 4), c = (i % (NC_SL / 4)) * 4;
-        float4 x = *reinterpret_cast<float4*>(tab_at(row, c));
-        const float4 y = *reinterpret_cast<const float4*>(tab_at(L + row, c));
+        float4 x = *reinterpret_cast<float4*>(tab_at(sm, row, c));
+        const float4 y = *reinterpret_cast<const float4*>(tab_at(sm, L + row, c));
         const float4 z = *reinterpret_cast<const float4*>(vec + V_C2B + c);
         x.x += y.x + z.x; x.y += y.y + z.y; x.z += y.z + z.z; x.w += y.w + z.w;
-        *reinterpret_cast<float4*>(tab_at(row, c)) = x;
+        *reinterpret_cast<float4*>(tab_at(sm, row, c)) = x;
       }
       rw_bar();
       {
@@ -580,8 +637,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         for (int u = 0; u < 4; ++u) {
           const int c = 16 * cg + 4 * u;
           const float4 x = *reinterpret_cast<const float4*>(fold_at(ok ? r : 0, c));
-          const float4 y = *reinterpret_cast<const float4*>(tab_at(srow, c));
-          const float4 z = *reinterpret_cast<const float4*>(tab_at(rrow, c));
+          const float4 y = *reinterpret_cast<const float4*>(tab_at(sm, srow, c));
+          const float4 z = *reinterpret_cast<const float4*>(tab_at(sm, rrow, c));
           v[4 * u] = ok ? x.x + y.x + z.x : 0.f;
           v[4 * u + 1] = ok ? x.y + y.y + z.y : 0.f;
           v[4 * u + 2] = ok ? x.z + y.z + z.z : 0.f;
@@ -623,17 +680,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     for (int l = 0; l < nl; ++l) {
       ev_wait(&sh.done[l == 0 ? 0 : D_LAYER(l - 1)], sh.abort);
       tc_fence_after();
-      rw_bar();                                      // the previous layer's vector readers
-      for (int i = tid; i < NC_SL; i += NC_RW) {
-        vec[V_AN + i] = a.an[l][c0s + i];
-        vec[V_FN + i] = a.fn[l][c0s + i];
-        vec[V_BO + i] = a.bo[l][c0s + i];
-        vec[V_B2 + (l & 1) * NC_SL + i] = a.b2[l][c0s + i];
-      }
-      for (int i = tid; i < NC_F; i += NC_RW) vec[V_B1 + i] = a.b1[l][i];
-      for (int i = tid; i < 3 * NC_D; i += NC_RW) vec[V_BQKV + i] = a.bqkv[l][i];
-      for (int i = tid; i < NC_NH * nd; i += NC_RW) s_dist[i] = a.dist[l][i] * NC_LOG2E;
-      if (tid < NC_NH) s_same[tid] = a.same[l][tid] * NC_LOG2E;
+      layer_vectors_finish(s_dist, s_same, tid, nd);   // issued a product earlier
       rw_bar();
       // x += b_2 of the previous layer; the row statistics, then (every CTA's W_2 is done)
       // x * g_attn (slice) everywhere
@@ -740,6 +787,9 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
             bulk_to_peer(pe.at(qq, src), src, 2 * CHUNK, pe.at(qq, &sh.xg[X_H(l)]));
           bulk_wait_read();
         }
+        // every reader of this layer's vectors is past the barrier: the next layer's
+        // vectors load while W_2 runs
+        if (l + 1 < nl) layer_vectors_issue(a, l + 1, vec, s_dist, s_same, tid, c0s, nd);
       }
       rw_signal(&sh.ready[R_H(l)], lane);
     }
