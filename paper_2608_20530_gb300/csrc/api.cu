@@ -318,8 +318,12 @@ lilicorr_status_t join_prologue(const lilicorr_head* h, cudaStream_t st) {
 
 // Candidate-dependent part, after the prologue: nodes, the Transformer, fusion and the
 // out/in heads. Writes oi = [W_o u + b_o | W_i u + b_i] (not yet normalised).
+// With `tail`, the cluster kernel also forms the pair scores and walks; *tail_done says
+// whether it did (otherwise the caller launches the pair kernel).
 lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* logp,
-                           cudaStream_t st) {
+                           cudaStream_t st, const ClusterTail* tail = nullptr,
+                           bool* tail_done = nullptr) {
+  if (tail_done) *tail_done = false;
   const lilicorr_head* h = c.h;
   const lilicorr_head_desc& d = c.d;
   const lilicorr_dtype_t F32 = LILICORR_F32, adt = c.adt;
@@ -330,8 +334,10 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   const bool cluster = h->cluster_maps &&
                        (g_fused_enabled == 3 ||
                         (g_fused_enabled == 1 && c.B <= net_cluster_capacity()));
-  if (cluster)
-    return launch_net_cluster(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
+  if (cluster) {
+    if (tail_done) *tail_done = tail != nullptr;
+    return launch_net_cluster(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st, tail);
+  }
   if (h->net_maps && (g_fused_enabled == 2 || (g_fused_enabled == 1 && c.B >= FUSED_MIN_B)))
     return launch_net_fused(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
@@ -784,7 +790,16 @@ lilicorr_status_t lilicorr_select_block_walk(const lilicorr_head* head, int B, c
                         at<void>(ws, w.partials), stream);
   LL_TRY(join_prologue(head, stream));                      // always rejoin, even on error
   LL_TRY(st);
-  LL_TRY(run_body(call, ids, logp, stream));
+  ClusterTail tail;
+  tail.anchor = at<float>(ws, w.anc);
+  tail.A = at<float>(ws, w.A);
+  tail.P = at<float>(ws, w.P);
+  tail.choice = at<int32_t>(ws, w.choice);
+  tail.tokens = tokens;
+  bool tail_done = false;
+  LL_TRY(run_body(call, ids, logp, stream, walk == LILICORR_WALK_GREEDY ? &tail : nullptr,
+                  &tail_done));
+  if (tail_done) return LILICORR_OK;
   PairWalkArgs a;
   memset(&a, 0, sizeof(a));
   a.B = B; a.L = d.L; a.K = d.K; a.d = d.d;

@@ -285,9 +285,19 @@ bool net_cluster_supported(const lilicorr_head_desc& d);
 void* net_cluster_maps_create(const lilicorr_head* h);
 void net_cluster_maps_free(void* p);
 int net_cluster_capacity();   // clusters that fit on the device at once
+// Steps (3) and (4) fused into the cluster kernel's tail: the anchor and pair scores
+// (written to A [B, K] and P [B, L-1, K, K]) and the greedy walk (choice, tokens [B, L]).
+struct ClusterTail {
+  const float* anchor;      // [B, d] anchor out vectors
+  float* A;
+  float* P;
+  int32_t* choice;
+  int32_t* tokens;
+};
 lilicorr_status_t launch_net_cluster(const lilicorr_head* h, int B, const int32_t* ids,
                                      const float* logp, const float* hproj, const float* t,
-                                     const float* cb, float* oi, uint32_t* status, cudaStream_t st);
+                                     const float* cb, float* oi, uint32_t* status, cudaStream_t st,
+                                     const ClusterTail* tail = nullptr);
 extern int g_fused_enabled;   // 0 never, 1 by batch size (default), 2 the one-CTA kernel
                               // always, 3 the cluster kernel always
 constexpr int FUSED_MIN_B = 8;

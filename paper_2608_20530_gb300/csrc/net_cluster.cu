@@ -34,6 +34,7 @@
 #include <new>
 
 #include "net_common.cuh"
+#include "walk.cuh"
 
 namespace lilicorr {
 
@@ -64,7 +65,7 @@ constexpr uint32_t OFF_HF = OFF_ACT + 4 * CHUNK;                   // 4 chunks
 constexpr uint32_t OFF_VEC = OFF_HF + 4 * CHUNK;
 constexpr int V_AN = 0, V_FN = 64, V_BO = 128, V_B2 = 192, V_FIN = 320, V_C2B = 384, V_T = 448,
               V_B1 = 512, V_BQKV = 1024, V_C1W = 1792, V_C1B = 3072, V_CB = 3328,
-              V_BOI = 3584, V_END = 3712;
+              V_BOI = 3584, V_ANC = 3712, V_END = 3776;
 constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [4][128] local partials
 // [2][4][128] the cluster's partials: [0] for the first RMSNorm of a layer and the final
 // one, [1] for the second (a peer can send the next statistics before this CTA has read
@@ -77,7 +78,7 @@ constexpr uint32_t OFF_IDS = OFF_SLOT + NC_M;                      // [128]
 constexpr uint32_t OFF_BAR = (OFF_IDS + NC_M * 4 + 63) & ~63u;
 constexpr int N_DONE = 2 + 4 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 2 + 6 * NC_MAX_LAYERS;
 constexpr int N_W1F = NC_MAX_LAYERS;
-constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_SLOTS + N_DONE + N_READY + N_XG + N_W1F) * 8;
+constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_SLOTS + N_DONE + N_READY + N_XG + N_W1F + 1) * 8;
 constexpr size_t NC_SMEM = 1024 + NC_SMEM_USED;
 static_assert(NC_SMEM <= 227 * 1024, "shared memory of the cluster network kernel");
 static_assert(OFF_ACT % 1024 == 0 && OFF_HF % 1024 == 0, "swizzle atoms");
@@ -139,6 +140,8 @@ struct ClusterArgs {
   const float* boi;
   float* oi;                // [B*LK, d2]
   uint32_t* status;
+  int tail;                 // the pair scores and the greedy walk in the kernel's tail
+  ClusterTail tl;
 };
 
 // K chunks and weight rows per chunk of each product slice
@@ -163,7 +166,11 @@ __device__ __forceinline__ void load_chunk(const ClusterMaps& m, int kind, int l
     case G_W1: tma_load_3d(dst, &m.w1[l], bar, 0, 128 * me, kc); break;
     case G_W2: tma_load_3d(dst, &m.w2[l], bar, 0, NC_SL * me, kc); break;
     case G_FUSE: tma_load_3d(dst, &m.fuse, bar, 0, 0, kc); break;
-    default: tma_load_3d(dst, &m.woi, bar, 0, 128 * me, kc); break;
+    default:   // out rows 64me.. and in rows d + 64me.. of [W_o; W_i]: both halves of
+               // this CTA's 64 columns of the out and in vectors
+      tma_load_3d(dst, &m.woi, bar, 0, NC_SL * me, kc);
+      tma_load_3d(static_cast<uint8_t*>(dst) + NC_SLOT, &m.woi, bar, 0, 4 * NC_SL + NC_SL * me, kc);
+      break;
   }
 }
 
@@ -182,7 +189,7 @@ __device__ __forceinline__ void schedule(const ClusterArgs& a, Op& op) {
 
 struct Shared {
   uint8_t* base;
-  uint64_t *full, *empty, *done, *ready, *xg, *w1f;
+  uint64_t *full, *empty, *done, *ready, *xg, *w1f, *prb;
   volatile int* abort;
 };
 
@@ -481,6 +488,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
   sh.ready = sh.done + N_DONE;
   sh.xg = sh.ready + N_READY;
   sh.w1f = sh.xg + N_XG;
+  sh.prb = sh.w1f + N_W1F;
   sh.abort = &abort_flag;
   float* s_ss = reinterpret_cast<float*>(sm + OFF_SS);
   float* s_ssx = reinterpret_cast<float*>(sm + OFF_SSX);
@@ -505,6 +513,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     }
     for (int e = 0; e < N_XG; ++e) mbar_init(&sh.xg[e], 1);
     for (int e = 0; e < N_W1F; ++e) mbar_init(&sh.w1f[e], NC_CC - 1);
+    mbar_init(sh.prb, NC_CC - 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // every exchange barrier: this CTA's own arrival now, the peers' bytes later
@@ -533,7 +542,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       cp_async16(vec + V_C2B + 4 * i, a.conf2_b + c0s + 4 * i);
       cp_async16(vec + V_FIN + 4 * i, a.final_norm + c0s + 4 * i);
     }
-    for (int i = tid; i < 128 / 4; i += NC_RW) cp_async16(vec + V_BOI + 4 * i, a.boi + 128 * me + 4 * i);
+    for (int i = tid; i < 2 * NC_SL / 4; i += NC_RW)     // out, then in biases of the slice
+      cp_async16(vec + V_BOI + 4 * i, a.boi + (i < NC_SL / 4 ? 0 : a.d2 / 2) + c0s + 4 * (i % (NC_SL / 4)));
     for (int i = tid; i < (a.L + a.K) * (NC_SL / 4); i += NC_RW) {
       const int row = a.L + i / (NC_SL / 4), c = (i % (NC_SL / 4)) * 4;
       const float* src = row < 2 * a.L ? a.slot + (size_t)(row - a.L) * NC_D + c0s + c
@@ -579,8 +589,10 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     for (int qq = 1; qq < NC_CC; ++qq) pe.base[qq - 1] = peer_addr(pe.local, (uint32_t)((me + qq) % NC_CC));
     // the sequence's vectors from earlier launches: the fusion layer's t block and t
     for (int i = tid; i < NC_D / 4; i += NC_RW) cp_async16(vec + V_CB + 4 * i, a.cb + (size_t)b * NC_D + 4 * i);
-    for (int i = tid; i < NC_SL / 4; i += NC_RW)
+    for (int i = tid; i < NC_SL / 4; i += NC_RW) {
       cp_async16(vec + V_T + 4 * i, a.t + (size_t)b * NC_D + c0s + 4 * i);
+      if (a.tail) cp_async16(vec + V_ANC + 4 * i, a.tl.anchor + (size_t)b * (a.d2 / 2) + c0s + 4 * i);
+    }
 
     // ---- nodes: x[:, slice] = fold[id] + W_h h_s + b_h + slot[s] + rank[k] + b_c2, and
     //      c1 = SiLU(W_c1 f + b_c1) over all 256 columns (the conf2 operand)
@@ -812,12 +824,17 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     tc_fence_after();
     drain_silu(sm + OFF_ACT, tscr, vec + V_CB, rsf, cg, r);
     rw_signal(&sh.ready[lb(nl) + 1], lane);
-    // ---- out / in heads: this CTA's 128 columns of [o | i] -> oi (fp32, not yet unit),
-    //      through a staging buffer (pieces swizzled by row) for row-contiguous stores
+    // ---- out / in heads: this CTA's 64 columns of the out and of the in vectors -> oi
+    //      (fp32, not yet unit) through a staging buffer (row r: 64 out then 64 in values,
+    //      16-byte pieces swizzled by row) for row-contiguous stores
     ev_wait(&sh.done[lb(nl) + 1], sh.abort);
     tc_fence_after();
     {
       uint8_t* stg = sm + OFF_HF;
+      auto stg_at = [&](int row, int piece) {
+        return reinterpret_cast<float4*>(stg + row * 512 + ((piece ^ (row & 7)) << 4));
+      };
+      float ss = 0.f;
 #pragma unroll 1
       for (int j = 0; j < 2; ++j) {
         const int cl = 32 * cg + 16 * j;            // column of the 128 staged
@@ -825,15 +842,96 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         ld16f(tscr + cl, v);
         const float* bo = vec + V_BOI + cl;
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          *reinterpret_cast<float4*>(stg + r * 512 + ((((cl >> 2) + u) ^ (r & 7)) << 4)) =
-              make_float4(v[4 * u] + bo[4 * u], v[4 * u + 1] + bo[4 * u + 1],
-                          v[4 * u + 2] + bo[4 * u + 2], v[4 * u + 3] + bo[4 * u + 3]);
+        for (int u = 0; u < 4; ++u) {
+          const float4 w = make_float4(v[4 * u] + bo[4 * u], v[4 * u + 1] + bo[4 * u + 1],
+                                       v[4 * u + 2] + bo[4 * u + 2], v[4 * u + 3] + bo[4 * u + 3]);
+          ss = fmaf(w.x, w.x, fmaf(w.y, w.y, fmaf(w.z, w.z, fmaf(w.w, w.w, ss))));
+          *stg_at(r, (cl >> 2) + u) = w;
+        }
       }
+      s_ss[cg * NC_M + r] = ss;                    // 32 columns' part of |o|^2 (cg < 2) or |i|^2
       rw_bar();
+      const int dh = a.d2 / 2;
       for (int row = wr; row < LK; row += NC_RW / 32)
-        *reinterpret_cast<float4*>(a.oi + ((size_t)b * LK + row) * a.d2 + 128 * me + 4 * lane) =
-            *reinterpret_cast<const float4*>(stg + row * 512 + ((lane ^ (row & 7)) << 4));
+        *reinterpret_cast<float4*>(a.oi + ((size_t)b * LK + row) * a.d2 + (lane < 16 ? 0 : dh) + c0s +
+                                   4 * (lane & 15)) = *stg_at(row, lane);
+      if (a.tail) {
+        // Steps (3), (4): the scores are cosines over all d columns (Eq. "pair"), so each
+        // CTA sums its 64 columns' part of every dot product and squared norm into a record
+        // in its (now idle) weight ring: pair dots [(L-1)][K][K] (out of slot s, in of
+        // slot s+1), anchor dots [K], |o|^2 [LK], |i|^2 [LK], |anchor|^2. The first CTA
+        // adds the peers' records (in rank order), forms the cosines and walks.
+        float* pr = reinterpret_cast<float*>(sm + OFF_RING);
+        const int npair = (L - 1) * K * K, o_ad = npair, o_on = o_ad + K, o_in = o_on + LK,
+                  o_an = o_in + LK, npr = o_an + 1;
+        for (int idx = tid; idx < npair; idx += NC_RW) {
+          const int s = idx / (K * K), j = (idx / K) % K, k = idx % K;
+          const int n1 = s * K + j, n2 = (s + 1) * K + k;
+          float dot = 0.f;
+#pragma unroll 4
+          for (int p = 0; p < 16; ++p) {
+            const float4 o = *stg_at(n1, p), i = *stg_at(n2, 16 + p);
+            dot = fmaf(o.x, i.x, fmaf(o.y, i.y, fmaf(o.z, i.z, fmaf(o.w, i.w, dot))));
+          }
+          pr[idx] = dot;
+        }
+        for (int k = tid; k < K; k += NC_RW) {
+          const float* an = vec + V_ANC;
+          float dot = 0.f;
+          for (int p = 0; p < 16; ++p) {
+            const float4 i = *stg_at(k, 16 + p);
+            dot = fmaf(an[4 * p], i.x, fmaf(an[4 * p + 1], i.y, fmaf(an[4 * p + 2], i.z, fmaf(an[4 * p + 3], i.w, dot))));
+          }
+          pr[o_ad + k] = dot;
+        }
+        if (cg == 0 && r < LK) {
+          pr[o_on + r] = s_ss[r] + s_ss[NC_M + r];
+          pr[o_in + r] = s_ss[2 * NC_M + r] + s_ss[3 * NC_M + r];
+        }
+        if (wr == 0) {
+          float q = 0.f;
+          for (int c = lane; c < NC_SL; c += 32) q = fmaf(vec[V_ANC + c], vec[V_ANC + c], q);
+          q = warp_sum(q);
+          if (lane == 0) pr[o_an] = q;
+        }
+        rw_bar();
+        if (me != 0) {
+          if (tid == 0) mbar_arrive_peer(pe.at(NC_CC - me, sh.prb));   // to rank 0
+        } else if (xg_wait(sh.prb, sh.abort)) {
+          for (int i = tid; i < npr; i += NC_RW) {
+            float v = pr[i];
+#pragma unroll
+            for (int q = 1; q < NC_CC; ++q) v += ld_peer_f32(pe.at(q, pr + i));
+            pr[i] = v;
+          }
+          rw_bar();
+          const float an = fmaxf(sqrtf(pr[o_an]), 1e-12f);
+          float* gP = a.tl.P + (size_t)b * npair;
+          for (int idx = tid; idx < npair; idx += NC_RW) {
+            const int s = idx / (K * K), j = (idx / K) % K, k = idx % K;
+            const float v = pr[idx] / (fmaxf(sqrtf(pr[o_on + s * K + j]), 1e-12f) *
+                                       fmaxf(sqrtf(pr[o_in + (s + 1) * K + k]), 1e-12f));
+            pr[idx] = v;
+            gP[idx] = v;
+          }
+          for (int k = tid; k < K; k += NC_RW) {
+            const float v = pr[o_ad + k] / (an * fmaxf(sqrtf(pr[o_in + k]), 1e-12f));
+            pr[o_ad + k] = v;
+            a.tl.A[(size_t)b * K + k] = v;
+          }
+          rw_bar();
+          if (wr == 0) {
+            walk::walk_sequence(pr + o_ad, pr, b, L, K, nullptr, s_slot);
+            __syncwarp();
+            for (int s = lane; s < L; s += 32) {
+              const size_t o = (size_t)b * L + s;
+              const int c = s_slot[s];
+              a.tl.choice[o] = c;
+              a.tl.tokens[o] = a.ids[o * K + c];
+            }
+          }
+        }
+      }
     }
   }
 
@@ -890,7 +988,7 @@ void* net_cluster_maps_create(const lilicorr_head* h) {
   memset(m, 0, sizeof(*m));
   bool ok = nc_chunk_map(&m->conf2, h->conf2_w, NC_D, NC_D, NC_SL) &&
             nc_chunk_map(&m->fuse, h->fuse_x, NC_D, 2 * NC_D, 256) &&
-            nc_chunk_map(&m->woi, h->woi, 2 * d.d, NC_D, 128);
+            nc_chunk_map(&m->woi, h->woi, 2 * d.d, NC_D, NC_SL);
   for (int l = 0; l < d.n_layers && ok; ++l) {
     const HeadW& w = h->layer[l];
     ok = nc_qkv_map(&m->wqkv[l], w.wqkv) && nc_chunk_map(&m->wo[l], w.wo, NC_D, NC_D, NC_SL) &&
@@ -944,7 +1042,8 @@ int net_cluster_capacity() {
 
 lilicorr_status_t launch_net_cluster(const lilicorr_head* h, int B, const int32_t* ids,
                                      const float* logp, const float* hproj, const float* t,
-                                     const float* cb, float* oi, uint32_t* status, cudaStream_t st) {
+                                     const float* cb, float* oi, uint32_t* status, cudaStream_t st,
+                                     const ClusterTail* tail) {
   if (B == 0) return LILICORR_OK;
   const ClusterMaps* m = static_cast<const ClusterMaps*>(h->cluster_maps);
   if (!m) return LILICORR_ERR_SHAPE;
@@ -966,6 +1065,10 @@ lilicorr_status_t launch_net_cluster(const lilicorr_head* h, int B, const int32_
   a.boi = h->boi;
   a.oi = oi;
   a.status = status;
+  if (tail) {
+    a.tail = 1;
+    a.tl = *tail;
+  }
   static bool configured[64] = {false};
   LL_TRY(allow_max_dynamic_smem(net_cluster_kernel, configured));
   cudaLaunchConfig_t cfg = {};

@@ -73,6 +73,12 @@ __device__ __forceinline__ void bulk_to_peer(uint32_t dst, const void* src, uint
 __device__ __forceinline__ void bulk_wait_read() {
   asm volatile("cp.async.bulk.commit_group;\n cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+// a float of a peer's shared memory (peer address)
+__device__ __forceinline__ float ld_peer_f32(uint32_t raddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(raddr) : "memory");
+  return v;
+}
 // one arrival on a peer's mbarrier (peer address), releasing this thread's prior writes
 __device__ __forceinline__ void mbar_arrive_peer(uint32_t rbar) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(rbar)
