@@ -261,13 +261,14 @@ __device__ __forceinline__ void st32f(uint32_t taddr, const float (&v)[32]) {
 
 // Attention core of one head (App. A: bidirectional attention over the L*K nodes with the
 // signed slot-distance and same-slot biases) for the 16 queries q0..q0+15 of one warp, in
-// blocks of 32 keys with an online softmax in log2 units; probabilities P = 2^(S - max) as
+// blocks of KB (32 or 64) keys with an online softmax in log2 units; probabilities P = 2^(S - max) as
 // fp16 pairs (one MUFU operation per pair). q, k (bf16) and v (fp16) of the head are at qb,
 // qb + 8192 and qb + 16384 (qkv_off layout). s_slot: slot of each node; sd: the head's
 // distance bias (log2 units) indexed by sj - si; same_l2: its same-slot bias (log2 units).
 // Out: the unnormalised outputs o[nb][e] in the mma m16n8 fragment layout (rows
 // q0 + lane/4 and q0 + lane/4 + 8, columns 8nb + 2(lane%4) + (e&1)) and the reciprocals of
 // the two rows' softmax sums.
+template <int KB = 64>
 __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const uint8_t* s_slot,
                                                const float* sd, float same_l2, int q0, int lane,
                                                float (&o)[4][4], float& inv0, float& inv1) {
@@ -285,14 +286,15 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
 #pragma unroll
   for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
 #pragma unroll 1
-  for (int kb0 = 0; kb0 < LK; kb0 += 32) {
-    float s4[4][4];
+  for (int kb0 = 0; kb0 < LK; kb0 += KB) {
+    constexpr int NB = KB / 8;                     // 8-key tiles of the block
+    float s4[NB][4];
 #pragma unroll
-    for (int nb = 0; nb < 4; ++nb) s4[nb][0] = s4[nb][1] = s4[nb][2] = s4[nb][3] = 0.f;
+    for (int nb = 0; nb < NB; ++nb) s4[nb][0] = s4[nb][1] = s4[nb][2] = s4[nb][3] = 0.f;
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
-      for (int nb = 0; nb < 4; nb += 2) {
+      for (int nb = 0; nb < NB; nb += 2) {
         uint32_t bf[4];
         const int key = kb0 + nb * 8 + (lane & 7) + ((lane >> 4) << 3);
         ldsm_x4(kb + qkv_off(key, ks * 2 + ((lane >> 3) & 1)), bf);
@@ -303,7 +305,7 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
     if (k8) {
       // K % 8 == 0: the 8 keys of a tile share one slot, so one bias per query row
 #pragma unroll
-      for (int nb = 0; nb < 4; ++nb) {
+      for (int nb = 0; nb < NB; ++nb) {
         const int jt = kb0 + nb * 8;
         const bool in = jt < LK;
         const int sj = s_slot[in ? jt : 0];
@@ -318,7 +320,7 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
       }
     } else {
 #pragma unroll
-      for (int nb = 0; nb < 4; ++nb) {
+      for (int nb = 0; nb < NB; ++nb) {
         const int j0 = kb0 + nb * 8 + 2 * t4;
         const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
 #pragma unroll
@@ -349,9 +351,9 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
       o[nb][0] *= c0; o[nb][1] *= c0;
       o[nb][2] *= c1; o[nb][3] *= c1;
     }
-    uint32_t pa[2][4];
+    uint32_t pa[NB / 2][4];
 #pragma unroll
-    for (int nb = 0; nb < 4; ++nb) {
+    for (int nb = 0; nb < NB; ++nb) {
       const uint32_t h01 = ex2_h2(pack_h2(s4[nb][0] - mn0, s4[nb][1] - mn0));
       const uint32_t h23 = ex2_h2(pack_h2(s4[nb][2] - mn1, s4[nb][3] - mn1));
       const float2 f01 = h2_to_f2(h01), f23 = h2_to_f2(h23);
@@ -367,7 +369,7 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
       }
     }
 #pragma unroll
-    for (int kk = 0; kk < 2; ++kk)
+    for (int kk = 0; kk < NB / 2; ++kk)
 #pragma unroll
       for (int nb = 0; nb < 4; nb += 2) {
         uint32_t vf[4];
