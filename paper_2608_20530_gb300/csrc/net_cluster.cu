@@ -713,8 +713,11 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       tc_fence_after();
       uint8_t* qs = sm + OFF_ACT + set * QKV_SET;
       const int hh = 2 * me + set;
-#pragma unroll 1
-      for (int part = (cg & 1) ? 2 : 0; part < ((cg & 1) ? 3 : 2); ++part) {
+      // the row's 96 values of the head split evenly over the two threads of the set:
+      // q and the first half of k, or the second half of k and v
+      const int odd = cg & 1;
+      {
+        const int part = odd ? 2 : 0;
         float v[32];
         ld32f(tscr + 64 * part + 32 * set, v);
         const float* bq = vec + V_BQKV + part * NC_D + hh * NC_HD;
@@ -726,6 +729,16 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         for (int p = 0; p < 4; ++p)
           *reinterpret_cast<uint4*>(dst + qkv_off(r, p)) =
               part == 2 ? pack8h(v + 8 * p) : pack8(v + 8 * p);
+      }
+      {
+        float v[16];
+        ld16f(tscr + 64 + 32 * set + 16 * odd, v);
+        const float* bq = vec + V_BQKV + NC_D + hh * NC_HD + 16 * odd;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] = fmaf(rs1, v[e], bq[e]);
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+          *reinterpret_cast<uint4*>(qs + 8192 + qkv_off(r, 2 * odd + p)) = pack8(v + 8 * p);
       }
       set_bar(set);
       {
