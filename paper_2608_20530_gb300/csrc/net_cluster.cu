@@ -1,32 +1,40 @@
 // Step (2), candidate-dependent part, on a thread-block cluster of four CTAs per sequence:
 // the node features, the two-layer scoring Transformer, the fusion layer and the out / in
-// heads (Sec. 3.2; App. A) for the bf16 head with D = 256, 8 heads, FFN 2D, L*K <= 128.
+// heads (Sec. 3.2; App. A) for the bf16 head with D = 256, 8 heads, FFN 2D, L*K <= 128;
+// optionally followed by steps (3) and (4) for the sequence (Eq. "pair", Sec. 3.5).
 //
 // The L*K nodes (zero-padded to 128) are the rows of every tensor-core tile, as in the
 // one-CTA kernel (net_fused.cu), but the columns are split over the cluster: CTA c of the
-// cluster owns columns 64c..64c+63 of the residual stream x (fp32, in its tensor memory)
-// and heads 2c, 2c+1. Each product computes only the CTA's output slice:
+// cluster owns columns 64c..64c+63 of the residual stream x (fp32, in its tensor memory),
+// heads 2c, 2c+1 and FFN hidden units 128c..128c+127. Each product computes only the CTA's
+// output slice:
 //   conf2, W_o, W_2     x[:, slice] += A W[slice, :]^T            (N = 64)
 //   q|k|v               the q, k, v rows of head pair c            (N = 192)
 //   W_1                 FFN hidden units 128c..128c+127            (N = 128)
-//   heads               [o | i][:, 128c..128c+127]                 (N = 128)
+//   heads               o[:, 64c..64c+63] and i[:, 64c..64c+63]    (N = 128)
 // while the fusion layer runs in full on every CTA (u is consumed locally by the heads).
 // The operands that need every CTA's slice are all-gathered through distributed shared
-// memory: each CTA writes its slice of RMSNorm(x) (before q|k|v and before W_1), of the
-// attention output (before W_o), of the FFN hidden state (before W_2; it fills both
-// operand buffers) and of the fusion input [xf | xf*t] into the same place
-// in all four CTAs' operand buffers with st.async, whose bytes complete the transaction
-// count of the receiving CTA's mbarrier for that exchange; the receiving MMA thread waits
-// on it (acquire, cluster scope). RMSNorm statistics travel the same way: each CTA sends
-// the per-row sums of squares of its 64 columns.
-// Buffer reuse needs no extra hand-shake: a CTA can only produce the next payload for a
-// buffer after an exchange that needs every CTA's contribution, which each CTA makes only
-// once its own readers of that buffer are done (e.g. W_1's input lands in ACT after the
-// second RMSNorm exchange, which needs the sender's W_o output, which needs this CTA's
-// attention output, written after this CTA's attention finished reading q, k, v in ACT).
+// memory: each CTA writes its slice of the RMSNorm operand (before q|k|v and before W_1),
+// of the attention output (before W_o), of the FFN hidden state (before W_2) and of the
+// fusion input [xf | xf*t] into its own operand buffer, and one thread copies those bytes
+// into the same place in the three peers with one bulk shared::cluster copy each, which
+// completes the receiving CTA's mbarrier for that exchange; the receiving MMA lane waits
+// on it (acquire, cluster scope). RMSNorm statistics (per-row sums of squares of each
+// CTA's 64 columns) travel as st.async words to the same kind of barrier.
+// Buffer reuse is ordered by the exchanges themselves: a CTA produces the next payload for
+// a buffer only after an exchange that needs every CTA's contribution, which each CTA
+// makes only once its own readers of that buffer are done (e.g. W_1's input lands in ACT
+// after the second RMSNorm exchange, which needs the sender's W_o output, which needs this
+// CTA's attention output, written after its attention finished reading q, k, v in ACT).
+// The one exception, the hidden state that overwrites the peers' W_1 operand, waits for a
+// word from every peer that its W_1 product is done (w1f).
+// With the tail enabled, each CTA sums its 64 columns' part of every pair dot product and
+// squared norm; the first CTA adds the peers' records (read across the cluster, in rank
+// order), forms the cosine scores and runs the greedy walk.
 //
-// Roles (576 threads): warp 0 lane 0 streams the weight slices by TMA through a two-stage
-// ring, warp 1 allocates tensor memory and lane 0 issues tcgen05.mma, warps 2-17 are row
+// Roles (576 threads): warp 0 lane 0 streams the weight slices by TMA through a ring of
+// eight 8 KB slots, warp 1 allocates tensor memory and walks the product schedule (lane 0
+// issues tcgen05.mma), warps 2-17 are row
 // workers (thread = row r = 32 (warp % 4) + lane and column group cg = (warp - 2) / 4:
 // 16 columns of the x slice, or 64 columns of a full-width drain). Every mbarrier wait is
 // bounded (about 2 s); on timeout the CTA records LILICORR_ERR_TIMEOUT, stops issuing and
@@ -269,7 +277,7 @@ struct Issuer {
     if (xw >= 0) xg_wait(&sh.xg[xw], sh.abort);
     __syncwarp();
     tc_fence_after();
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // peers' st.async data
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // peers' copied data
     const int nk = n_chunks(kind), ns = tile_rows(kind) / 64;
     const bool onto_x = kind == G_CONF2 || kind == G_WO || kind == G_W2;
     const uint32_t d = tmem + (onto_x ? X_COL : SCR_COL);
