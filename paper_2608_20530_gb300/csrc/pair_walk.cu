@@ -29,6 +29,26 @@ namespace {
 using namespace walk;
 
 constexpr int PW_THREADS = 256;
+
+// Asynchronous global -> shared copies: every thread issues all of its copies before
+// any wait, so a staging loop costs one memory latency rather than one per iteration.
+__device__ __forceinline__ void cp16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
+               ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;"
+               ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_wait_all() {
+  asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
+}
+// The sequence's scores A [K] then P [(L-1) K K] into shared memory (caller syncs).
+__device__ __forceinline__ void stage_scores(float* sm, const float* gA, const float* gP, int K,
+                                             int n_scores) {
+  for (int i = threadIdx.x; i < n_scores; i += PW_THREADS) cp4(sm + i, i < K ? gA + i : gP + (i - K));
+  cp_wait_all();
+}
 constexpr float UNIT_EPS = 1e-12f;
 constexpr size_t PW_SMEM_MAX = 200 * 1024;     // dynamic shared memory the launcher may ask for
 
@@ -112,10 +132,11 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
                   (reinterpret_cast<uintptr_t>(a.anchor) & 15) == 0;
   if (v4) {
     const int dv = d >> 2;
-    for (int k = 0; k < K; ++k)
-      for (int c = threadIdx.x; c < dv; c += PW_THREADS)
-        reinterpret_cast<float4*>(s_in + (size_t)k * d)[c] =
-            __ldcg(reinterpret_cast<const float4*>(inb + (size_t)k * a.ld_vec) + c);
+    for (int i = threadIdx.x; i < K * dv; i += PW_THREADS) {
+      const int k = i / dv, c = i - k * dv;
+      cp16(s_in + (size_t)k * d + 4 * c, inb + (size_t)k * a.ld_vec + 4 * c);
+    }
+    cp_wait_all();
   } else {
     for (int i = threadIdx.x; i < K * d; i += PW_THREADS) {
       const int k = i / d, c = i % d;
@@ -213,8 +234,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
   const float* A = gA;
   const float* P = gP;
   if (a.scores_in_smem) {                       // reuse the staging buffer for the scores
-    for (int i = threadIdx.x; i < n_scores; i += PW_THREADS)
-      sm[i] = i < K ? __ldcg(gA + i) : __ldcg(gP + (i - K));
+    stage_scores(sm, gA, gP, K, n_scores);
     __syncthreads();
     A = sm;
     P = sm + K;
@@ -235,7 +255,7 @@ __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
   const float* A = a.A + (size_t)b * K;
   const float* P = a.P + (size_t)b * (L - 1) * K * K;
   if (a.scores_in_smem) {
-    for (int i = threadIdx.x; i < n_scores; i += PW_THREADS) sm[i] = i < K ? A[i] : P[i - K];
+    stage_scores(sm, A, P, K, n_scores);
     __syncthreads();
     A = sm;
     P = sm + K;
