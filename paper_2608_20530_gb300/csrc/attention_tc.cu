@@ -44,6 +44,10 @@ __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], 
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+__device__ __forceinline__ void cp_async_16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
+               ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src) : "memory");
+}
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&v);
@@ -78,26 +82,26 @@ attention_mma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D,
   const size_t ld = 3 * (size_t)D;
   const __nv_bfloat16* base = qkv + (size_t)b * LK * ld + (size_t)h * HD;
 
-  // ---- stage K, V (all keys, zero rows past LK) and this CTA's queries
+  // ---- stage K, V (all keys, zero rows past LK) and this CTA's queries: asynchronous
+  // copies, all issued before one wait
   constexpr int RV = HD / 8;                 // 16-byte vectors per row
   const uint4 zero = make_uint4(0, 0, 0, 0);
-#pragma unroll 4
   for (int i = threadIdx.x; i < LKp * RV; i += AT_WARPS * 32) {
     const int j = i / RV, c = (i % RV) * 8;
-    uint4 kv = zero, vv = zero;
     if (j < LK) {
-      kv = *reinterpret_cast<const uint4*>(base + (size_t)j * ld + D + c);
-      vv = *reinterpret_cast<const uint4*>(base + (size_t)j * ld + 2 * D + c);
+      cp_async_16(Ks + (size_t)j * HP + c, base + (size_t)j * ld + D + c);
+      cp_async_16(Vs + (size_t)j * HP + c, base + (size_t)j * ld + 2 * D + c);
+    } else {
+      *reinterpret_cast<uint4*>(Ks + (size_t)j * HP + c) = zero;
+      *reinterpret_cast<uint4*>(Vs + (size_t)j * HP + c) = zero;
     }
-    *reinterpret_cast<uint4*>(Ks + (size_t)j * HP + c) = kv;
-    *reinterpret_cast<uint4*>(Vs + (size_t)j * HP + c) = vv;
   }
   for (int i = threadIdx.x; i < AT_QROWS * RV; i += AT_WARPS * 32) {
     const int j = i / RV, c = (i % RV) * 8;
-    uint4 qv = zero;
-    if (q0 + j < LK) qv = *reinterpret_cast<const uint4*>(base + (size_t)(q0 + j) * ld + c);
-    *reinterpret_cast<uint4*>(Qs + (size_t)j * HP + c) = qv;
+    if (q0 + j < LK) cp_async_16(Qs + (size_t)j * HP + c, base + (size_t)(q0 + j) * ld + c);
+    else *reinterpret_cast<uint4*>(Qs + (size_t)j * HP + c) = zero;
   }
+  asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
   for (int i = threadIdx.x; i < 2 * L - 1; i += AT_WARPS * 32)
     s_dist[i] = dist[(size_t)h * (2 * L - 1) + i] * LOG2E;
   const bool k8 = (K & 7) == 0;
