@@ -37,6 +37,7 @@ constexpr int TK_WARPS = TK_THREADS / 32;
 constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch
 constexpr int TK_MAX_SPLITS = 64;
 constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
+constexpr int TK_FEW_ROW_CTAS = 256;   // CTAs over all rows when rows are few
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr unsigned FULL = 0xffffffffu;
 
@@ -590,12 +591,13 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
 TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   const int vec = dt == LILICORR_BF16 ? 8 : 4;
   const int nvec = V / vec;
-  // Few rows: split each over CTAs until the resident slots (4 CTAs per SM) are covered.
-  // Once the rows alone fill half of the slots, one CTA per row: every split adds a
-  // partial record and a merge, which costs more than the imbalance it removes.
+  // Few rows: split each over about 256 CTAs in all (a sweep over 16-256 rows of a
+  // 151,936-wide vocabulary put the optimum at 192-256 CTAs: more pieces add partial
+  // records and merge work faster than they shorten the stream). Once the rows alone
+  // fill half of the resident slots (4 CTAs per SM), one CTA per row.
   const int slots = num_sms() * 4;
   const int min_chunk = 256;                 // vectors (4 KB) per CTA at least
-  int splits = rows * 2 >= slots ? 1 : ceil_div(slots, rows);
+  int splits = rows * 2 >= slots ? 1 : ceil_div(TK_FEW_ROW_CTAS, rows);
   splits = max(1, min(splits, ceil_div(max(nvec, 1), min_chunk)));
   splits = min(splits, min(TK_MAX_SPLITS, TK_MERGE_MAX / K));
   TopkPlan p;
