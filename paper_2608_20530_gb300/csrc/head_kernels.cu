@@ -112,17 +112,17 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
   }
 }
 
-template <typename TA, typename TW, typename TC>
+template <typename TA, typename TW, typename TC, int MB>
 __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
   pdl_wait();
-  __shared__ float red[SK_THREADS / 32][SK_MB * SK_NB];
+  __shared__ float red[SK_THREADS / 32][MB * SK_NB];
   const TA* A = static_cast<const TA*>(g.A);
   const TW* W = static_cast<const TW*>(g.W);
-  const int n0 = blockIdx.x * SK_NB, m0 = blockIdx.y * SK_MB;
-  const int nb = min(SK_NB, g.N - n0), mb = min(SK_MB, g.M - m0);
-  float acc[SK_MB][SK_NB];
+  const int n0 = blockIdx.x * SK_NB, m0 = blockIdx.y * MB;
+  const int nb = min(SK_NB, g.N - n0), mb = min(MB, g.M - m0);
+  float acc[MB][SK_NB];
 #pragma unroll
-  for (int i = 0; i < SK_MB; ++i)
+  for (int i = 0; i < MB; ++i)
 #pragma unroll
     for (int j = 0; j < SK_NB; ++j) acc[i][j] = 0.f;
   for (int k = threadIdx.x * 8; k < g.Kd; k += SK_THREADS * 8) {
@@ -135,16 +135,16 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
         for (int e = 0; e < 8; ++e) w[j][e] = 0.f;
     }
     // all row loads first (predicated, no early exit) so they are in flight together
-    float a[SK_MB][8];
+    float a[MB][8];
 #pragma unroll
-    for (int i = 0; i < SK_MB; ++i) {
+    for (int i = 0; i < MB; ++i) {
       if (i < mb) load8(A + (size_t)(m0 + i) * g.lda + k, a[i]);
       else
 #pragma unroll
         for (int e = 0; e < 8; ++e) a[i][e] = 0.f;
     }
 #pragma unroll
-    for (int i = 0; i < SK_MB; ++i)
+    for (int i = 0; i < MB; ++i)
 #pragma unroll
       for (int j = 0; j < SK_NB; ++j)
 #pragma unroll
@@ -152,14 +152,16 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 #pragma unroll
-  for (int i = 0; i < SK_MB; ++i)
+  for (int i = 0; i < MB; ++i) {
+    if (i >= mb) break;                            // rows past M: nothing to reduce
 #pragma unroll
     for (int j = 0; j < SK_NB; ++j) {
       const float v = warp_sum(acc[i][j]);
       if (lane == 0) red[warp][i * SK_NB + j] = v;
     }
+  }
   __syncthreads();
-  if (threadIdx.x < SK_MB * SK_NB) {
+  if (threadIdx.x < MB * SK_NB) {
     const int i = threadIdx.x / SK_NB, j = threadIdx.x % SK_NB;
     if (i < mb && j < nb) {
       float v = 0.f;
@@ -175,11 +177,20 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
   }
 }
 
+template <typename TA, typename TW, int MB>
+lilicorr_status_t skinny_dispatch_m(const GemmArgs& g, cudaStream_t st) {
+  dim3 grid(ceil_div(g.N, SK_NB), ceil_div(g.M, MB));
+  if (g.c_dt == LILICORR_F32) LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, float, MB>, grid, SK_THREADS, 0, st, g));
+  else LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, __nv_bfloat16, MB>, grid, SK_THREADS, 0, st, g));
+  return LILICORR_OK;
+}
+// rows per CTA: one per sequence-level row (M = 1), four for a few, else sixteen
 template <typename TA, typename TW>
 lilicorr_status_t skinny_dispatch_c(const GemmArgs& g, dim3 grid, cudaStream_t st) {
-  if (g.c_dt == LILICORR_F32) LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, float>, grid, SK_THREADS, 0, st, g));
-  else LL_TRY(launch_k(gemm_skinny_kernel<TA, TW, __nv_bfloat16>, grid, SK_THREADS, 0, st, g));
-  return LILICORR_OK;
+  (void)grid;
+  if (g.M == 1) return skinny_dispatch_m<TA, TW, 1>(g, st);
+  if (g.M <= 4) return skinny_dispatch_m<TA, TW, 4>(g, st);
+  return skinny_dispatch_m<TA, TW, SK_MB>(g, st);
 }
 template <typename TA>
 lilicorr_status_t skinny_dispatch_w(const GemmArgs& g, dim3 grid, cudaStream_t st) {
