@@ -28,13 +28,22 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
                                        const float* bias, const float* residual, int act, int path,
                                        uint32_t* status, cudaStream_t stream);
 
-/* Switch for the fused scoring-network kernel (one CTA per sequence; bf16 heads with
- * D = 256, 8 heads, FFN 2D, L*K <= 128 and 2L + K <= 64). mode 1 (the default) uses
- * it for calls of 8 or more sequences, mode 2 for every call, mode 0 never, so a test
- * can run both paths on the same inputs. Process-wide; set it between calls, not
+/* Switch for the fused scoring-network kernels (bf16 heads with D = 256, 8 heads,
+ * FFN 2D, L*K <= 128): mode 1 (the default) takes the cluster kernel (four CTAs per
+ * sequence) while every sequence's cluster fits on the GPU and the one-CTA kernel for
+ * calls of 8 or more sequences beyond that, mode 2 the one-CTA kernel for every call,
+ * mode 3 the cluster kernel for every call, mode 0 neither (the chain of kernels), so a
+ * test can run the paths on the same inputs. Process-wide; set it between calls, not
  * while another thread is enqueueing. Returns 1 if `head` (may be NULL) can take the
- * fused kernel, else 0. */
+ * kernel that `mode` names, else 0. */
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode);
+
+/* Switch for the chain's attention core (Sec. 3.2 and App. A: bidirectional attention
+ * with the slot-distance and same-slot biases, bf16 heads): mode 1 runs it on the
+ * tcgen05 tensor cores where the head width is 32 or 64 and a sequence has at most 256
+ * nodes, mode 0 (the default: the faster of the two so far) on the mma.sync kernel.
+ * Process-wide, like the switch above. Returns the previous mode. */
+int lilicorr_test_attention_path(int mode);
 
 #ifdef __cplusplus
 }

@@ -1,7 +1,7 @@
 """GPU check of the scoring network's linear-layer kernels (building blocks of step 2)
 against a plain PyTorch fp32 matmul of the same bf16/fp32 operands: the tensor-core
 (tcgen05) kernels (tiled, and one tile of rows with whole-K copies), the tiled and the
-few-row CUDA-core kernels, with bias, SiLU,
+few-row CUDA-core kernels (one, four or sixteen rows per CTA), with bias, SiLU,
 residual, bf16 output, ragged M/N and long Kd."""
 import pytest
 import torch
@@ -30,7 +30,7 @@ def _ref(A, W, bias, residual, act):
 CASES = [  # M, N, Kd
     (128, 256, 256), (128, 64, 64), (300, 768, 256), (129, 64, 4096), (512, 512, 4096),
     (256, 1536, 512), (1000, 200, 512), (4096, 512, 512), (16, 256, 4096), (1, 256, 256),
-    (64, 1024, 2048),
+    (64, 1024, 2048), (3, 264, 4096), (4, 256, 512), (5, 104, 256), (1, 8, 4096),
 ]
 
 
