@@ -100,11 +100,20 @@ attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D
     if (p < HD / 8 && j < LK) cp16(dst, base + (size_t)j * ld + D + 8 * p);
     else *reinterpret_cast<uint4*>(dst) = zero;
   }
-  for (int i = tid; i < LKp * (HD / 8); i += UA_THREADS) {
-    const int j = i / (HD / 8), p = i % (HD / 8);
-    const uint4 v = j < LK ? *reinterpret_cast<const uint4*>(base + (size_t)j * ld + 2 * D + 8 * p)
-                           : zero;
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  // V: every load of this thread first (up to UA_MAX_KEYS * 8 / UA_THREADS = 8), then the
+  // transposing stores, so the loads are in flight together
+  constexpr int VN = UA_MAX_KEYS * (HD / 8) / UA_THREADS;
+  uint4 vv[VN];
+#pragma unroll
+  for (int u = 0; u < VN; ++u) {
+    const int i = tid + u * UA_THREADS, j = i / (HD / 8), p = i % (HD / 8);
+    vv[u] = j < LK ? *reinterpret_cast<const uint4*>(base + (size_t)j * ld + 2 * D + 8 * p) : zero;
+  }
+#pragma unroll
+  for (int u = 0; u < VN; ++u) {
+    const int i = tid + u * UA_THREADS, j = i / (HD / 8), p = i % (HD / 8);
+    if (j >= LKp) continue;
+    const uint32_t w[4] = {vv[u].x, vv[u].y, vv[u].z, vv[u].w};
     uint8_t* chunk = sV + (size_t)(j >> 6) * HD * 128;
     const int kp = (j & 63) >> 3, ko = (j & 7) * 2;
 #pragma unroll
