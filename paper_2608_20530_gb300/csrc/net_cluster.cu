@@ -84,7 +84,8 @@ constexpr uint32_t OFF_SAME = OFF_DIST + NC_NH * (2 * NC_MAX_L - 1) * 4;
 constexpr uint32_t OFF_SLOT = OFF_SAME + NC_NH * 4;                // [128]
 constexpr uint32_t OFF_IDS = OFF_SLOT + NC_M;                      // [128]
 constexpr uint32_t OFF_BAR = (OFF_IDS + NC_M * 4 + 63) & ~63u;
-constexpr int N_DONE = 2 + 4 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 2 + 6 * NC_MAX_LAYERS;
+constexpr int N_DONE = 2 + 4 * NC_MAX_LAYERS + 1, N_READY = N_DONE, N_XG = 3 + 6 * NC_MAX_LAYERS;
+constexpr int X_C1 = N_XG - 1;            // exchange of the confidence MLP's first layer
 constexpr int N_W1F = NC_MAX_LAYERS;
 constexpr uint32_t NC_SMEM_USED = OFF_BAR + (2 * NC_SLOTS + N_DONE + N_READY + N_XG + N_W1F + 1) * 8;
 constexpr size_t NC_SMEM = 1024 + NC_SMEM_USED;
@@ -264,7 +265,7 @@ struct Issuer {
     // peers' slices
     int rd = -1, xw = -1, dn = -1;
     switch (kind) {
-      case G_CONF2: rd = 0; dn = 0; break;
+      case G_CONF2: rd = 0; xw = X_C1; dn = 0; break;
       case G_QKV: rd = R_XN(l); xw = X_XN(l); dn = D_QKV(l); break;
       case G_WO: rd = R_ATT(l); xw = X_ATT(l); dn = D_WO(l); break;
       case G_W1: rd = R_XN2(l); xw = X_XN2(l); dn = D_W1(l); break;
@@ -448,10 +449,11 @@ __device__ void drain_silu(uint8_t* buf, uint32_t tscr, const float* bias, float
   }
 }
 
-// The drafter-state, slot and rank table rows of this CTA's slice in ACT: 256-byte rows
+// The drafter-state, slot and rank table rows of this CTA's slice in HF chunks 2-3: 256-byte rows
 // (64 fp32) whose 16-byte pieces are XOR-swizzled by row; c is a multiple of 4 below 64.
 __device__ __forceinline__ float* tab_at(uint8_t* sm, int row, int c) {
-  return reinterpret_cast<float*>(sm + OFF_ACT) + (size_t)row * NC_SL + ((((c >> 2) ^ (row & 7))) << 2);
+  return reinterpret_cast<float*>(sm + OFF_HF + 2 * CHUNK) + (size_t)row * NC_SL +
+         ((((c >> 2) ^ (row & 7))) << 2);
 }
 
 // Layer l's vectors (this CTA's slices of the norm gains, b_o and b_2; b_1, the q|k|v
@@ -535,6 +537,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
     }
     mbar_expect_tx(&sh.xg[xb(nl)], XB_SS);
     mbar_expect_tx(&sh.xg[xb(nl) + 1], 2 * XB_SLICE);
+    mbar_expect_tx(&sh.xg[X_C1], XB_SLICE);
   }
   const int c0s = NC_SL * me;                        // first column of this CTA's slice
   const int nd = 2 * a.L - 1;
@@ -624,7 +627,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         f[3] = K > 1 ? (float)k / (float)(K - 1) : 0.f;
         f[4] = k == 0 ? 1.f : 0.f;
       }
-      // slice rows of the drafter state, slot and rank tables (ACT, 256-byte rows whose
+      // slice rows of the drafter state, slot and rank tables (HF chunks 2-3, 256-byte rows whose
       // 16-byte pieces are XOR-swizzled by row) and of the folded embedding (HF)
       float* fold_s = reinterpret_cast<float*>(sm + OFF_HF);
       auto fold_at = [&](int row, int c) {
@@ -666,13 +669,13 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         }
         st16f(tx + 16 * cg, v);
       }
-      rw_bar();                                      // ACT (the tables) free for c1
-#pragma unroll 1
-      for (int j = 0; j < 2; ++j) {
-        const int c0 = 64 * cg + 32 * j;
-        float c1[32];
+      // c1 for this CTA's 64 columns (16 per thread) into chunk me of ACT, then to the
+      // peers (the W_c2 operand needs all 256)
+      {
+        const int c0 = NC_SL * me + 16 * cg;
+        float c1[16];
 #pragma unroll
-        for (int e = 0; e < 32; e += 4) {
+        for (int e = 0; e < 16; e += 4) {
           float4 z = *reinterpret_cast<const float4*>(vec + V_C1B + c0 + e);
 #pragma unroll
           for (int i = 0; i < LILICORR_N_CONF; ++i) {
@@ -689,7 +692,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
           c1[e + 2] = ok ? z.z : 0.f;
           c1[e + 3] = ok ? z.w : 0.f;
         }
-        put32(sm + OFF_ACT, r, c0, c1);
+        put16(sm + OFF_ACT, me, r, cg, c1);
+        send_all(sm + OFF_ACT + (size_t)me * CHUNK, CHUNK, &sh.xg[X_C1], tid, pe);
       }
       tmem_wait_st();
       if (cg == 0) s_slot[r] = (uint8_t)min(r / K, L - 1);   // read after the next rw_bar
@@ -997,7 +1001,7 @@ bool nc_qkv_map(CUtensorMap* m, const void* W) {
 bool net_cluster_supported(const lilicorr_head_desc& d) {
   return d.dtype == LILICORR_BF16 && d.D == NC_D && d.ffn == NC_F && d.n_heads == NC_NH &&
          d.n_layers >= 1 && d.n_layers <= NC_MAX_LAYERS && d.L >= 1 && d.L <= NC_MAX_L &&
-         d.K >= 1 && d.L * d.K <= NC_M && (2 * d.L + d.K) * NC_SL * 4 <= 4 * (int)CHUNK &&
+         d.K >= 1 && d.L * d.K <= NC_M && (2 * d.L + d.K) * NC_SL * 4 <= 2 * (int)CHUNK &&
          2 * d.d == NC_CC * 128 && encode_fn() != nullptr;
 }
 
