@@ -73,7 +73,7 @@ constexpr uint32_t OFF_HF = OFF_ACT + 4 * CHUNK;                   // 4 chunks
 constexpr uint32_t OFF_VEC = OFF_HF + 4 * CHUNK;
 constexpr int V_AN = 0, V_FN = 64, V_BO = 128, V_B2 = 192, V_FIN = 320, V_C2B = 384, V_T = 448,
               V_B1 = 512, V_BQKV = 1024, V_C1W = 1792, V_C1B = 3072, V_CB = 3328,
-              V_BOI = 3584, V_ANC = 3712, V_END = 3776;
+              V_BOI = 3584, V_ANC = 3712, V_TF = 3776, V_END = 4032;
 constexpr uint32_t OFF_SS = OFF_VEC + V_END * 4;                   // [4][128] local partials
 // [2][4][128] the cluster's partials: [0] for the first RMSNorm of a layer and the final
 // one, [1] for the second (a peer can send the next statistics before this CTA has read
@@ -536,7 +536,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       mbar_expect_tx(&sh.xg[X_H(l)], XB_H);
     }
     mbar_expect_tx(&sh.xg[xb(nl)], XB_SS);
-    mbar_expect_tx(&sh.xg[xb(nl) + 1], 2 * XB_SLICE);
+    mbar_expect_tx(&sh.xg[xb(nl) + 1], XB_SLICE);
     mbar_expect_tx(&sh.xg[X_C1], XB_SLICE);
   }
   const int c0s = NC_SL * me;                        // first column of this CTA's slice
@@ -604,6 +604,8 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       cp_async16(vec + V_T + 4 * i, a.t + (size_t)b * NC_D + c0s + 4 * i);
       if (a.tail) cp_async16(vec + V_ANC + 4 * i, a.tl.anchor + (size_t)b * (a.d2 / 2) + c0s + 4 * i);
     }
+    for (int i = tid; i < NC_D / 4; i += NC_RW)          // all of t (the x*t block)
+      cp_async16(vec + V_TF + 4 * i, a.t + (size_t)b * NC_D + 4 * i);
 
     // ---- nodes: x[:, slice] = fold[id] + W_h h_s + b_h + slot[s] + rank[k] + b_c2, and
     //      c1 = SiLU(W_c1 f + b_c1) over all 256 columns (the conf2 operand)
@@ -841,8 +843,34 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
       norm_stats(tx, vec + V_B2 + ((nl - 1) & 1) * NC_SL, false, cg, r, me, s_ss, s_ssx,
                  &sh.xg[xb(nl)], pe, v);
       rsf = norm_recv(r, s_ssx, &sh.xg[xb(nl)], sh.abort);
-      norm_operand(v, vec + V_FIN, sm + OFF_ACT, vec + V_T, sm + OFF_HF, &sh.xg[xb(nl) + 1], cg, r,
-                   me, tid, pe);
+      // xf here and in the peers (ACT); xf * t of this CTA's slice into HF here
+      float vt[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) vt[e] = v[e] * vec[V_FIN + 16 * cg + e] * vec[V_T + 16 * cg + e];
+      put16(sm + OFF_HF, me, r, cg, vt);
+      norm_operand(v, vec + V_FIN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[xb(nl) + 1], cg, r, me,
+                   tid, pe);
+    }
+    // xf * t of the peers' slices from their xf, once it is here (one exchange instead of
+    // two): 16 columns of each peer chunk per thread
+    xg_wait(&sh.xg[xb(nl) + 1], sh.abort);
+#pragma unroll 1
+    for (int qq = 1; qq < NC_CC; ++qq) {
+      const int q = (me + qq) % NC_CC;
+#pragma unroll
+      for (int p = 0; p < 2; ++p) {
+        const uint32_t off = (uint32_t)q * CHUNK + swz(r, 2 * cg + p);
+        const uint4 w = *reinterpret_cast<const uint4*>(sm + OFF_ACT + off);
+        const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+        const float* tq = vec + V_TF + NC_SL * q + 16 * cg + 8 * p;
+        float x8[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          x8[2 * e] = __uint_as_float(wv[e] << 16) * tq[2 * e];
+          x8[2 * e + 1] = __uint_as_float(wv[e] & 0xFFFF0000u) * tq[2 * e + 1];
+        }
+        *reinterpret_cast<uint4*>(sm + OFF_HF + off) = pack8(x8);
+      }
     }
     rw_signal(&sh.ready[lb(nl)], lane);
     ev_wait(&sh.done[lb(nl)], sh.abort);
