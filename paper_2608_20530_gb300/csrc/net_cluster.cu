@@ -398,29 +398,13 @@ __device__ void norm_stats(uint32_t tx, const float* bias, bool write_back, int 
     for (int q = 1; q < NC_CC; ++q) st_peer4(pe.at(q, dst), __float_as_uint(part), pe.at(q, xss));
   }
 }
-// norm_operand: v * gain into chunk me of `buf` everywhere (exchange `xop`), and with t,
-// v * gain * t into chunk me of `buf2`.
-__device__ void norm_operand(float (&v)[16], const float* gain, uint8_t* buf, const float* t,
-                             uint8_t* buf2, uint64_t* xop, int cg, int r, int me, int tid,
-                             const Peers& pe) {
+// norm_operand: v * gain into chunk me of `buf`, here and in the peers (exchange `xop`).
+__device__ void norm_operand(float (&v)[16], const float* gain, uint8_t* buf, uint64_t* xop,
+                             int cg, int r, int me, int tid, const Peers& pe) {
 #pragma unroll
   for (int e = 0; e < 16; ++e) v[e] *= gain[16 * cg + e];
   put16(buf, me, r, cg, v);
-  if (t) {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] *= t[16 * cg + e];
-    put16(buf2, me, r, cg, v);
-  }
-  fence_async_shared();
-  rw_bar();
-  if (tid == 0) {
-#pragma unroll
-    for (int q = 1; q < NC_CC; ++q) {
-      bulk_to_peer(pe.at(q, buf + (size_t)me * CHUNK), buf + (size_t)me * CHUNK, CHUNK, pe.at(q, xop));
-      if (t) bulk_to_peer(pe.at(q, buf2 + (size_t)me * CHUNK), buf2 + (size_t)me * CHUNK, CHUNK, pe.at(q, xop));
-    }
-    bulk_wait_read();
-  }
+  send_all(buf + (size_t)me * CHUNK, CHUNK, xop, tid, pe);
 }
 // norm_recv: 1 / rms of row r over the 256 columns, once every CTA's partial is here.
 // A rw_bar separates it from the next norm_stats, which rewrites s_ss / s_ssx.
@@ -716,7 +700,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         norm_stats(tx, l == 0 ? nullptr : vec + V_B2 + ((l - 1) & 1) * NC_SL, true, cg, r, me,
                    s_ss, s_ssx, &sh.xg[X_SS(l)], pe, v);
         rs1 = norm_recv(r, s_ssx, &sh.xg[X_SS(l)], sh.abort);
-        norm_operand(v, vec + V_AN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[X_XN(l)], cg, r, me, tid,
+        norm_operand(v, vec + V_AN, sm + OFF_ACT, &sh.xg[X_XN(l)], cg, r, me, tid,
                      pe);
       }
       rw_signal(&sh.ready[R_XN(l)], lane);
@@ -782,7 +766,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
         float v[16];
         norm_stats(tx, vec + V_BO, true, cg, r, me, s_ss, s_ssx + NC_CC * NC_M, &sh.xg[X_SS2(l)],
                    pe, v);
-        norm_operand(v, vec + V_FN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[X_XN2(l)], cg, r, me,
+        norm_operand(v, vec + V_FN, sm + OFF_ACT, &sh.xg[X_XN2(l)], cg, r, me,
                      tid, pe);
       }
       rw_signal(&sh.ready[R_XN2(l)], lane);
@@ -848,7 +832,7 @@ __global__ void __launch_bounds__(NC_THREADS, 1)
 #pragma unroll
       for (int e = 0; e < 16; ++e) vt[e] = v[e] * vec[V_FIN + 16 * cg + e] * vec[V_T + 16 * cg + e];
       put16(sm + OFF_HF, me, r, cg, vt);
-      norm_operand(v, vec + V_FIN, sm + OFF_ACT, nullptr, nullptr, &sh.xg[xb(nl) + 1], cg, r, me,
+      norm_operand(v, vec + V_FIN, sm + OFF_ACT, &sh.xg[xb(nl) + 1], cg, r, me,
                    tid, pe);
     }
     // xf * t of the peers' slices from their xf, once it is here (one exchange instead of
