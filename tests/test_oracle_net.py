@@ -187,3 +187,60 @@ def test_fusion_with_zero_target_reduces_to_first_block():
     assert np.allclose(out.reshape(L * K, d), o / np.linalg.norm(o, axis=1, keepdims=True))
     a = W["anc_b"] / np.linalg.norm(W["anc_b"])
     assert np.allclose(anc, a)
+
+
+def test_transformer_matches_torch_encoder_stack():
+    """The whole pre-norm stack (App. A) against torch's own encoder layers with RMSNorm
+    swapped in, SiLU as the FFN activation and the bias tables as a per-head additive mask:
+    pins the order of norm, residual and FFN that the per-component pins leave open."""
+    rng = np.random.default_rng(4)
+    L, K, D, F, nh, nl = 4, 3, 32, 64, 8, 2
+    N = L * K
+    W = {}
+    for i in range(nl):
+        p = f"l{i}."
+        for n in ("wq", "wk", "wv", "wo"):
+            W[p + n] = rng.standard_normal((D, D)) * 0.3
+        for n in ("bq", "bk", "bv", "bo", "b2"):
+            W[p + n] = rng.standard_normal(D) * 0.3
+        W[p + "w1"] = rng.standard_normal((F, D)) * 0.3
+        W[p + "b1"] = rng.standard_normal(F) * 0.3
+        W[p + "w2"] = rng.standard_normal((D, F)) * 0.3
+        W[p + "an"] = 1 + 0.2 * rng.standard_normal(D)
+        W[p + "fn"] = 1 + 0.2 * rng.standard_normal(D)
+        W[p + "dist"] = rng.standard_normal((nh, 2 * L - 1))
+        W[p + "same"] = rng.standard_normal(nh)
+    W["final_norm"] = 1 + 0.2 * rng.standard_normal(D)
+    x = rng.standard_normal((N, D))
+    got = oracle.transformer(x, W, L, K, nh, nl)
+
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a))
+    slot = np.arange(N) // K
+    rel = slot[None, :] - slot[:, None] + L - 1
+    y = t(x)[None]
+    with torch.no_grad():
+        for i in range(nl):
+            p = f"l{i}."
+            layer = torch.nn.TransformerEncoderLayer(D, nh, F, dropout=0.0, activation=Fn.silu,
+                                                     batch_first=True, norm_first=True)
+            layer.norm1 = torch.nn.RMSNorm(D, eps=1e-6)
+            layer.norm2 = torch.nn.RMSNorm(D, eps=1e-6)
+            layer = layer.double().eval()
+            layer.self_attn.in_proj_weight.copy_(t(np.concatenate([W[p + "wq"], W[p + "wk"],
+                                                                   W[p + "wv"]])))
+            layer.self_attn.in_proj_bias.copy_(t(np.concatenate([W[p + "bq"], W[p + "bk"],
+                                                                 W[p + "bv"]])))
+            layer.self_attn.out_proj.weight.copy_(t(W[p + "wo"]))
+            layer.self_attn.out_proj.bias.copy_(t(W[p + "bo"]))
+            layer.linear1.weight.copy_(t(W[p + "w1"]))
+            layer.linear1.bias.copy_(t(W[p + "b1"]))
+            layer.linear2.weight.copy_(t(W[p + "w2"]))
+            layer.linear2.bias.copy_(t(W[p + "b2"]))
+            layer.norm1.weight.copy_(t(W[p + "an"]))
+            layer.norm2.weight.copy_(t(W[p + "fn"]))
+            mask = W[p + "dist"][:, rel] + W[p + "same"][:, None, None] * (rel == L - 1)
+            y = layer(y, src_mask=t(mask))
+        fin = torch.nn.RMSNorm(D, eps=1e-6).double()
+        fin.weight.copy_(t(W["final_norm"]))
+        want = fin(y)[0].numpy()
+    assert np.allclose(got, want, atol=1e-11)
