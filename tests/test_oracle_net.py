@@ -244,3 +244,94 @@ def test_transformer_matches_torch_encoder_stack():
         fin.weight.copy_(t(W["final_norm"]))
         want = fin(y)[0].numpy()
     assert np.allclose(got, want, atol=1e-11)
+
+
+def _zero_node_weights(H, D, L, K):
+    return {"emb_w": np.zeros((D, H)), "emb_b": np.zeros(D), "hid_w": np.zeros((D, H)),
+            "hid_b": np.zeros(D), "conf1_w": np.zeros((D, 5)), "conf1_b": np.zeros(D),
+            "conf2_w": np.zeros((D, D)), "conf2_b": np.zeros(D), "slot": np.zeros((L, D)),
+            "rank": np.zeros((K, D))}
+
+
+def test_nodes_decompose_into_the_four_terms():
+    """Sec. 3.2: each node is the sum of four terms. Switching all but one family of
+    weights off isolates each term, so a swapped slot/rank index, a token paired with the
+    wrong embedding row or a missing SiLU in the confidence network fails here."""
+    rng = np.random.default_rng(5)
+    H, D, L, K = 12, 6, 3, 4                        # L != K so slot and rank cannot swap
+    ids = rng.integers(0, 50, (L, K))
+    logp = -np.sort(rng.random((L, K)) * 4, axis=1)
+    hidden = rng.standard_normal((L, H))
+    E = rng.standard_normal((L, K, H))
+    base = _zero_node_weights(H, D, L, K)
+
+    W = dict(base, slot=rng.standard_normal((L, D)), rank=rng.standard_normal((K, D)))
+    n = oracle.nodes(ids, logp, hidden, E, W).reshape(L, K, D)
+    assert np.allclose(n, W["slot"][:, None, :] + W["rank"][None, :, :], atol=0)
+
+    W = dict(base, emb_w=rng.standard_normal((D, H)), emb_b=rng.standard_normal(D))
+    n = oracle.nodes(ids, logp, hidden, E, W).reshape(L, K, D)
+    for s in range(L):
+        for k in range(K):
+            assert np.allclose(n[s, k], W["emb_w"] @ E[s, k] + W["emb_b"])
+
+    W = dict(base, conf1_w=rng.standard_normal((D, 5)), conf1_b=rng.standard_normal(D),
+             conf2_w=rng.standard_normal((D, D)), conf2_b=rng.standard_normal(D))
+    n = oracle.nodes(ids, logp, hidden, E, W).reshape(L, K, D)
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a))
+    mlp = torch.nn.Sequential(torch.nn.Linear(5, D), torch.nn.SiLU(),
+                              torch.nn.Linear(D, D)).double()
+    with torch.no_grad():
+        mlp[0].weight.copy_(t(W["conf1_w"])); mlp[0].bias.copy_(t(W["conf1_b"]))
+        mlp[2].weight.copy_(t(W["conf2_w"])); mlp[2].bias.copy_(t(W["conf2_b"]))
+        for s in range(L):
+            lp = logp[s]
+            feats = np.stack([lp, np.exp(lp), lp[0] - lp, np.arange(K) / (K - 1),
+                              (np.arange(K) == 0).astype(float)], axis=1)
+            assert np.allclose(n[s], mlp(t(feats)).numpy(), atol=1e-13)
+
+
+def test_target_state_reads_the_mean_of_the_captured_layers():
+    """App. A: the five captured target layers are averaged before the RMSNorm over H, so
+    their order does not matter, a uniform positive scale cancels in the norm (up to its
+    epsilon), and five equal layers reduce to one."""
+    rng = np.random.default_rng(6)
+    H, D = 16, 8
+    W = {"tgt_norm": 1 + 0.1 * rng.standard_normal(H), "tgt_w": rng.standard_normal((D, H)),
+         "tgt_b": rng.standard_normal(D)}
+    T = rng.standard_normal((5, H))
+    t0 = oracle.target_state(T, W)
+    assert np.allclose(oracle.target_state(T[::-1], W), t0, atol=1e-13)
+    assert np.allclose(oracle.target_state(7.0 * T, W), t0, atol=1e-6)
+    one = T[2]
+    want = W["tgt_w"] @ (one / np.sqrt(np.mean(one * one) + 1e-6) * W["tgt_norm"]) + W["tgt_b"]
+    assert np.allclose(oracle.target_state(np.tile(one, (5, 1)), W), want, atol=1e-12)
+    # the mean, not the first or last layer: moving one layer moves t
+    T2 = T.copy()
+    T2[4] += 1.0
+    assert not np.allclose(oracle.target_state(T2, W), t0)
+
+
+def test_heads_are_scale_free_and_the_anchor_ignores_the_nodes():
+    """Sec. 3.2: out/in vectors are unit-normalised, so a positive scale of a head's
+    weights and bias leaves them unchanged; the anchor's vector depends on t alone."""
+    rng = np.random.default_rng(7)
+    D, d, L, K = 8, 6, 3, 2
+    W = {"fuse_w": rng.standard_normal((D, 3 * D)), "fuse_b": rng.standard_normal(D),
+         "out_w": rng.standard_normal((d, D)), "out_b": rng.standard_normal(d),
+         "in_w": rng.standard_normal((d, D)), "in_b": rng.standard_normal(d),
+         "anc_w": rng.standard_normal((d, D)), "anc_b": rng.standard_normal(d)}
+    x = rng.standard_normal((L * K, D))
+    t = rng.standard_normal(D)
+    out, inn, anc = oracle.fuse_and_heads(x, t, W, L, K)
+    W2 = dict(W, out_w=3 * W["out_w"], out_b=3 * W["out_b"], in_w=0.5 * W["in_w"],
+              in_b=0.5 * W["in_b"])
+    out2, inn2, anc2 = oracle.fuse_and_heads(x, t, W2, L, K)
+    assert np.allclose(out, out2, atol=1e-14) and np.allclose(inn, inn2, atol=1e-14)
+    _, _, anc3 = oracle.fuse_and_heads(rng.standard_normal((L * K, D)), t, W, L, K)
+    assert np.allclose(anc, anc3, atol=0)
+    # the x*t block: with x = 0 only the t block and bias remain, the same for every node
+    out0, _, _ = oracle.fuse_and_heads(np.zeros((L * K, D)), t, W, L, K)
+    u = Fn.silu(torch.from_numpy(W["fuse_w"][:, D:2 * D] @ t + W["fuse_b"])).numpy()
+    o = W["out_w"] @ u + W["out_b"]
+    assert np.allclose(out0.reshape(L * K, d), o / np.linalg.norm(o))
