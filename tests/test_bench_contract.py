@@ -2,6 +2,7 @@
 one JSON line with the keys of the measurement contract."""
 import json
 import os
+import socket
 import subprocess
 import sys
 
@@ -25,3 +26,22 @@ def test_reference_arm_prints_the_contract_line():
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
     assert d["e2e"]["value"] == d["value"] and d["cpu_baseline"]["kind"] == "oracle"
     assert d["cpu_baseline"]["cores"] >= 1
+
+
+def test_reference_arm_under_two_gloo_ranks_prints_once():
+    """Under torchrun (N = 2, gloo on the host) rank 0 alone runs the oracle and prints the
+    line; the other rank exits 0 without work."""
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    with socket.socket() as sk:                      # a free port on the loopback address
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    r = subprocess.run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1",
+                        "--nproc-per-node", "2", "--master-addr", "127.0.0.1",
+                        "--master-port", str(port), "bench.py", "--impl", "reference",
+                        "--gpus", "2", "--steps", "1", "--warmup", "3"],
+                       cwd=ROOT, capture_output=True, text=True, timeout=600, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.strip().startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
