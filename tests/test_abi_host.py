@@ -92,3 +92,53 @@ def test_status_strings(lib):
     for s in range(8):
         assert lib.lilicorr_status_str(s)
     assert lib.lilicorr_version() >= 1
+
+
+def test_widened_calls_check_arguments_before_launching(lib):
+    """Shape and argument errors come back synchronously, before any launch: the exact
+    path, the local softmax, the path diagnostics, coverage/acceptance, the vocabulary
+    shards and the fused LM head."""
+    bp = lib.lilicorr_best_path
+    assert bp(1, 0, 4, None, None, None, 8.0, None, None, None, None) == 2          # L = 0
+    assert bp(1, 65, 4, None, None, None, 8.0, None, None, None, None) == 2         # L > MAX_L
+    assert bp(1, 4, 33, None, None, None, 8.0, None, None, None, None) == 2         # K > MAX_K
+    assert bp(1, 4, 4, None, None, None, 0.0, None, None, None, None) == 1          # sigma = 0
+    assert bp(1, 4, 4, None, None, None, float("nan"), None, None, None, None) == 1
+    assert bp(0, 4, 4, None, None, None, 8.0, None, None, None, None) == 0          # no work
+    assert bp(1, 4, 4, None, None, None, 8.0, None, None, None, None) == 1          # nulls
+
+    ls = lib.lilicorr_local_softmax
+    assert ls(-1, 4, 4, None, None, 8.0, None, None, None) == 2
+    assert ls(1, 4, 4, None, None, -1.0, None, None, None) == 1
+    assert ls(1, 4, 4, None, None, float("inf"), None, None, None) == 1
+    assert ls(0, 4, 4, None, None, 8.0, None, None, None) == 0
+    assert ls(1, 4, 4, None, None, 8.0, None, None, None) == 1
+
+    pp = lib.lilicorr_path_probs
+    assert pp(1, 4, 0, None, None, None, 8.0, None, None, None, None) == 2
+    assert pp(1, 4, 4, None, None, None, 0.0, None, None, None, None) == 1
+    assert pp(1, 4, 4, None, None, None, 8.0, None, None, None, None) == 1
+
+    ba = lib.lilicorr_block_acceptance
+    assert ba(1, 0, 4, None, None, None, None, None, None, None) == 2
+    assert ba(0, 4, 4, None, None, None, None, None, None, None) == 0
+    assert ba(1, 4, 4, None, None, None, None, None, None, None) == 1
+
+    part, merge = lib.lilicorr_topk_lse_partial, lib.lilicorr_topk_lse_merge
+    assert part(None, 5, 4, 100, 8, 0, None, None, 0, None) == 3                   # dtype
+    assert part(None, 0, 4, 100, 0, 0, None, None, 0, None) == 2                   # K = 0
+    assert part(None, 0, 4, 100, 8, -1, None, None, 0, None) == 1                  # id offset
+    assert part(None, 0, 4, 100, 8, 2**31 - 50, None, None, 0, None) == 1          # ids overflow
+    assert part(None, 0, 0, 100, 8, 0, None, None, 0, None) == 0
+    assert part(None, 0, 4, 100, 8, 0, None, None, 0, None) == 1
+    assert merge(None, 0, 4, 8, None, None, None, None, None) == 2                 # P = 0
+    assert merge(None, 1025, 4, 8, None, None, None, None, None) == 2              # P*K > 8192
+    assert merge(None, 2, 0, 8, None, None, None, None, None) == 0
+    assert merge(None, 2, 4, 8, None, None, None, None, None) == 1
+    assert lib.lilicorr_topk_partial_bytes(0) == 0 and lib.lilicorr_topk_partial_bytes(33) == 0
+    assert lib.lilicorr_topk_partial_bytes(8) >= 8 + 8 * 8                         # m, s, keys
+
+    lm = lib.lilicorr_lm_head_topk
+    assert lm(None, None, 4, 4096, 4, 8, None, None, None, None, 0, None) == 2     # K > V
+    assert lm(None, None, 4, 4096, 100, 0, None, None, None, None, 0, None) == 2   # K = 0
+    assert lm(None, None, 0, 4096, 100, 8, None, None, None, None, 0, None) == 0
