@@ -8,13 +8,14 @@ K = 8, d = 256, H = 4096), 1000 distinct blocks drawn from seeds 1..1000 and
 resident in HBM (4.9 GB of logits, larger than L2, so no L2 flush is needed).
 One step selects all 1000 blocks one after another, each a complete batch-1
 call of lilicorr_select_block; the calls are captured 25 to a CUDA graph and the
-graphs replayed. Batched
-workloads (``--workload serving_b32`` etc.) time one call over the batch per step.
+graphs replayed. ``--workload serving_b32`` etc. time batched calls instead.
 
 Prints one JSON line (rank 0): device-timed throughput (``value``), the same
 metric end to end through pinned host buffers (``e2e``), the top-K kernel's
 roofline measured live with CUDA events, SM clocks sampled during the timed
-region, and the CPU oracle timed on a bounded sample (``cpu_baseline``).
+region, ``by_workload`` (the batched workloads, each entropy tier on its own:
+call time, the top-K pass's bandwidth and the end-to-end roofline fraction), and
+the CPU oracle timed on all host cores on a bounded sample (``cpu_baseline``).
 ``--impl reference`` times the CPU oracle itself as the reference arm.
 """
 from __future__ import annotations
@@ -22,7 +23,7 @@ from __future__ import annotations
 import os
 
 for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
-    os.environ.setdefault(_v, "1")          # the oracle baseline runs on one core
+    os.environ.setdefault(_v, "1")          # one BLAS thread per oracle worker process
 
 import argparse
 import json
@@ -58,9 +59,9 @@ def parse_args():
                    help="distinct batches per step (batched workloads; default: up to 8, "
                         "about 1.6 GB of logits)")
     p.add_argument("--e2e-host-blocks", type=int, default=64)
-    p.add_argument("--calls-per-graph", type=int, default=25,
-                   help="batch-1 select_block calls captured in one CUDA graph")
-    p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-by-workload", dest="by_workload", action="store_false",
+                   help="skip the batched workloads' section of the default run")
     p.add_argument("--no-cpu-baseline", action="store_true")
     return p.parse_args()
 
@@ -178,49 +179,117 @@ def peaks():
 
 
 # --------------------------------------------------------------------------- CPU oracle leg
-def oracle_blocks_per_s(wl, W, seeds, seconds: float):
-    """The oracle, as it stands, selecting whole blocks one after another on the host."""
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+_ORACLE_JOB = {}      # the workload and weights the forked workers select with
+
+
+def _oracle_noop(_):
+    return os.getpid()
+
+
+def _oracle_block(seed):
+    """One whole block through the oracle, as it stands (runs in a pool worker)."""
     import oracle
+    wl, W = _ORACLE_JOB["wl"], _ORACLE_JOB["W"]
+    inp = workloads.sequence_inputs(wl, seed)
     emb = lambda ids: workloads.embed_rows(wl.V, wl.H, wl.dtype, ids)
-    done, t0 = 0, time.perf_counter()
-    for seed in seeds:
-        inp = workloads.sequence_inputs(wl, seed)
-        oracle.select_sequence(inp["logits"], inp["hidden"], inp["target"], emb, W, wl.K)
-        done += 1
-        if time.perf_counter() - t0 >= seconds:
-            break
-    dt = time.perf_counter() - t0
-    return done / dt, done, dt
+    oracle.select_sequence(inp["logits"], inp["hidden"], inp["target"], emb, W, wl.K)
+    return 1
 
 
-def run_reference(args, world, rank):
-    """Reference arm: the CPU oracle on the host cores, one block per step."""
+class OraclePool:
+    """The oracle on every host core: one worker process per core, one BLAS thread each.
+
+    The workers are forked at construction, before this process touches the GPU (a child
+    forked after CUDA initialisation can hang), after the embedding table is built, so
+    they share its pages instead of each regenerating it."""
+
+    def __init__(self, wl, W):
+        import concurrent.futures as cf
+        import multiprocessing as mp
+        _ORACLE_JOB.update(wl=wl, W=W)
+        workloads.embed_table(wl.V, wl.H, wl.dtype)        # cached in this process
+        self.cores = host_cores()
+        self.ex = cf.ProcessPoolExecutor(self.cores, mp_context=mp.get_context("fork"))
+        list(self.ex.map(_oracle_noop, range(self.cores)))   # fork every worker now
+
+    def run(self, seeds):
+        """Select the blocks ``seeds`` on all workers; returns the wall time."""
+        t0 = time.perf_counter()
+        n = sum(self.ex.map(_oracle_block, seeds))
+        assert n == len(seeds)
+        return time.perf_counter() - t0
+
+    def rate(self, seeds, seconds: float):
+        """Blocks/s over waves of one block per worker until ``seconds`` have passed."""
+        done, dt, i = 0, 0.0, 0
+        while dt < seconds and i < len(seeds):
+            wave = seeds[i:i + self.cores]
+            dt += self.run(wave)
+            done += len(wave)
+            i += len(wave)
+        return done / dt, done, dt
+
+    def close(self):
+        self.ex.shutdown()
+
+
+def workload_config(wl, nblk: int, world: int) -> dict:
+    """The ``config`` object of both arms' JSON lines (the same workload description)."""
+    es = 2 if wl.dtype == "bf16" else 4
+    batch1 = wl.blocks > 1
+    B = 1 if batch1 else wl.B
+    gb = nblk * B * wl.L * wl.V * es / 1e9
+    return {"workload": wl.name, "B": B, "L": wl.L, "V": wl.V, "K": wl.K, "d": wl.d, "D": wl.D,
+            "H": wl.H, "blocks_per_step": nblk,
+            "l2": "inputs larger than L2 (no flush): %.2f GB of logits in %d distinct resident %s"
+                  % (gb, nblk, "blocks" if batch1 else "batches"),
+            "graphs": f"{GRAPH_CALLS} select_block calls per CUDA graph, replayed",
+            "parallelism": f"dp{world}"}
+
+
+def default_blocks(wl, args) -> int:
+    if wl.blocks > 1:
+        return args.blocks or wl.blocks
+    es = 2 if wl.dtype == "bf16" else 4
+    return args.batches or max(1, min(8, int(1.6e9 // (wl.B * wl.L * wl.V * es))))
+
+
+def run_reference(args, world, rank, pool):
+    """Reference arm: the CPU oracle on all host cores (one block per worker per step)."""
     if rank != 0:
         return
     wl = workloads.WORKLOADS[args.workload]
-    W = workloads.head_weights(wl)
     seeds = wl.block_seeds() if wl.blocks > 1 else wl.seeds()
-    workloads.embed_table(wl.V, wl.H, wl.dtype)          # generate once, outside the timing
+    C = pool.cores
+    wave = lambda i: [seeds[(i * C + j) % len(seeds)] for j in range(C)]
     for i in range(args.warmup):
-        oracle_blocks_per_s(wl, W, [seeds[i % len(seeds)]], 0.0)
-    t0 = time.perf_counter()
-    for i in range(args.steps):
-        oracle_blocks_per_s(wl, W, [seeds[(args.warmup + i) % len(seeds)]], 0.0)
-    dt = time.perf_counter() - t0
-    v = args.steps / dt
-    sample = f"{args.steps} sequences of the {wl.name} workload, one per step"
+        pool.run(wave(i))
+    dt = sum(pool.run(wave(args.warmup + i)) for i in range(args.steps))
+    v = args.steps * C / dt
+    sample = (f"{args.steps} steps of {C} sequences of the {wl.name} workload, one per "
+              f"worker process (fp64 NumPy, 1 BLAS thread each)")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": wl.name, "B": 1, "L": wl.L, "V": wl.V,
-                                        "K": wl.K, "d": wl.d, "H": wl.H},
-        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "data": "synthetic", "config": workload_config(wl, default_blocks(wl, args), world),
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": C, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
 
 # --------------------------------------------------------------------------- GPU arm
+GRAPH_CALLS = 25          # select_block calls captured per CUDA graph (batch-1 workload)
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal
+
+
 def upload(a: np.ndarray, dtype: str, dev) -> torch.Tensor:
     t = torch.from_numpy(np.ascontiguousarray(a))
     return (t.to(torch.bfloat16) if dtype == "bf16" else t).to(dev)
@@ -245,7 +314,156 @@ def gen_blocks(wl, seeds, dev, chunk=50):
     return logits, hidden, target, planted
 
 
-def run_ours(args, world, rank, local):
+def gen_batches(wl, nb, tier, rank, dev):
+    """nb distinct batches [nb, B, L, V] etc.; batch 0 of rank 0 is the workload's own."""
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    B = wl.B
+    logits = torch.empty((nb, B, wl.L, wl.V), dtype=tdt, device=dev)
+    hidden = torch.empty((nb, B, wl.L, wl.H), dtype=tdt, device=dev)
+    target = torch.empty((nb, B, wl.n_tgt, wl.H), dtype=tdt, device=dev)
+    for j in range(nb):
+        inp = workloads.batch_inputs(wl, [s + rank * 100000 + j * 1000003 for s in wl.seeds(tier)],
+                                     tier)
+        logits[j] = upload(inp["logits"], wl.dtype, dev)
+        hidden[j] = upload(inp["hidden"], wl.dtype, dev)
+        target[j] = upload(inp["target"], wl.dtype, dev)
+        del inp
+    return logits, hidden, target
+
+
+def graph_of(fns):
+    """One CUDA graph replaying the calls ``fns`` in order."""
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for f in fns:
+            f()
+    return g
+
+
+def time_replays(graphs, stream, reps: int, warm: int = 2) -> float:
+    """ms per replay of the graph list, CUDA events on the launching stream."""
+    for _ in range(warm):
+        for g in graphs:
+            g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        for g in graphs:
+            g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def head_weight_bytes(wl) -> int:
+    """Bytes of the head's weights read once per call (bf16), excluding the [V, .] table
+    and the embedding projection that the folded table replaces."""
+    es = 2 if wl.dtype == "bf16" else 4
+    n = sum(int(np.prod(sh)) for name, sh in workloads.head_param_shapes(
+        wl.H, wl.D, wl.d, wl.F, wl.n_heads, wl.L, wl.K, wl.n_layers)
+        if name not in ("emb_w", "emb_b"))
+    return n * es
+
+
+def algorithmic(wl, B: int):
+    """Algorithmic bytes and flops of one select_block call over B sequences."""
+    es = 2 if wl.dtype == "bf16" else 4
+    N = B * wl.L * wl.K
+    D, H, L, K = wl.D, wl.H, wl.L, wl.K
+    logit_bytes = B * L * wl.V * es
+    nbytes = (logit_bytes + B * L * H * es + B * wl.n_tgt * H * es + N * D * 4
+              + head_weight_bytes(wl) + B * L * 4)
+    flops = (2 * B * L * H * D + 2 * B * H * D + 44 * N * D * D + 8 * B * (L * K) ** 2 * D
+             + 2 * wl.d * B * ((L - 1) * K * K + K))
+    return logit_bytes, nbytes, flops
+
+
+def roofline_fracs(wl, B, us_call, us_topk, pk):
+    hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
+    tf = float(pk.get("bf16_tflops_sustained", pk.get("bf16_tflops", 1700.0)))
+    logit_bytes, nbytes, flops = algorithmic(wl, B)
+    t_bytes = nbytes / (hbm * 1e9) * 1e6
+    t_flops = flops / (tf * 1e12) * 1e6
+    topk_gbs = logit_bytes / (us_topk * 1e-6) / 1e9
+    return {
+        "topk_us": round(us_topk, 2), "topk_gbs": round(topk_gbs, 1),
+        "topk_frac": round(topk_gbs / hbm, 4), "topk_frac_nominal": round(topk_gbs / NOMINAL_HBM_GBS, 4),
+        "alg_bytes_per_call": nbytes, "alg_gflop_per_call": round(flops / 1e9, 2),
+        "floor_us": {"hbm": round(t_bytes, 2), "tensor": round(t_flops, 2)},
+        "e2e_frac": round(max(t_bytes, t_flops) / us_call, 4),
+        "e2e_frac_bytes_over_hbm": round(t_bytes / us_call, 4),
+    }
+
+
+def bench_batched(ll, name, tier, dev, stream, E, pk, rank, min_bytes=6e8, reps=5):
+    """One batched workload (one tier) through select_block: device-timed calls over
+    distinct resident batches (inputs larger than L2), the top-K pass alone, and the
+    same calls end to end from pinned host buffers."""
+    wl = workloads.WORKLOADS[name]
+    es = 2 if wl.dtype == "bf16" else 4
+    B = wl.B
+    nb = max(1, int(np.ceil(min_bytes / (B * wl.L * wl.V * es))))
+    W = workloads.head_weights(wl)
+    head = ll.Head.from_workload(wl, W, E)
+    logits, hidden, target = gen_batches(wl, nb, tier, rank, dev)
+    ws = head.workspace(B)
+    tokens = torch.empty((nb, B, wl.L), dtype=torch.int32, device=dev)
+    n0 = ll.launch_count()
+    ll.select_block(head, logits[0], hidden[0], target[0], ws=ws, tokens=tokens[0])
+    launches = ll.launch_count() - n0
+    torch.cuda.synchronize()
+    if ws.status() != 0:
+        raise RuntimeError(f"{name}: device status set")
+    calls = [lambda j=j: ll.select_block(head, logits[j], hidden[j], target[j], ws=ws,
+                                         tokens=tokens[j]) for j in range(nb)]
+    g = graph_of(calls)
+    us_call = time_replays([g], stream, reps) * 1e3 / nb
+    rows = B * wl.L
+    tk_ws = ll.Workspace(ll.lib().lilicorr_topk_lse_workspace_bytes(rows, wl.V, wl.K))
+    flat = logits.view(nb, rows, wl.V)
+    ll.topk_lse(flat[0], wl.K, ws=tk_ws)
+    tg = graph_of([lambda j=j: ll.topk_lse(flat[j], wl.K, ws=tk_ws) for j in range(nb)] * 2)
+    us_topk = time_replays([tg], stream, reps) * 1e3 / (2 * nb)
+    # end to end: each call copies its batch from pinned host memory and its tokens back
+    h_l = logits.cpu().pin_memory()
+    h_h = hidden.cpu().pin_memory()
+    h_t = target.cpu().pin_memory()
+    h_tok = torch.empty((nb, B, wl.L), dtype=torch.int32).pin_memory()
+    d_l, d_h, d_t = torch.empty_like(logits[0]), torch.empty_like(hidden[0]), torch.empty_like(target[0])
+    d_tok = torch.empty((B, wl.L), dtype=torch.int32, device=dev)
+
+    def e2e_call(j):
+        d_l.copy_(h_l[j], non_blocking=True)
+        d_h.copy_(h_h[j], non_blocking=True)
+        d_t.copy_(h_t[j], non_blocking=True)
+        ll.select_block(head, d_l, d_h, d_t, ws=ws, tokens=d_tok)
+        h_tok[j].copy_(d_tok, non_blocking=True)
+    eg = graph_of([lambda j=j: e2e_call(j) for j in range(nb)])
+    us_e2e = time_replays([eg], stream, max(2, reps // 2), warm=1) * 1e3 / nb
+    if ws.status() != 0 or tk_ws.status() != 0:
+        raise RuntimeError(f"{name}: device status set")
+    h2d = (d_l.numel() + d_h.numel() + d_t.numel()) * es
+    out = {"tier": (wl.tiers[tier] if wl.tiers else None), "B": B, "K": wl.K, "D": wl.D,
+           "us_per_call": round(us_call, 2), "sequences_per_s": round(B / (us_call * 1e-6), 1),
+           "calls_per_s": round(1e6 / us_call, 1), "launches_per_call": launches,
+           "distinct_batches": nb,
+           "e2e": {"us_per_call": round(us_e2e, 2),
+                   "sequences_per_s": round(B / (us_e2e * 1e-6), 1),
+                   "h2d_bytes_per_call": h2d, "d2h_bytes_per_call": B * wl.L * 4}}
+    out.update(roofline_fracs(wl, B, us_call, us_topk, pk))
+    head.close()
+    del logits, hidden, target, h_l, h_h, h_t, flat
+    torch.cuda.empty_cache()
+    return out
+
+
+BATCHED = [("serving_b32", 0), ("entropy_tiers_b64", 0), ("entropy_tiers_b64", 1),
+           ("entropy_tiers_b64", 2), ("ties_b256", 0)]
+
+
+def run_ours(args, world, rank, local, pool):
     import __graft_entry__
     __graft_entry__.build()
     import paper_2608_20530_gb300 as ll
@@ -258,10 +476,11 @@ def run_ours(args, world, rank, local):
     E = workloads.embed_table(wl.V, wl.H, wl.dtype)
     head = ll.Head.from_workload(wl, W, E)
     stream = torch.cuda.current_stream()
+    pk, pk_kind = peaks()
 
     batch1 = wl.blocks > 1
+    nblk = default_blocks(wl, args)
     if batch1:
-        nblk = args.blocks or wl.blocks
         seeds = [s + rank * nblk for s in wl.block_seeds()[:nblk]] if nblk <= wl.blocks else \
             [wl.seed_base + i + rank * nblk for i in range(nblk)]
         logits, hidden, target, planted = gen_blocks(wl, seeds, dev)
@@ -269,24 +488,9 @@ def run_ours(args, world, rank, local):
     else:
         # several distinct batches per step, captured together like the batch-1 blocks (a
         # serving loop does not pay one graph launch per call)
-        batch_bytes = wl.B * wl.L * wl.V * es
-        nblk = args.batches or max(1, min(8, int(1.6e9 // batch_bytes)))
         B = wl.B
-        tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-        logits = torch.empty((nblk, B, wl.L, wl.V), dtype=tdt, device=dev)
-        hidden = torch.empty((nblk, B, wl.L, wl.H), dtype=tdt, device=dev)
-        target = torch.empty((nblk, B, wl.n_tgt, wl.H), dtype=tdt, device=dev)
+        logits, hidden, target = gen_batches(wl, nblk, 0, rank, dev)
         planted = None
-        for j in range(nblk):
-            inp = workloads.batch_inputs(wl, [s + rank * 100000 + j * 1000003 for s in wl.seeds()])
-            logits[j] = upload(inp["logits"], wl.dtype, dev)
-            hidden[j] = upload(inp["hidden"], wl.dtype, dev)
-            target[j] = upload(inp["target"], wl.dtype, dev)
-            if inp["planted"] is not None:
-                if planted is None:
-                    planted = np.zeros((nblk,) + inp["planted"].shape, np.int32)
-                planted[j] = inp["planted"]
-            del inp
     ws = head.workspace(B)
     tokens = torch.empty((nblk, B, wl.L), dtype=torch.int32, device=dev)
 
@@ -298,14 +502,12 @@ def run_ours(args, world, rank, local):
     if ws.status() != 0:
         raise RuntimeError("device status set on the first call")
 
-    G = max(1, min(args.calls_per_graph, nblk))
+    G = max(1, min(GRAPH_CALLS, nblk))
     graphs = []
     for i0 in range(0, nblk, G):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g):
-            for i in range(i0, min(i0 + G, nblk)):
-                ll.select_block(head, logits[i], hidden[i], target[i], ws=ws, tokens=tokens[i])
-        graphs.append(g)
+        graphs.append(graph_of([lambda i=i: ll.select_block(head, logits[i], hidden[i], target[i],
+                                                            ws=ws, tokens=tokens[i])
+                                for i in range(i0, min(i0 + G, nblk))]))
     torch.cuda.synchronize()
 
     def step():
@@ -339,30 +541,25 @@ def run_ours(args, world, rank, local):
 
     # ---- end to end: pinned host inputs -> device -> select -> tokens back to pinned host
     nh = min(args.e2e_host_blocks, nblk)
-    h_logits = torch.empty((nh,) + tuple(logits.shape[1:]), dtype=logits.dtype).pin_memory()
-    h_hidden = torch.empty((nh,) + tuple(hidden.shape[1:]), dtype=hidden.dtype).pin_memory()
-    h_target = torch.empty((nh,) + tuple(target.shape[1:]), dtype=target.dtype).pin_memory()
-    h_logits.copy_(logits[:nh].cpu())
-    h_hidden.copy_(hidden[:nh].cpu())
-    h_target.copy_(target[:nh].cpu())
+    h_logits = logits[:nh].cpu().pin_memory()
+    h_hidden = hidden[:nh].cpu().pin_memory()
+    h_target = target[:nh].cpu().pin_memory()
     h_tokens = torch.empty((nh, B, wl.L), dtype=torch.int32).pin_memory()
     d_logits = torch.empty_like(logits[0])
     d_hidden = torch.empty_like(hidden[0])
     d_target = torch.empty_like(target[0])
     d_tokens = torch.empty((B, wl.L), dtype=torch.int32, device=dev)
+
+    def e2e_call(i):
+        d_logits.copy_(h_logits[i], non_blocking=True)
+        d_hidden.copy_(h_hidden[i], non_blocking=True)
+        d_target.copy_(h_target[i], non_blocking=True)
+        ll.select_block(head, d_logits, d_hidden, d_target, ws=ws, tokens=d_tokens)
+        h_tokens[i].copy_(d_tokens, non_blocking=True)
+
     # each e2e graph holds G calls, each: its inputs host -> device, select, tokens -> host
-    e2e_graphs = []
-    for k in range(-(-nh // G)):
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g):
-            for j in range(G):
-                i = (k * G + j) % nh
-                d_logits.copy_(h_logits[i], non_blocking=True)
-                d_hidden.copy_(h_hidden[i], non_blocking=True)
-                d_target.copy_(h_target[i], non_blocking=True)
-                ll.select_block(head, d_logits, d_hidden, d_target, ws=ws, tokens=d_tokens)
-                h_tokens[i].copy_(d_tokens, non_blocking=True)
-        e2e_graphs.append(g)
+    e2e_graphs = [graph_of([lambda i=(k * G + j) % nh: e2e_call(i) for j in range(G)])
+                  for k in range(-(-nh // G))]
     n_e2e_replays = -(-nblk // G)
     e2e_calls = n_e2e_replays * G
 
@@ -383,40 +580,22 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     barrier(world)
     e2e_ms = max_over_ranks(world, e0.elapsed_time(e1))
-    e2e_value = e2e_calls * B * args.steps * world / (e2e_ms / 1e3) if not batch1 else \
-        e2e_calls * args.steps * world / (e2e_ms / 1e3)
+    e2e_value = e2e_calls * (1 if batch1 else B) * args.steps * world / (e2e_ms / 1e3)
     h2d = (d_logits.numel() * d_logits.element_size() + d_hidden.numel() * d_hidden.element_size()
            + d_target.numel() * d_target.element_size()) * e2e_calls
     d2h = d_tokens.numel() * 4 * e2e_calls
+    del h_logits, h_hidden, h_target, e2e_graphs
 
     # ---- the exact best path (App. E) in place of the greedy walk: the same calls on a
     # sample of the blocks, both walks captured alike and timed back to back
     nv = min(nblk, 100)
     walk_ms = {}
     for walk in ("greedy", "viterbi"):
-        gl = []
-        for i0 in range(0, nv, G):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                for i in range(i0, min(i0 + G, nv)):
-                    ll.select_block(head, logits[i], hidden[i], target[i], ws=ws, tokens=tokens[i],
-                                    walk=walk)
-            gl.append(g)
-        for g in gl:
-            g.replay()
-        torch.cuda.synchronize()
-        best = None
-        for _ in range(3):
-            w0 = torch.cuda.Event(enable_timing=True)
-            w1 = torch.cuda.Event(enable_timing=True)
-            w0.record(stream)
-            for g in gl:
-                g.replay()
-            w1.record(stream)
-            torch.cuda.synchronize()
-            t = w0.elapsed_time(w1)
-            best = t if best is None else min(best, t)
-        walk_ms[walk] = best / nv
+        gl = [graph_of([lambda i=i: ll.select_block(head, logits[i], hidden[i], target[i], ws=ws,
+                                                     tokens=tokens[i], walk=walk)
+                        for i in range(i0, min(i0 + G, nv))]) for i0 in range(0, nv, G)]
+        walk_ms[walk] = min(time_replays(gl, stream, 1, warm=1 if k == 0 else 0)
+                            for k in range(3)) / nv
     if ws.status() != 0:
         raise RuntimeError("device status set by the walk comparison")
 
@@ -441,22 +620,11 @@ def run_ours(args, world, rank, local):
             ll.block_acceptance(inter["ids"], tokens[nd - 1], truth)
         diag_call()
         torch.cuda.synchronize()
-        dg = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(dg):
-            for _ in range(50):
-                diag_call()
-        dg.replay()
-        torch.cuda.synchronize()
-        d0 = torch.cuda.Event(enable_timing=True)
-        d1 = torch.cuda.Event(enable_timing=True)
-        d0.record(stream)
-        dg.replay()
-        d1.record(stream)
-        torch.cuda.synchronize()
+        dg = graph_of([diag_call] * 50)
         diag = {"truth": "planted token per slot", "blocks": nd * B,
                 "mean_oracle_prefix": round(prefix_sum / (nd * B), 3),
                 "mean_accepted": round(acc_sum / (nd * B), 3),
-                "us_per_call": round(d0.elapsed_time(d1) * 1e3 / 50, 2),
+                "us_per_call": round(time_replays([dg], stream, 1, warm=1) * 1e3 / 50, 2),
                 "note": "path_probs + block_acceptance on one call's outputs"}
 
     # ---- roofline of the top-K pass: its launches back to back in one captured graph,
@@ -468,25 +636,14 @@ def run_ours(args, world, rank, local):
     for i in range(min(reps, 8)):
         ll.topk_lse(flat[i % nblk], wl.K, ws=tk_ws)
     torch.cuda.synchronize()
-    tg = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(tg):
-        for i in range(reps):
-            ll.topk_lse(flat[i % nblk], wl.K, ws=tk_ws)
-    tg.replay()
-    torch.cuda.synchronize()
-    k0 = torch.cuda.Event(enable_timing=True)
-    k1 = torch.cuda.Event(enable_timing=True)
-    k0.record(stream)
-    tg.replay()
-    k1.record(stream)
-    torch.cuda.synchronize()
-    tk_ms = k0.elapsed_time(k1) / reps
+    tg = graph_of([lambda i=i: ll.topk_lse(flat[i % nblk], wl.K, ws=tk_ws) for i in range(reps)])
+    tk_ms = time_replays([tg], stream, 1, warm=1) / reps
     alg_bytes = rows * wl.V * es
-    pk, pk_kind = peaks()
     hbm = float(pk.get("hbm_gbs", FALLBACK_HBM_GBS))
     achieved = alg_bytes / (tk_ms / 1e3) / 1e9
     roofline = {"kernel": "topk_lse_kernel", "bound": "hbm", "achieved": round(achieved, 1),
                 "peak": hbm, "peak_kind": pk_kind, "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                "frac_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
                 "traffic": profiled_traffic("topk_lse.cu", wl.name),
                 "alg_bytes_per_launch": alg_bytes, "us_per_launch": round(tk_ms * 1e3, 3)}
 
@@ -504,19 +661,7 @@ def run_ours(args, world, rank, local):
     def timed(fn, n=20):
         fn()
         torch.cuda.synchronize()
-        gr = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gr):
-            for _ in range(n):
-                fn()
-        gr.replay()
-        torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        gr.replay()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        return e0.elapsed_time(e1) * 1e3 / n
+        return time_replays([graph_of([fn] * n)], stream, 1, warm=1) * 1e3 / n
 
     part_us = timed(lambda: ll.topk_lse_partial(sl[0], wl.K, 0, ws=sws[0]))
     merge_us = timed(lambda: ll.topk_lse_merge(recs, wl.K))
@@ -563,28 +708,45 @@ def run_ours(args, world, rank, local):
 
     l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
     in_bytes = logits.numel() * es
-    if in_bytes > l2_bytes:
-        l2_note = "inputs larger than L2 (%.0f MB): %.2f GB of logits" % (l2_bytes / 1e6, in_bytes / 1e9)
-        l2_note += (" in %d distinct resident blocks" % nblk if batch1 else
-                    " in %d distinct resident batches" % nblk)
-    else:
-        l2_note = ("inputs fit in L2 (%.2f GB of logits, L2 %.0f MB): a profiling size, "
-                   "not a bench configuration" % (in_bytes / 1e9, l2_bytes / 1e6))
+    del logits, hidden, target, flat, graphs
+    head.close()
+    torch.cuda.empty_cache()
+
+    # ---- the batched workloads (spec batch >= 32): each tier on its own
+    by_workload = None
+    if args.by_workload and batch1:
+        bclk = ClockSampler()
+        bclk.start()
+        by_workload = {}
+        for name, tier in BATCHED:
+            key = name if not workloads.WORKLOADS[name].tiers else f"{name}.tau{workloads.WORKLOADS[name].tiers[tier]}"
+            by_workload[key] = bench_batched(ll, name, tier, dev, stream, E, pk, rank)
+        by_workload["clocks"] = bclk.stop()
+        by_workload["note"] = ("each: select_block over distinct resident batches (>= 0.6 GB of "
+                               "logits, larger than L2) in one CUDA graph, CUDA events; topk_* = "
+                               "the top-K pass alone over the same batches (fractions of the "
+                               "measured copy bandwidth and of the nominal 7.9 TB/s); e2e_frac = "
+                               "max(bytes/HBM, flops/sustained bf16) over the call time, "
+                               "algorithmic bytes and flops per call; e2e = the same calls with "
+                               "their inputs copied from pinned host memory and tokens back")
+
+    config = workload_config(wl, nblk, world)
+    if in_bytes <= l2_bytes:
+        config["l2"] = ("inputs fit in L2 (%.2f GB of logits, L2 %.0f MB): a profiling size, "
+                        "not a bench configuration" % (in_bytes / 1e9, l2_bytes / 1e6))
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": {"workload": wl.name, "B": B, "L": wl.L, "V": wl.V, "K": wl.K, "d": wl.d,
-                   "D": wl.D, "H": wl.H, "blocks_per_step": nblk,
-                   "l2": l2_note,
-                   "graphs": f"{G} select_block calls per CUDA graph, replayed",
-                   "parallelism": f"dp{world}"},
+        "config": config,
         "us_per_block": ms_per_step * 1e3 / nblk,
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "note": f"pinned host blocks cycled ({nh} distinct), copies captured with each call"},
         "gpu_launches": launches_per_call * nblk * args.steps,
+        "roofline": roofline,
+        "by_workload": by_workload,
         "diagnostics": diag,
         "walk_viterbi": {"us_per_call": round(walk_ms["viterbi"] * 1e3, 2),
                          "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
@@ -592,26 +754,35 @@ def run_ours(args, world, rank, local):
                          "sample": f"{nv} calls of this workload, best of 3"},
         "vocab_sharded": sharded,
         "lm_head_fused": lm_head,
-        "roofline": roofline,
     }
-    if rank == 0 and not args.no_cpu_baseline:
+    if pool is not None:
         seeds_cpu = wl.block_seeds() if batch1 else wl.seeds()
-        v, n, dt = oracle_blocks_per_s(wl, W, seeds_cpu, args.cpu_seconds)
+        v, n, dt = pool.rate(seeds_cpu, args.cpu_seconds)
         result["cpu_baseline"] = {
-            "value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{n} sequences of the {wl.name} workload in {dt:.1f} s (fp64 NumPy, 1 thread)"}
+            "value": v, "unit": UNIT, "cores": pool.cores, "kind": "oracle",
+            "sample": f"{n} sequences of the {wl.name} workload in {dt:.1f} s, one per worker "
+                      f"process on {pool.cores} host cores (fp64 NumPy, 1 BLAS thread each)"}
     if rank == 0:
         print(json.dumps(result))
-    head.close()
 
 
 def main():
     args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    pool = None
+    if rank == 0 and (args.impl == "reference" or not args.no_cpu_baseline):
+        # forked before this process initialises CUDA
+        wl = workloads.WORKLOADS[args.workload]
+        pool = OraclePool(wl, workloads.head_weights(wl))
     world, rank, local = dist_setup(args)
-    if args.impl == "reference":
-        run_reference(args, world, rank)
-    else:
-        run_ours(args, world, rank, local)
+    try:
+        if args.impl == "reference":
+            run_reference(args, world, rank, pool)
+        else:
+            run_ours(args, world, rank, local, pool)
+    finally:
+        if pool is not None:
+            pool.close()
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()

@@ -2,6 +2,11 @@
  * lilicorr_testing.h - test hooks of the LiLiCorr library. Not part of the
  * selection path; they expose internal building blocks so tests can check them
  * one at a time.
+ *
+ * The two path switches below (lilicorr_test_fused_path, lilicorr_test_attention_path)
+ * change process-global dispatch state that every head and every host thread reads when
+ * it enqueues a call. They are not synchronised: set them only while no other thread is
+ * enqueueing work through the library, and put the default back afterwards.
  */
 #ifndef LILICORR_TESTING_H_
 #define LILICORR_TESTING_H_
@@ -27,6 +32,18 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
                                        lilicorr_dtype_t c_dt, int ldc, int M, int N, int Kd,
                                        const float* bias, const float* residual, int act, int path,
                                        uint32_t* status, cudaStream_t stream);
+
+/* The failure branch of the tensor-core linear layer's bounded waits (path 3 of
+ * lilicorr_test_linear, with C = A W^T, bf16 A [M, Kd] and W [N, Kd] row-major, fp32 C
+ * [M, N]), made to run: the kernel's producer issues none of its copies, so the MMA
+ * warp waits on a barrier that nothing arrives on. Every wait gives up after wait_cycles
+ * SM cycles (1e5 .. 4e9; the production limit is 4e9, about 2 s); the kernel then records
+ * LILICORR_ERR_TIMEOUT in *status (a device uint32 word, required), stops issuing, frees
+ * its tensor memory and returns, leaving the context usable. C receives unspecified
+ * values. LILICORR_ERR_SHAPE for shapes the tensor-core kernel does not take. */
+lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, float* C, int M, int N,
+                                               int Kd, long long wait_cycles, uint32_t* status,
+                                               cudaStream_t stream);
 
 /* Switch for the fused scoring-network kernels (bf16 heads with D = 256, 8 heads,
  * FFN 2D, L*K <= 128): mode 1 (the default) takes the cluster kernel (four CTAs per

@@ -80,6 +80,7 @@ _SIGS = {
     "lilicorr_topk_lse_noalloc": (_I, [_P, _I, _I, _I, _I, _P, _P, _P, _P]),
     "lilicorr_test_linear": (_I, [_P, _I, _I, _P, _I, _I, _P, _I, _I, _I, _I, _I, _P, _P, _I, _I,
                                   _P, _P]),
+    "lilicorr_test_linear_timeout": (_I, [_P, _P, _P, _I, _I, _I, ctypes.c_longlong, _P, _P]),
 }
 
 
@@ -490,6 +491,20 @@ def test_linear(A: torch.Tensor, W: torch.Tensor, out_dtype=torch.float32, bias=
                                       _dtype_code(W), W.stride(0), C.data_ptr(), _dtype_code(C),
                                       C.stride(0), M, N, Kd, _ptr(bias), _ptr(residual), act,
                                       path, _ptr(status), _stream()), "test_linear")
+    return C
+
+
+def test_linear_timeout(A: torch.Tensor, W: torch.Tensor, wait_cycles: int,
+                        status: torch.Tensor) -> torch.Tensor:
+    """Test hook: the tensor-core linear layer with its copies withheld, so its bounded
+    waits run out after ``wait_cycles`` SM cycles and it records the timeout status in
+    ``status`` (a device int32/uint32 word) instead of hanging. Returns C (unspecified)."""
+    M, Kd = A.shape
+    N = W.shape[0]
+    C = torch.empty((M, N), dtype=torch.float32, device=A.device)
+    _check(lib().lilicorr_test_linear_timeout(A.data_ptr(), W.data_ptr(), C.data_ptr(), M, N, Kd,
+                                              int(wait_cycles), status.data_ptr(), _stream()),
+           "test_linear_timeout")
     return C
 
 

@@ -856,6 +856,18 @@ lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int
   return LILICORR_ERR_ARG;
 }
 
+lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, float* C, int M, int N,
+                                               int Kd, long long wait_cycles, uint32_t* status,
+                                               cudaStream_t stream) {
+  if (!A || !W || !C || !status || M <= 0 || N <= 0 || Kd <= 0) return LILICORR_ERR_ARG;
+  if (wait_cycles < 100000 || wait_cycles > 4000000000ll) return LILICORR_ERR_ARG;
+  GemmArgs g = gemm(A, LILICORR_BF16, Kd, W, LILICORR_BF16, Kd, C, LILICORR_F32, N, M, N, Kd);
+  g.status = status;
+  g.wait_limit = wait_cycles;
+  g.test_starve = 1;
+  return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_SHAPE;
+}
+
 int lilicorr_test_attention_path(int mode) {
   const int prev = g_attn_umma;
   g_attn_umma = mode ? 1 : 0;

@@ -15,9 +15,10 @@
 //     per-sequence bias / SiLU / the residual (brought in by a TMA load), write the
 //     chunk into a 128-byte-swizzled staging buffer and store it with one TMA bulk
 //     tensor store (double-buffered staging and residual buffers).
-// Every mbarrier wait is bounded (about 2 s of SM cycles); on timeout the kernel records
-// LILICORR_ERR_TIMEOUT in the status word, stops issuing work while keeping every
-// thread on its barriers, lets copies in flight land, frees its tensor memory, returns.
+// Every mbarrier wait is bounded (about 2 s of SM cycles, or a shorter limit a test hook
+// sets); on timeout the kernel records LILICORR_ERR_TIMEOUT in the status word, stops
+// issuing work while keeping every thread on its barriers, lets copies in flight land,
+// frees its tensor memory, returns.
 #include "tc_ptx.cuh"
 
 namespace lilicorr {
@@ -73,7 +74,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                    const __grid_constant__ CUtensorMap mapW,
                    const __grid_constant__ CUtensorMap mapC,
                    const __grid_constant__ CUtensorMap mapR, TcEpilogue ep, int M, int N, int Kd,
-                   uint32_t* status) {
+                   uint32_t* status, long long wait_limit, int starve) {
   using Cfg = TcCfg<BN, OUT_BF16>;
   constexpr int S = Cfg::STAGES, CH = Cfg::CH, NCH = Cfg::NCH;
   extern __shared__ uint8_t smem_raw[];
@@ -120,15 +121,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   pdl_wait();                      // inputs come from the preceding launch
 
   if (warp == 0) {
-    // ---- producer: TMA into the stage ring, tile after tile
-    if (lane == 0) {
+    // ---- producer: TMA into the stage ring, tile after tile (none at all under the
+    //      test hook that starves the consumers to exercise their bounded waits)
+    if (lane == 0 && !starve) {
       uint32_t g = 0;                            // k-blocks issued so far
       for (int t = blockIdx.x; t < tiles && !abort_flag; t += gridDim.x) {
         const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
         for (int i = 0; i < nk; ++i, ++g) {
           const int s = (int)(g % S);
           const uint32_t ph = (g / S) & 1u;
-          if (!mbar_wait(&empty[s], ph ^ 1u, WAIT_LIMIT_CYCLES)) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, wait_limit)) {
             abort_flag = 1;
             break;
           }
@@ -145,7 +147,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       uint32_t g = 0, lt = 0;
       for (int t = blockIdx.x; t < tiles && !abort_flag; t += gridDim.x, ++lt) {
         const uint32_t acc = lt & 1u, aph = (lt >> 1) & 1u;
-        if (!mbar_wait(&acc_empty[acc], aph ^ 1u, WAIT_LIMIT_CYCLES)) {
+        if (!mbar_wait(&acc_empty[acc], aph ^ 1u, wait_limit)) {
           abort_flag = 1;
           break;
         }
@@ -154,7 +156,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         for (int i = 0; i < nk; ++i, ++g) {
           const int s = (int)(g % S);
           const uint32_t ph = (g / S) & 1u;
-          if (!mbar_wait(&full[s], ph, WAIT_LIMIT_CYCLES)) {
+          if (!mbar_wait(&full[s], ph, wait_limit)) {
             abort_flag = 1;
             break;
           }
@@ -192,7 +194,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       epi_bar();                                  // s_bias free again
       for (int j = threadIdx.x - 64; j < BN; j += EPI_THREADS)
         s_bias[j] = (ep.bias && n0 + j < N) ? ep.bias[n0 + j] : 0.f;
-      if (!abort_flag && !mbar_wait(&acc_full[acc], (lt >> 1) & 1u, WAIT_LIMIT_CYCLES))
+      if (!abort_flag && !mbar_wait(&acc_full[acc], (lt >> 1) & 1u, wait_limit))
         abort_flag = 1;
       tc_fence_after();
       epi_bar();
@@ -230,7 +232,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           if (lane == 0) mbar_arrive(&acc_empty[acc]);
         }
         if (ep.has_residual && !abort_flag &&
-            !mbar_wait(&res_full[b], (cc >> 1) & 1u, WAIT_LIMIT_CYCLES))
+            !mbar_wait(&res_full[b], (cc >> 1) & 1u, wait_limit))
           abort_flag = 1;
 #pragma unroll
         for (int j = 0; j < HC; j += 4) {
@@ -292,7 +294,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       set_status(status, LILICORR_ERR_TIMEOUT);
       // let copies still in flight land before the shared memory is released
       const long long t0 = clock64();
-      while (clock64() - t0 < WAIT_LIMIT_CYCLES / 10) {
+      while (clock64() - t0 < wait_limit / 10) {
       }
     }
     __syncthreads();
@@ -330,8 +332,9 @@ lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   ep.act = g.act;
   const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  LL_TRY(launch_k(gemm_tc_kernel<BN, OUT_BF16>, grid, TC_THREADS, Cfg::SMEM, st, ma, mw, mc, mr, ep, g.M, g.N,
-                                                                     g.Kd, g.status));
+  const long long wait = g.wait_limit > 0 ? g.wait_limit : WAIT_LIMIT_CYCLES;
+  LL_TRY(launch_k(gemm_tc_kernel<BN, OUT_BF16>, grid, TC_THREADS, Cfg::SMEM, st, ma, mw, mc, mr, ep,
+                  g.M, g.N, g.Kd, g.status, wait, g.test_starve));
   return LILICORR_OK;
 }
 

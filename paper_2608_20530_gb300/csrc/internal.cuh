@@ -262,6 +262,9 @@ struct GemmArgs {
   int act;
   int M, N, Kd;
   uint32_t* status;        // device status word (bounded-wait timeouts), may be null
+  long long wait_limit;    // SM cycles per bounded wait of the tensor-core kernel; 0: ~2 s
+  int test_starve;         // test hook only: the tensor-core kernel's producer issues no
+                           // copies, so its consumers' waits run out (see the testing header)
 };
 lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
 lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st);   // M <= 64

@@ -7,6 +7,7 @@ after a tie sends the two walks different ways.
 """
 from __future__ import annotations
 
+import dataclasses
 import functools
 from typing import Dict, List, Tuple
 
@@ -27,17 +28,24 @@ def to_dev(a: np.ndarray, dtype: str, device="cuda"):
     return t.to(device)
 
 
-def compare_path(choice: np.ndarray, A: np.ndarray, P: np.ndarray, tol: float) -> Tuple[int, int]:
+@dataclasses.dataclass
+class PathCheck:
+    prefix: int       # steps where the GPU path equals the oracle's, from the start
+    ties: int         # tied steps along the GPU path (oracle runner-up within tol)
+    exact: int        # steps of the identical prefix that are not ties: a wrong
+                      # candidate there would have failed the comparison
+
+
+def check_path(choice: np.ndarray, A: np.ndarray, P: np.ndarray, tol: float) -> PathCheck:
     """Check the GPU's chosen path against the oracle's scores.
 
     (1) Every step, followed along the GPU's own path through the oracle's full score
         tensor, picks a candidate within ``tol`` of the best continuation of the GPU's
         previous choice (a valid greedy step, ties allowed).
     (2) Up to the first step where the two paths differ, they are identical, and that
-        step must be a tie (oracle runner-up within ``tol``).
-    Returns (length of the identical prefix, tied steps along the GPU path)."""
+        step must be a tie (oracle runner-up within ``tol``)."""
     L = len(choice)
-    ties = 0
+    ties = exact = 0
     prefix = None
     prev = None
     oprev = None
@@ -47,17 +55,25 @@ def compare_path(choice: np.ndarray, A: np.ndarray, P: np.ndarray, tol: float) -
         assert row.max() - row[c] <= tol, (
             f"step {s}: gpu picked {c} ({row[c]:.6f}), best continuation {row.max():.6f}")
         srt = np.sort(row)
-        if len(row) > 1 and srt[-1] - srt[-2] <= tol:
-            ties += 1
+        tied = len(row) > 1 and srt[-1] - srt[-2] <= tol
+        ties += int(tied)
         if prefix is None:
             orow = np.asarray(A if s == 0 else P[s - 1, oprev], dtype=np.float64)
             ob = int(np.argmax(orow))
             if ob != c:
                 assert orow.max() - orow[c] <= tol
                 prefix = s
+            else:
+                exact += int(not tied)
             oprev = ob
         prev = c
-    return (L if prefix is None else prefix), ties
+    return PathCheck(L if prefix is None else prefix, ties, exact)
+
+
+def compare_path(choice: np.ndarray, A: np.ndarray, P: np.ndarray, tol: float) -> Tuple[int, int]:
+    """check_path's (identical prefix length, tied steps)."""
+    r = check_path(choice, A, P, tol)
+    return r.prefix, r.ties
 
 
 @functools.lru_cache(maxsize=2)

@@ -7,6 +7,7 @@ import torch
 
 import oracle
 import workloads
+import _oracle_pool
 from _helpers import TOL_VEC, embed_fn, to_dev, workload_data
 
 pytestmark = pytest.mark.gpu
@@ -57,25 +58,35 @@ def test_tiny_f32_head():
     _check_head(wl, W, inp, ids, logp, range(wl.B))
 
 
-@pytest.mark.parametrize("name", ["serving_b32", "ties_b256"])
-def test_bf16_heads_sampled_sequences(name):
-    wl, W, inp = workload_data(name)
-    # top-K of every sequence by the oracle is slow at full size; sampled sequences use
-    # the oracle's ids, the rest use a cheap argpartition (their vectors are not checked)
-    B = wl.B
-    ids = np.zeros((B, wl.L, wl.K), np.int64)
-    logp = np.zeros((B, wl.L, wl.K))
-    seqs = [0, B - 1]
-    x = inp["logits"]
-    for b in range(B):
-        if b in seqs:
-            for s in range(wl.L):
-                ids[b, s], logp[b, s], _ = oracle.topk_lse(x[b, s], wl.K)
-        else:
-            part = np.argpartition(-x[b], wl.K, axis=1)[:, :wl.K]
-            ids[b] = part
-            logp[b] = -np.arange(wl.K, dtype=float)
-    _check_head(wl, W, inp, ids, logp, seqs)
+@pytest.mark.parametrize("name,tier", [("serving_b32", 0), ("entropy_tiers_b64", 2),
+                                       ("ties_b256", 0)])
+def test_bf16_heads_every_sequence(name, tier):
+    """The oracle's own top-K of every sequence feeds both sides; every sequence's
+    vectors are compared (the oracle network fanned out over the host cores)."""
+    wl, W, inp = workload_data(name, tier)
+    seeds = wl.seeds(tier)
+    ids, logp, _ = _oracle_pool.topk(wl, seeds, tier)
+    lp32 = logp.astype(np.float32).astype(np.float64)    # what the GPU receives
+    refs = _oracle_pool.network(wl, seeds, ids, lp32, tier)
+    ll = _ll()
+    head = ll.Head.from_workload(wl, W, workloads.embed_table(wl.V, wl.H, wl.dtype))
+    try:
+        out, inn, anc = ll.embed_in_out(head, to_dev(ids.astype(np.int32), "f32"),
+                                        to_dev(logp.astype(np.float32), "f32"),
+                                        to_dev(inp["hidden"], wl.dtype),
+                                        to_dev(inp["target"], wl.dtype))
+        torch.cuda.synchronize()
+    finally:
+        head.close()
+    out, inn, anc = out.cpu().numpy(), inn.cpu().numpy(), anc.cpu().numpy()
+    tol = TOL_VEC[wl.dtype]
+    worst = 0.0
+    for b, r in enumerate(refs):
+        e = max(np.abs(out[b] - r["out"]).max(), np.abs(inn[b] - r["in"]).max(),
+                np.abs(anc[b] - r["anchor"]).max())
+        assert e <= tol, (b, e)
+        worst = max(worst, e)
+    print(f"{name} tier {tier}: {len(refs)} sequences, worst vector error {worst:.2e}")
 
 
 def test_max_nodes_fp32_head():

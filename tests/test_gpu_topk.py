@@ -1,11 +1,14 @@
 """GPU parity of step (1), top-K + log-normaliser (Sec. 3.2; App. A "Serving"), against
-the oracle: ids bit-exact, log-probs and log-normaliser within 1e-3."""
+the oracle: ids bit-exact, log-probs and log-normaliser within 1e-3, on every row of
+every full-size workload (the oracle fanned out over the host cores) and on ragged,
+tied, -0/-inf and non-finite rows."""
 import numpy as np
 import pytest
 import torch
 
 import oracle
 import workloads
+import _oracle_pool
 from _helpers import TOL_LOGP, to_dev, workload_data
 
 pytestmark = pytest.mark.gpu
@@ -51,21 +54,50 @@ def test_tiny_workload_all_rows():
     _check_rows(x, wl.K, ids, logp, lse, range(x.shape[0]))
 
 
-@pytest.mark.parametrize("name,tier", [("single_request", 0), ("serving_b32", 0),
-                                       ("entropy_tiers_b64", 0), ("entropy_tiers_b64", 1),
-                                       ("entropy_tiers_b64", 2), ("ties_b256", 0)])
-def test_full_size_workloads_sampled_rows(name, tier):
+def _check_all(ids, logp, lse, oids, ologp, olse):
+    """Every row: ids bit-exact, log-probs and normaliser within 1e-3."""
+    bad = np.nonzero(~np.all(ids == oids, axis=-1))[0]
+    assert bad.size == 0, f"{bad.size} rows differ, first {bad[0]}: {ids[bad[0]]} vs {oids[bad[0]]}"
+    assert np.abs(lse - olse).max() <= TOL_LOGP
+    assert np.abs(logp - ologp).max() <= TOL_LOGP
+
+
+@pytest.mark.parametrize("name,tier", [("serving_b32", 0), ("entropy_tiers_b64", 0),
+                                       ("entropy_tiers_b64", 1), ("entropy_tiers_b64", 2),
+                                       ("ties_b256", 0)])
+def test_full_size_workloads_every_row(name, tier):
+    """One call over the whole batch (the launch of the batched selection), every row
+    against the oracle's full sort."""
     wl, _, inp = workload_data(name, tier)
     x = inp["logits"].reshape(-1, wl.V)
     ids, logp, lse, st = _run(x, wl.K, wl.dtype)
     assert st == 0
-    rng = np.random.default_rng(17)
-    rows = sorted(set([0, x.shape[0] - 1] + list(rng.integers(0, x.shape[0], 6))))
-    _check_rows(x, wl.K, ids, logp, lse, rows)
-    # every row: ids sorted by (logit desc, id asc) and logp consistent with lse
-    xv = np.take_along_axis(x, ids.astype(np.int64), axis=1)
-    assert np.all(np.diff(xv, axis=1) <= 0)
-    assert np.allclose(logp, xv - lse[:, None], atol=1e-5)
+    oids, ologp, olse = _oracle_pool.topk(wl, wl.seeds(tier), tier)
+    _check_all(ids, logp, lse, oids.reshape(ids.shape), ologp.reshape(logp.shape),
+               olse.reshape(lse.shape))
+
+
+def test_single_request_every_block():
+    """All 1000 blocks of the batch-1 workload, each its own 16-row call (the split-row
+    launch the batch-1 selection makes), against the oracle."""
+    ll = _ll()
+    wl = workloads.WORKLOADS["single_request"]
+    seeds = wl.block_seeds()
+    oids, ologp, olse = _oracle_pool.topk(wl, seeds)
+    ws = ll.Workspace(ll.lib().lilicorr_topk_lse_workspace_bytes(wl.L, wl.V, wl.K))
+    got = []
+    for i0 in range(0, len(seeds), 100):
+        inp = workloads.batch_inputs(wl, seeds[i0:i0 + 100])
+        t = to_dev(inp["logits"], wl.dtype)
+        outs = [ll.topk_lse(t[j], wl.K, ws=ws) for j in range(t.shape[0])]
+        torch.cuda.synchronize()
+        got += [[o.cpu().numpy() for o in r] for r in outs]
+        del t, inp
+    assert ws.status() == 0
+    ids = np.stack([g[0] for g in got])
+    logp = np.stack([g[1] for g in got])
+    lse = np.stack([g[2] for g in got])
+    _check_all(ids, logp, lse, oids, ologp, olse)
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])

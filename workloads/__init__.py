@@ -32,6 +32,7 @@ N_TGT_LAYERS = 5       # captured target layers (App. A "Architecture")
 N_LAYERS = 2           # scoring Transformer layers (Table "hparams")
 N_HEADS = 8            # attention heads (Table "hparams")
 WEIGHT_STD = 0.02
+UNIT_EMBED_STD = 1.0   # the wide-margin parity case: token embeddings at the hidden states' scale
 
 
 @dataclasses.dataclass(frozen=True)
@@ -234,32 +235,34 @@ def head_weights(wl: Workload, seed: int = WEIGHT_SEED) -> Dict[str, np.ndarray]
 
 
 # --------------------------------------------------------------------------- embedding table
-def _embed_chunk(V: int, H: int, c: int, seed: int) -> np.ndarray:
+def _embed_chunk(V: int, H: int, c: int, seed: int, std: float = WEIGHT_STD) -> np.ndarray:
     r0 = c * EMBED_CHUNK_ROWS
     n = min(EMBED_CHUNK_ROWS, V - r0)
     rng = np.random.default_rng(np.random.PCG64([seed, c]))
-    return rng.standard_normal((n, H), dtype=np.float32) * np.float32(WEIGHT_STD)
+    return rng.standard_normal((n, H), dtype=np.float32) * np.float32(std)
 
 
-_EMBED_CACHE: Dict[Tuple[int, int, str, int], np.ndarray] = {}
+_EMBED_CACHE: Dict[Tuple[int, int, str, int, float], np.ndarray] = {}
 
 
-def embed_table(V: int, H: int, dtype: str, seed: int = EMBED_SEED) -> np.ndarray:
-    """Frozen token-embedding table [V, H] ~ N(0, 0.02).
+def embed_table(V: int, H: int, dtype: str, seed: int = EMBED_SEED,
+                std: float = WEIGHT_STD) -> np.ndarray:
+    """Frozen token-embedding table [V, H] ~ N(0, std) (std 0.02 by default, like the
+    head's weights; ``UNIT_EMBED_STD`` for the wide-margin parity case).
 
     Returned as bf16 bit patterns (uint16) for ``dtype == "bf16"`` and float32
     otherwise. Rows are drawn in chunks of EMBED_CHUNK_ROWS with per-chunk seeds,
     so ``embed_rows`` can regenerate any row without the full table. The last
     table built is cached in-process.
     """
-    key = (V, H, dtype, seed)
+    key = (V, H, dtype, seed, float(std))
     if key in _EMBED_CACHE:
         return _EMBED_CACHE[key]
     nchunks = (V + EMBED_CHUNK_ROWS - 1) // EMBED_CHUNK_ROWS
     out = np.empty((V, H), dtype=np.uint16 if dtype == "bf16" else np.float32)
 
     def fill(c: int) -> None:
-        a = _embed_chunk(V, H, c, seed)
+        a = _embed_chunk(V, H, c, seed, std)
         r0 = c * EMBED_CHUNK_ROWS
         out[r0:r0 + a.shape[0]] = bf16_bits(a) if dtype == "bf16" else a
 
@@ -270,16 +273,17 @@ def embed_table(V: int, H: int, dtype: str, seed: int = EMBED_SEED) -> np.ndarra
     return out
 
 
-def embed_rows(V: int, H: int, dtype: str, ids: np.ndarray, seed: int = EMBED_SEED) -> np.ndarray:
+def embed_rows(V: int, H: int, dtype: str, ids: np.ndarray, seed: int = EMBED_SEED,
+               std: float = WEIGHT_STD) -> np.ndarray:
     """Rows ``ids`` of the embedding table as float32 values, regenerated per chunk."""
     ids = np.asarray(ids, dtype=np.int64).reshape(-1)
-    key = (V, H, dtype, seed)
+    key = (V, H, dtype, seed, float(std))
     if key in _EMBED_CACHE:
         t = _EMBED_CACHE[key][ids]
         return bf16_bits_to_f32(t) if dtype == "bf16" else t.astype(np.float32)
     rows = np.empty((ids.size, H), dtype=np.float32)
     for c in np.unique(ids // EMBED_CHUNK_ROWS):
-        a = _embed_chunk(V, H, int(c), seed)
+        a = _embed_chunk(V, H, int(c), seed, std)
         a = round_to_bf16(a) if dtype == "bf16" else a
         sel = np.nonzero(ids // EMBED_CHUNK_ROWS == c)[0]
         rows[sel] = a[ids[sel] - c * EMBED_CHUNK_ROWS]
