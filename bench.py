@@ -59,6 +59,8 @@ def parse_args():
                    help="distinct batches per step (batched workloads; default: up to 8, "
                         "about 1.6 GB of logits)")
     p.add_argument("--e2e-host-blocks", type=int, default=64)
+    p.add_argument("--copy-streams", type=int, default=2,
+                   help="streams the end-to-end host-to-device copies are spread over")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-by-workload", dest="by_workload", action="store_false",
                    help="skip the batched workloads' section of the default run")
@@ -397,7 +399,7 @@ def roofline_fracs(wl, B, us_call, us_topk, pk):
     }
 
 
-def bench_batched(ll, name, tier, dev, stream, E, pk, rank, min_bytes=6e8, reps=5):
+def bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams, min_bytes=6e8, reps=5):
     """One batched workload (one tier) through select_block: device-timed calls over
     distinct resident batches (inputs larger than L2), the top-K pass alone, and the
     same calls end to end from pinned host buffers."""
@@ -426,22 +428,18 @@ def bench_batched(ll, name, tier, dev, stream, E, pk, rank, min_bytes=6e8, reps=
     ll.topk_lse(flat[0], wl.K, ws=tk_ws)
     tg = graph_of([lambda j=j: ll.topk_lse(flat[j], wl.K, ws=tk_ws) for j in range(nb)] * 2)
     us_topk = time_replays([tg], stream, reps) * 1e3 / (2 * nb)
-    # end to end: each call copies its batch from pinned host memory and its tokens back
-    h_l = logits.cpu().pin_memory()
-    h_h = hidden.cpu().pin_memory()
-    h_t = target.cpu().pin_memory()
+    # end to end: each call copies its batch from pinned host memory and its tokens back,
+    # the next call's copies overlapping this call's compute
+    h_in = [logits.cpu().pin_memory(), hidden.cpu().pin_memory(), target.cpu().pin_memory()]
     h_tok = torch.empty((nb, B, wl.L), dtype=torch.int32).pin_memory()
-    d_l, d_h, d_t = torch.empty_like(logits[0]), torch.empty_like(hidden[0]), torch.empty_like(target[0])
-    d_tok = torch.empty((B, wl.L), dtype=torch.int32, device=dev)
-
-    def e2e_call(j):
-        d_l.copy_(h_l[j], non_blocking=True)
-        d_h.copy_(h_h[j], non_blocking=True)
-        d_t.copy_(h_t[j], non_blocking=True)
-        ll.select_block(head, d_l, d_h, d_t, ws=ws, tokens=d_tok)
-        h_tok[j].copy_(d_tok, non_blocking=True)
-    eg = graph_of([lambda j=j: e2e_call(j) for j in range(nb)])
-    us_e2e = time_replays([eg], stream, max(2, reps // 2), warm=1) * 1e3 / nb
+    d_in = [[torch.empty_like(t[0]) for t in (logits, hidden, target)] for _ in range(2)]
+    d_tok = [torch.empty((B, wl.L), dtype=torch.int32, device=dev) for _ in range(2)]
+    n_e2e = max(nb, 4)
+    eg = pipelined_e2e_graph(
+        lambda x, tok: ll.select_block(head, x[0], x[1], x[2], ws=ws, tokens=tok),
+        h_in, d_in, h_tok, d_tok, [j % nb for j in range(n_e2e)], copy_streams)
+    us_e2e = time_replays([eg], stream, max(2, reps // 2), warm=1) * 1e3 / n_e2e
+    d_l, d_h, d_t = d_in[0]
     if ws.status() != 0 or tk_ws.status() != 0:
         raise RuntimeError(f"{name}: device status set")
     h2d = (d_l.numel() + d_h.numel() + d_t.numel()) * es
@@ -453,10 +451,83 @@ def bench_batched(ll, name, tier, dev, stream, E, pk, rank, min_bytes=6e8, reps=
                    "sequences_per_s": round(B / (us_e2e * 1e-6), 1),
                    "h2d_bytes_per_call": h2d, "d2h_bytes_per_call": B * wl.L * 4}}
     out.update(roofline_fracs(wl, B, us_call, us_topk, pk))
+    out["walk"] = walk_latency(ll, head, logits[0], hidden[0], target[0], ws, B, stream)
     head.close()
-    del logits, hidden, target, h_l, h_h, h_t, flat
+    del logits, hidden, target, h_in, d_in, flat
     torch.cuda.empty_cache()
     return out
+
+
+def pipelined_e2e_graph(select, h_in, d_in, h_tok, d_tok, order, copy_streams):
+    """One CUDA graph of len(order) end-to-end calls: call j copies host item order[j]
+    (pinned tensors h_in[k][i]) into device buffer set j % 2 on the copy streams, runs
+    ``select(inputs, tokens)`` on the capturing stream once its copies have landed, and
+    copies the tokens back to h_tok[i]. The copies of call j + 1 run while call j computes
+    (a buffer set is refilled only after the call two back has finished with it); the
+    logits, the largest input, are split across the copy streams."""
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        s0 = torch.cuda.current_stream()
+        start = torch.cuda.Event()
+        start.record(s0)
+        for cs in copy_streams:
+            cs.wait_event(start)
+        done = []
+        nc = len(copy_streams)
+        for j, i in enumerate(order):
+            b = j % 2
+            landed = []
+            for k, cs in enumerate(copy_streams):
+                with torch.cuda.stream(cs):
+                    if j >= 2:
+                        cs.wait_event(done[j - 2])
+                    for t, (h, d) in enumerate(zip(h_in, d_in[b])):
+                        if t == 0:          # logits: one slice of rows per copy stream
+                            hv, dv = h[i].view(-1, h.shape[-1]), d.view(-1, d.shape[-1])
+                            r0 = hv.shape[0] * k // nc
+                            r1 = hv.shape[0] * (k + 1) // nc
+                            if r1 > r0:
+                                dv[r0:r1].copy_(hv[r0:r1], non_blocking=True)
+                        elif k == t % nc:
+                            d.copy_(h[i], non_blocking=True)
+                    e = torch.cuda.Event()
+                    e.record(cs)
+                    landed.append(e)
+            for e in landed:
+                s0.wait_event(e)
+            select(d_in[b], d_tok[b])
+            h_tok[i].copy_(d_tok[b], non_blocking=True)
+            e = torch.cuda.Event()
+            e.record(s0)
+            done.append(e)
+        for cs in copy_streams:
+            e = torch.cuda.Event()
+            e.record(cs)
+            s0.wait_event(e)
+    return g
+
+
+def walk_latency(ll, head, logits, hidden, target, ws, B, stream, n=50):
+    """Steps (3) and (4) on their own, after one selection: the pair-score kernel on the
+    call's unit vectors, the greedy walk and the exact best path on its scores, each
+    captured n times in a graph (us per launch, launch overhead included)."""
+    ll.select_block(head, logits, hidden, target, ws=ws)
+    inter = ll.select_block_intermediates(head, B, ws)
+    ids, logp = inter["ids"].clone(), inter["logp"].clone()
+    out, inn, anc = ll.embed_in_out(head, ids, logp, hidden, target)
+    A, P = ll.pair_scores(out, inn, anc)
+    ll.greedy_walk(A, P, ids)
+    ll.best_path(A, P, ids)
+    torch.cuda.synchronize()
+
+    def per_call(fn):
+        return round(time_replays([graph_of([fn] * n)], stream, 3, warm=1) * 1e3 / n, 2)
+    return {"pair_scores_us": per_call(lambda: ll.pair_scores(out, inn, anc)),
+            "greedy_walk_us": per_call(lambda: ll.greedy_walk(A, P, ids)),
+            "best_path_us": per_call(lambda: ll.best_path(A, P, ids)),
+            "note": f"standalone launches on one call's outputs (B = {B}), {n} per graph; in "
+                    "select_block the cluster network kernel forms the pair scores and walks "
+                    "in its own tail (no launch), elsewhere the pair kernel walks in its last CTA"}
 
 
 BATCHED = [("serving_b32", 0), ("entropy_tiers_b64", 0), ("entropy_tiers_b64", 1),
@@ -539,29 +610,23 @@ def run_ours(args, world, rank, local, pool):
     if ws.status() != 0:
         raise RuntimeError("device status set during the timed region")
 
-    # ---- end to end: pinned host inputs -> device -> select -> tokens back to pinned host
+    # ---- end to end: pinned host inputs -> device -> select -> tokens back to pinned host;
+    # each graph holds G calls, the next call's copies overlapping this call's compute
     nh = min(args.e2e_host_blocks, nblk)
-    h_logits = logits[:nh].cpu().pin_memory()
-    h_hidden = hidden[:nh].cpu().pin_memory()
-    h_target = target[:nh].cpu().pin_memory()
+    h_in = [logits[:nh].cpu().pin_memory(), hidden[:nh].cpu().pin_memory(),
+            target[:nh].cpu().pin_memory()]
     h_tokens = torch.empty((nh, B, wl.L), dtype=torch.int32).pin_memory()
-    d_logits = torch.empty_like(logits[0])
-    d_hidden = torch.empty_like(hidden[0])
-    d_target = torch.empty_like(target[0])
-    d_tokens = torch.empty((B, wl.L), dtype=torch.int32, device=dev)
-
-    def e2e_call(i):
-        d_logits.copy_(h_logits[i], non_blocking=True)
-        d_hidden.copy_(h_hidden[i], non_blocking=True)
-        d_target.copy_(h_target[i], non_blocking=True)
-        ll.select_block(head, d_logits, d_hidden, d_target, ws=ws, tokens=d_tokens)
-        h_tokens[i].copy_(d_tokens, non_blocking=True)
-
-    # each e2e graph holds G calls, each: its inputs host -> device, select, tokens -> host
-    e2e_graphs = [graph_of([lambda i=(k * G + j) % nh: e2e_call(i) for j in range(G)])
+    d_in = [[torch.empty_like(t[0]) for t in (logits, hidden, target)] for _ in range(2)]
+    d_tok = [torch.empty((B, wl.L), dtype=torch.int32, device=dev) for _ in range(2)]
+    copy_streams = [torch.cuda.Stream() for _ in range(args.copy_streams)]
+    sel = lambda x, tok: ll.select_block(head, x[0], x[1], x[2], ws=ws, tokens=tok)
+    e2e_graphs = [pipelined_e2e_graph(sel, h_in, d_in, h_tokens, d_tok,
+                                      [(k * G + j) % nh for j in range(G)], copy_streams)
                   for k in range(-(-nh // G))]
     n_e2e_replays = -(-nblk // G)
     e2e_calls = n_e2e_replays * G
+    d_logits, d_hidden, d_target = d_in[0]
+    d_tokens = d_tok[0]
 
     def e2e_step():
         for r in range(n_e2e_replays):
@@ -584,7 +649,7 @@ def run_ours(args, world, rank, local, pool):
     h2d = (d_logits.numel() * d_logits.element_size() + d_hidden.numel() * d_hidden.element_size()
            + d_target.numel() * d_target.element_size()) * e2e_calls
     d2h = d_tokens.numel() * 4 * e2e_calls
-    del h_logits, h_hidden, h_target, e2e_graphs
+    del h_in, e2e_graphs
 
     # ---- the exact best path (App. E) in place of the greedy walk: the same calls on a
     # sample of the blocks, both walks captured alike and timed back to back
@@ -598,6 +663,7 @@ def run_ours(args, world, rank, local, pool):
                             for k in range(3)) / nv
     if ws.status() != 0:
         raise RuntimeError("device status set by the walk comparison")
+    walk = walk_latency(ll, head, logits[0], hidden[0], target[0], ws, B, stream)
 
     # ---- diagnostics of the chosen blocks (Eq. "localar" probabilities and gaps along the
     # walk; coverage / oracle prefix / accepted prefix against the planted tokens)
@@ -720,7 +786,7 @@ def run_ours(args, world, rank, local, pool):
         by_workload = {}
         for name, tier in BATCHED:
             key = name if not workloads.WORKLOADS[name].tiers else f"{name}.tau{workloads.WORKLOADS[name].tiers[tier]}"
-            by_workload[key] = bench_batched(ll, name, tier, dev, stream, E, pk, rank)
+            by_workload[key] = bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams)
         by_workload["clocks"] = bclk.stop()
         by_workload["note"] = ("each: select_block over distinct resident batches (>= 0.6 GB of "
                                "logits, larger than L2) in one CUDA graph, CUDA events; topk_* = "
@@ -743,7 +809,9 @@ def run_ours(args, world, rank, local, pool):
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
-                "note": f"pinned host blocks cycled ({nh} distinct), copies captured with each call"},
+                "note": f"pinned host blocks cycled ({nh} distinct); each call's copies (logits "
+                        f"split over {args.copy_streams} copy streams) captured with it, "
+                        f"overlapping the previous call's compute"},
         "gpu_launches": launches_per_call * nblk * args.steps,
         "roofline": roofline,
         "by_workload": by_workload,
@@ -752,6 +820,7 @@ def run_ours(args, world, rank, local, pool):
                          "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
                          "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
                          "sample": f"{nv} calls of this workload, best of 3"},
+        "walk": walk,
         "vocab_sharded": sharded,
         "lm_head_fused": lm_head,
     }
