@@ -196,6 +196,7 @@ namespace lilicorr {
 // ----------------------------------------------------------------------------- workspace
 struct TopkPlan {
   int splits;          // CTAs per row
+  int threads;         // threads per CTA
   int chunk_vecs;      // 16-byte vectors per split
   size_t rec_bytes;    // bytes of one partial record
 };

@@ -4,7 +4,8 @@
 // extraction with vocabulary-wide logit normalisation. Here every logit is read
 // from HBM exactly once:
 //   * grid = (splits, rows): each CTA streams one contiguous chunk of one row with
-//     16-byte loads, a batch of 4 per thread in flight;
+//     16-byte loads in batches of 4 per thread, the next batch's loads in flight while
+//     the current one is reduced;
 //   * every thread keeps an online (max, sum exp) pair, merged by warp shuffles;
 //   * candidates are order-preserving 64-bit keys (value, then lower id first). Each
 //     warp appends the elements that reach its value bound to a key buffer in shared
@@ -32,8 +33,8 @@ namespace lilicorr {
 
 namespace {
 
-constexpr int TK_THREADS = 256;
-constexpr int TK_WARPS = TK_THREADS / 32;
+constexpr int TK_THREADS = 256;        // CTA size of the few-row plan and of the merges
+constexpr int TK_THREADS_MANY = 128;   // CTA size when the rows alone fill the GPU
 constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch
 constexpr int TK_MAX_SPLITS = 64;
 constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
@@ -100,7 +101,8 @@ __device__ __forceinline__ void rank_place(const uint64_t* keys, int n, int K, u
 // K largest of groups[g][0..K) for g < ngroups (each group sorted descending, zeros =
 // empty), CTA-wide. Every group's K-th key bounds the answer's K-th from below, so only
 // keys >= the largest such bound survive; they are compacted and rank-counted.
-// surv: scratch of TK_MERGE_MAX keys; out[0..K) receives the result. All threads call.
+// surv: scratch of TK_MERGE_MAX keys; out[0..K) receives the result. All NT threads call.
+template <int NT>
 __device__ void cta_select(const uint64_t* groups, int ngroups, int stride, int K, uint64_t* surv,
                            int* s_count, uint64_t* s_bound, uint64_t* out) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -117,15 +119,15 @@ __device__ void cta_select(const uint64_t* groups, int ngroups, int stride, int 
     }
     if (lane == 0) { *s_bound = b; *s_count = 0; }
   }
-  for (int i = tid; i < K; i += TK_THREADS) out[i] = 0ull;
+  for (int i = tid; i < K; i += NT) out[i] = 0ull;
   __syncthreads();
   const uint64_t bound = *s_bound;
-  for (int i = tid; i < ngroups * K; i += TK_THREADS) {
+  for (int i = tid; i < ngroups * K; i += NT) {
     const uint64_t k = groups[(size_t)(i / K) * stride + i % K];
     if (k != 0ull && k >= bound) surv[atomicAdd(s_count, 1)] = k;
   }
   __syncthreads();
-  rank_place(surv, *s_count, K, out, tid, TK_THREADS);
+  rank_place(surv, *s_count, K, out, tid, NT);
   __syncthreads();
 }
 
@@ -263,32 +265,61 @@ __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], ui
   }
 }
 
-// One batch: TK_UNROLL 16-byte vectors per thread (vectors it + u*TK_THREADS + tid).
-// CHECK = false: every vector is inside the chunk (no predicates). The values stay in
-// registers; the online (max, sum exp) takes one rescale check per batch; the warp looks
-// at the values for candidates only if some lane's batch maximum reaches the bound.
-// s_wtop[warp]: the warps' published r-th largest lane maxima (r = ceil(K / TK_WARPS)).
-template <typename T, bool CHECK>
-__device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int it, int v_end,
+// A batch: TK_UNROLL 16-byte vectors per thread (vectors it + u*NT + tid, NT threads).
+// CHECK = false: every vector is inside the chunk (no predicates); otherwise vectors past
+// v_end read as -inf, which adds nothing to the sum and never becomes a candidate.
+template <typename T, int NT, bool CHECK>
+__device__ __forceinline__ void load_batch(const uint4* __restrict__ vp, int it, int v_end, int tid,
+                                           uint4 (&raw)[TK_UNROLL]) {
+  constexpr uint32_t NI = Vec<T>::NEG_INF4;
+#pragma unroll
+  for (int u = 0; u < TK_UNROLL; ++u) {
+    const int v = it + u * NT + tid;
+    raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(NI, NI, NI, NI);
+  }
+}
+
+// The sum of exp(x - m) over one 16-byte vector, added into two packed accumulators (the
+// values are unpacked pair by pair, so the raw words stay the only copy in registers).
+template <typename T>
+__device__ __forceinline__ void exp_vec(const uint4& r, uint64_t l2, uint64_t nm, uint64_t& a0,
+                                        uint64_t& a1) {
+  const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+  if constexpr (sizeof(T) == 2) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float t0, t1;
+      unpack2(fma2(pack2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xFFFF0000u)), l2, nm),
+              t0, t1);
+      const uint64_t e = pack2(ex2(t0), ex2(t1));
+      if (i & 1) a1 = add2(a1, e); else a0 = add2(a0, e);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; i += 2) {
+      float t0, t1;
+      unpack2(fma2(pack2(__uint_as_float(w[i]), __uint_as_float(w[i + 1])), l2, nm), t0, t1);
+      const uint64_t e = pack2(ex2(t0), ex2(t1));
+      if ((i >> 1) & 1) a1 = add2(a1, e); else a0 = add2(a0, e);
+    }
+  }
+}
+
+// Reduce one loaded batch: the online (max, sum exp) with one rescale check per batch, then
+// the candidates, which the warp looks at only if some lane's batch maximum reaches the
+// bound. s_wtop[warp]: the warps' published r-th largest lane maxima (r = ceil(K / warps)).
+template <typename T, int NT, bool CHECK>
+__device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int it, int v_end,
                                               uint32_t id_base, int K, int tid, int lane,
                                               float& m, float& s, WarpCand& w,
                                               uint32_t* s_cta_thr, float* s_wtop) {
   constexpr int VEC = Vec<T>::N;
-  uint4 raw[TK_UNROLL];
-#pragma unroll
-  for (int u = 0; u < TK_UNROLL; ++u) {
-    const int v = it + u * TK_THREADS + tid;
-    constexpr uint32_t NI = Vec<T>::NEG_INF4;          // outside the chunk: contributes nothing
-    raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(NI, NI, NI, NI);
-  }
-  float x[TK_UNROLL][VEC];
   float vmx[TK_UNROLL];
   float bmax = -INFINITY;
 #pragma unroll
   for (int u = 0; u < TK_UNROLL; ++u) {
     vmx[u] = Vec<T>::vmax(raw[u]);
     bmax = fmaxf(bmax, vmx[u]);
-    Vec<T>::unpack(raw[u], x[u]);
   }
   // online log-sum-exp, one rescale per batch (rarely taken after the first batches)
   if (bmax > m) {
@@ -300,14 +331,7 @@ __device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int 
     const uint64_t l2 = pack2(LOG2E, LOG2E), nm = pack2(-ml, -ml);
     uint64_t a0 = pack2(0.f, 0.f), a1 = a0;
 #pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u)
-#pragma unroll
-      for (int j = 0; j < VEC; j += 2) {
-        float t0, t1;
-        unpack2(fma2(pack2(x[u][j], x[u][j + 1]), l2, nm), t0, t1);
-        const uint64_t e = pack2(ex2(t0), ex2(t1));
-        if ((j >> 1) & 1) a1 = add2(a1, e); else a0 = add2(a0, e);
-      }
+    for (int u = 0; u < TK_UNROLL; ++u) exp_vec<T>(raw[u], l2, nm, a0, a1);
     float p0, p1, p2, p3;
     unpack2(a0, p0, p1);
     unpack2(a1, p2, p3);
@@ -318,14 +342,15 @@ __device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int 
   if (!__any_sync(FULL, bmax >= w.thr)) return;
   {
     // the CTA-wide bound from the warps' published lane maxima
-    const int r = (K + TK_WARPS - 1) / TK_WARPS;
+    constexpr int NW = NT / 32;
+    const int r = (K + NW - 1) / NW;
     const float mine = r == 1 ? warp_max(m) : warp_kth_largest(m, r, lane);
     volatile float* wtop = s_wtop;
     if (lane == 0) wtop[tid >> 5] = mine;             // lane maxima only grow
     __syncwarp();
     float cb = INFINITY;
 #pragma unroll
-    for (int i = 0; i < TK_WARPS; ++i) cb = fminf(cb, wtop[i]);
+    for (int i = 0; i < NW; ++i) cb = fminf(cb, wtop[i]);
     if (cb > w.thr) {
       w.thr = cb;
       if (lane == 0) atomicMax(s_cta_thr, ord32(cb));
@@ -343,12 +368,40 @@ __device__ __forceinline__ void process_batch(const uint4* __restrict__ vp, int 
 #pragma unroll
   for (int u = 0; u < TK_UNROLL; ++u) {
     if (!__any_sync(FULL, vmx[u] >= w.thr)) continue;
-    const int v = it + u * TK_THREADS + tid;
-    warp_append<VEC>(w, x[u], id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
+    const int v = it + u * NT + tid;
+    float x[VEC];
+    Vec<T>::unpack(raw[u], x);
+    warp_append<VEC>(w, x, id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
   }
   if (w.n >= 2 * K) {                                  // the buffer's K-th key bounds it
     warp_compact(w, K, lane);
     if (lane == 0) atomicMax(s_cta_thr, ord32(w.thr));
+  }
+}
+
+// Stream vectors [v_begin, v_end) through process_batch with the next batch's loads in
+// flight while the current one is reduced; full batches in the loop, the ragged last one
+// after it.
+template <typename T, int NT>
+__device__ __forceinline__ void stream_chunk(const uint4* __restrict__ vp, int v_begin, int v_end,
+                                             uint32_t id_base, int K, int tid, int lane, float& m,
+                                             float& s, WarpCand& w, uint32_t* s_cta_thr,
+                                             float* s_wtop) {
+  constexpr int STEP = TK_UNROLL * NT;
+  const int full_end = v_begin + (v_end - v_begin) / STEP * STEP;
+  uint4 cur[TK_UNROLL], nxt[TK_UNROLL];
+  if (v_begin < full_end) load_batch<T, NT, false>(vp, v_begin, v_end, tid, cur);
+#pragma unroll 1
+  for (int it = v_begin; it < full_end; it += STEP) {
+    if (it + STEP < full_end) load_batch<T, NT, false>(vp, it + STEP, v_end, tid, nxt);
+    process_batch<T, NT, false>(cur, it, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr, s_wtop);
+#pragma unroll
+    for (int u = 0; u < TK_UNROLL; ++u) cur[u] = nxt[u];
+  }
+  if (full_end < v_end) {
+    load_batch<T, NT, true>(vp, full_end, v_end, tid, cur);
+    process_batch<T, NT, true>(cur, full_end, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr,
+                               s_wtop);
   }
 }
 
@@ -393,22 +446,23 @@ __device__ __forceinline__ void write_row(int row, int K, float m, float s, cons
   }
 }
 
-template <typename T>
-__global__ void __launch_bounds__(TK_THREADS, 4)
+template <typename T, int NT>
+__global__ void __launch_bounds__(NT, 1024 / NT)
 topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chunk_vecs,
                 size_t rec_bytes, int32_t* __restrict__ ids, float* __restrict__ logp,
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
                 unsigned char* partials, PartialOut pout) {
   pdl_wait();
   constexpr int VEC = Vec<T>::N;
-  __shared__ uint64_t s_buf[TK_WARPS][TK_CAP];   // the warps' candidates
-  __shared__ uint64_t s_tmp[TK_WARPS][LILICORR_MAX_K];
+  constexpr int NW = NT / 32;
+  __shared__ uint64_t s_buf[NW][TK_CAP];         // the warps' candidates
+  __shared__ uint64_t s_tmp[NW][LILICORR_MAX_K];
   __shared__ uint64_t s_keys[TK_MERGE_MAX];       // the splits' lists (last CTA)
   __shared__ uint64_t s_merge[TK_MERGE_MAX];
   __shared__ uint64_t s_top[LILICORR_MAX_K];
-  __shared__ float s_m[TK_WARPS], s_s[TK_WARPS];
+  __shared__ float s_m[NW], s_s[NW];
   __shared__ uint32_t s_cta_thr;                // CTA-wide value bound (order image)
-  __shared__ float s_wtop[TK_WARPS];            // the warps' r-th largest lane maxima
+  __shared__ float s_wtop[NW];                  // the warps' r-th largest lane maxima
   __shared__ int s_last, s_count;
   __shared__ uint64_t s_bound;
 
@@ -430,7 +484,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   w.n = 0;
   w.thr = -INFINITY;
   if (tid == 0) s_cta_thr = ord32(-INFINITY);
-  if (tid < TK_WARPS) s_wtop[tid] = -INFINITY;
+  if (tid < NW) s_wtop[tid] = -INFINITY;
   __syncthreads();
 
   float m = -INFINITY, s = 0.f;
@@ -449,14 +503,9 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
     }
   }
 
-  // main stream: full batches without predicates, then the remainder
+  // main stream: batches of 16-byte vectors, the next one's loads in flight
   const uint4* vp = reinterpret_cast<const uint4*>(rp + e0);
-  constexpr int STEP = TK_UNROLL * TK_THREADS;
-  const int full_end = v_begin + (v_end - v_begin) / STEP * STEP;
-  for (int it = v_begin; it < full_end; it += STEP)
-    process_batch<T, false>(vp, it, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
-  if (full_end < v_end)
-    process_batch<T, true>(vp, full_end, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
+  stream_chunk<T, NT>(vp, v_begin, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
 
   // (max, sum) of the warp, then of the CTA
   const float wm = warp_max(m);
@@ -467,7 +516,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   // (the bound never exceeds the CTA's K-th value, so the K largest keys all survive)
   if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr));
   if (tid == 0) s_count = 0;
-  for (int i = tid; i < LILICORR_MAX_K; i += TK_THREADS) s_top[i] = 0ull;
+  for (int i = tid; i < LILICORR_MAX_K; i += NT) s_top[i] = 0ull;
   __syncthreads();
   {
     const float bound = unord32(s_cta_thr);
@@ -487,16 +536,16 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
     warp_compact(w, K, lane);
     if (lane < LILICORR_MAX_K) s_keys[warp * LILICORR_MAX_K + lane] = lane < w.n ? w.buf[lane] : 0ull;
     __syncthreads();
-    cta_select(s_keys, TK_WARPS, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
+    cta_select<NT>(s_keys, NW, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
   } else {
-    rank_place(s_merge, s_count, K, s_top, tid, TK_THREADS);
+    rank_place(s_merge, s_count, K, s_top, tid, NT);
     __syncthreads();
   }
 
   float cm = -INFINITY, cs = 0.f;
   if (warp == 0) {
-    const float pm = lane < TK_WARPS ? s_m[lane] : -INFINITY;
-    const float ps = lane < TK_WARPS ? s_s[lane] : 0.f;
+    const float pm = lane < NW ? s_m[lane] : -INFINITY;
+    const float ps = lane < NW ? s_s[lane] : 0.f;
     cm = warp_max(pm);
     cs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - cm) * LOG2E));
   }
@@ -524,12 +573,12 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
 
   // last CTA of the row: merge all splits (their lists staged in shared memory)
   const int n = splits * K;
-  for (int i = tid; i < n; i += TK_THREADS) {
+  for (int i = tid; i < n; i += NT) {
     const Rec* r = reinterpret_cast<const Rec*>(partials + ((size_t)row * splits + i / K) * rec_bytes);
     s_keys[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
   }
   __syncthreads();
-  cta_select(s_keys, splits, K, K, s_merge, &s_count, &s_bound, s_top);
+  cta_select<NT>(s_keys, splits, K, K, s_merge, &s_count, &s_bound, s_top);
   if (warp == 0) {
     float pm = -INFINITY, ps = 0.f;
     for (int i = lane; i < splits; i += 32) {
@@ -569,7 +618,7 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
     s_keys[i] = id < 0 ? 0ull : make_key(v, (uint32_t)id);
   }
   __syncthreads();
-  cta_select(s_keys, P, K, K, s_merge, &s_count, &s_bound, s_top);
+  cta_select<TK_THREADS>(s_keys, P, K, K, s_merge, &s_count, &s_bound, s_top);
   if (warp == 0) {
     float pm = -INFINITY, ps = 0.f;
     for (int p = lane; p < P; p += 32) {
@@ -591,17 +640,27 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
 TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   const int vec = dt == LILICORR_BF16 ? 8 : 4;
   const int nvec = V / vec;
-  // Few rows: split each over about 256 CTAs in all (a sweep over 16-256 rows of a
-  // 151,936-wide vocabulary put the optimum at 192-256 CTAs: more pieces add partial
-  // records and merge work faster than they shorten the stream). Once the rows alone
-  // fill half of the resident slots (4 CTAs per SM), one CTA per row.
-  const int slots = num_sms() * 4;
+  const int sms = num_sms();
   const int min_chunk = 256;                 // vectors (4 KB) per CTA at least
-  int splits = rows * 2 >= slots ? 1 : ceil_div(TK_FEW_ROW_CTAS, rows);
+  int splits = 1, threads = TK_THREADS;
+  if (rows * 2 < sms * 4) {
+    // Few rows (not filling half of the 4-per-SM slots): split each over about 256 CTAs of
+    // 256 threads in all (a sweep over 16-256 rows of a 151,936-wide vocabulary put the
+    // optimum at 192-256 CTAs: more pieces add partial records and merge work faster than
+    // they shorten the stream).
+    splits = ceil_div(TK_FEW_ROW_CTAS, rows);
+  } else if (rows >= 16 * sms) {
+    // Many rows per SM: one CTA of 128 threads per row, up to 8 resident per SM, so each SM
+    // always has rows in flight while others finish (4096 rows of 151,936: 233 us against
+    // 256 us with 256-thread CTAs). Splitting rows never paid: every piece repeats the
+    // candidate bound's warm-up and adds a merge (+30-40 % at 512-4096 rows).
+    threads = TK_THREADS_MANY;
+  }
   splits = max(1, min(splits, ceil_div(max(nvec, 1), min_chunk)));
   splits = min(splits, min(TK_MAX_SPLITS, TK_MERGE_MAX / K));
   TopkPlan p;
   p.splits = splits;
+  p.threads = threads;
   p.chunk_vecs = ceil_div(max(nvec, 1), splits);
   p.rec_bytes = align_up(8 + 8 * (size_t)K, 16);
   return p;
@@ -620,14 +679,28 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
   if (rows == 0) return LILICORR_OK;
   const TopkPlan p = topk_plan(rows, V, K, dt);
   dim3 grid(p.splits, rows);
-  if (dt == LILICORR_BF16)
-    LL_TRY(launch_k(topk_lse_kernel<uint16_t>, grid, TK_THREADS, 0, st, 
-        static_cast<const uint16_t*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials), pout));
-  else
-    LL_TRY(launch_k(topk_lse_kernel<float>, grid, TK_THREADS, 0, st, 
-        static_cast<const float*>(logits), V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp,
-        lse, status, counters, static_cast<unsigned char*>(partials), pout));
+  unsigned char* part = static_cast<unsigned char*>(partials);
+  if (dt == LILICORR_BF16) {
+    const uint16_t* x = static_cast<const uint16_t*>(logits);
+    if (p.threads == TK_THREADS_MANY)
+      LL_TRY(launch_k(topk_lse_kernel<uint16_t, TK_THREADS_MANY>, grid, TK_THREADS_MANY, 0, st, x,
+                      V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters,
+                      part, pout));
+    else
+      LL_TRY(launch_k(topk_lse_kernel<uint16_t, TK_THREADS>, grid, TK_THREADS, 0, st, x, V, K,
+                      p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
+                      pout));
+  } else {
+    const float* x = static_cast<const float*>(logits);
+    if (p.threads == TK_THREADS_MANY)
+      LL_TRY(launch_k(topk_lse_kernel<float, TK_THREADS_MANY>, grid, TK_THREADS_MANY, 0, st, x, V,
+                      K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters,
+                      part, pout));
+    else
+      LL_TRY(launch_k(topk_lse_kernel<float, TK_THREADS>, grid, TK_THREADS, 0, st, x, V, K,
+                      p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
+                      pout));
+  }
   return LILICORR_OK;
 }
 
