@@ -3,10 +3,10 @@
  * selection path; they expose internal building blocks so tests can check them
  * one at a time.
  *
- * The two path switches below (lilicorr_test_fused_path, lilicorr_test_attention_path)
- * change process-global dispatch state that every head and every host thread reads when
- * it enqueues a call. They are not synchronised: set them only while no other thread is
- * enqueueing work through the library, and put the default back afterwards.
+ * The path switch below (lilicorr_test_fused_path) changes process-global dispatch state
+ * that every head and every host thread reads when it enqueues a call. It is not
+ * synchronised: set it only while no other thread is enqueueing work through the library,
+ * and put the default back afterwards.
  */
 #ifndef LILICORR_TESTING_H_
 #define LILICORR_TESTING_H_
@@ -54,13 +54,6 @@ lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, flo
  * while another thread is enqueueing. Returns 1 if `head` (may be NULL) can take the
  * kernel that `mode` names, else 0. */
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode);
-
-/* Switch for the chain's attention core (Sec. 3.2 and App. A: bidirectional attention
- * with the slot-distance and same-slot biases, bf16 heads): mode 1 runs it on the
- * tcgen05 tensor cores where the head width is 32 or 64 and a sequence has at most 256
- * nodes, mode 0 (the default: the faster of the two so far) on the mma.sync kernel.
- * Process-wide, like the switch above. Returns the previous mode. */
-int lilicorr_test_attention_path(int mode);
 
 #ifdef __cplusplus
 }

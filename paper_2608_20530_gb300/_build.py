@@ -14,7 +14,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "lib")
 LIB = os.path.join(LIBDIR, "liblilicorr.so")
-SOURCES = ["api.cu", "topk_lse.cu", "head_kernels.cu", "pair_walk.cu", "attention_umma.cu", "gemm_tc.cu",
+SOURCES = ["api.cu", "topk_lse.cu", "head_kernels.cu", "pair_walk.cu", "gemm_tc.cu",
            "attention_tc.cu", "net_fused.cu",
            "diagnostics.cu", "gemm_small.cu", "lm_head.cu",
            "net_cluster.cu"]

@@ -18,7 +18,6 @@ size_t pair_walk_smem_bytes(int L, int K, int d);
 
 static std::atomic<uint64_t> g_launches{0};
 int g_fused_enabled = 1;
-int g_attn_umma = 0;   // the tcgen05 attention core: off until it beats the mma.sync one
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int num_sms() {
@@ -354,10 +353,7 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
     g = c.G(c.xn, adt, D, l.wqkv, D, c.qkv, c.qkv_dt, 3 * D, N, 3 * D, D);
     g.bias = l.bqkv;
     LL_TRY(run_gemm(g, st));
-    if (c.tc_attn && g_attn_umma && attention_umma_supported(d.L, d.K, D, d.n_heads))
-      LL_TRY(launch_attention_umma(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att,
-                                   c.status, st));
-    else if (c.tc_attn)
+    if (c.tc_attn)
       LL_TRY(launch_attention_tc(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att, st));
     else
       LL_TRY(launch_attention(static_cast<const float*>(c.qkv), c.B, d.L, d.K, D, d.n_heads,
@@ -866,12 +862,6 @@ lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, flo
   g.wait_limit = wait_cycles;
   g.test_starve = 1;
   return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_SHAPE;
-}
-
-int lilicorr_test_attention_path(int mode) {
-  const int prev = g_attn_umma;
-  g_attn_umma = mode ? 1 : 0;
-  return prev;
 }
 
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode) {

@@ -302,13 +302,6 @@ lilicorr_status_t launch_net_cluster(const lilicorr_head* h, int B, const int32_
                                      const float* logp, const float* hproj, const float* t,
                                      const float* cb, float* oi, uint32_t* status, cudaStream_t st,
                                      const ClusterTail* tail = nullptr);
-// the chain's attention core on tcgen05 (attention_umma.cu): 32- or 64-wide heads, up to
-// 256 nodes per sequence; g_attn_umma 1 uses it where supported, 0 (the default) never
-bool attention_umma_supported(int L, int K, int D, int n_heads);
-lilicorr_status_t launch_attention_umma(const void* qkv, int B, int L, int K, int D, int n_heads,
-                                        const float* dist, const float* same, void* out,
-                                        uint32_t* status, cudaStream_t st);
-extern int g_attn_umma;
 extern int g_fused_enabled;   // 0 never, 1 by batch size (default), 2 the one-CTA kernel
                               // always, 3 the cluster kernel always
 constexpr int FUSED_MIN_B = 8;
