@@ -17,7 +17,7 @@ LIB = os.path.join(LIBDIR, "liblilicorr.so")
 SOURCES = ["api.cu", "topk_lse.cu", "head_kernels.cu", "pair_walk.cu", "gemm_tc.cu",
            "attention_tc.cu", "net_fused.cu",
            "diagnostics.cu", "gemm_small.cu", "lm_head.cu",
-           "net_cluster.cu"]
+           "net_cluster.cu", "net_pair.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", INCLUDE, "-I", CSRC]

@@ -340,6 +340,9 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   }
   if (h->net_maps && (g_fused_enabled == 2 || (g_fused_enabled == 1 && c.B >= FUSED_MIN_B)))
     return launch_net_fused(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
+  // 129-256 nodes per sequence: two CTAs per sequence, one 128-node tile each
+  if (h->pair_maps && g_fused_enabled != 0)
+    return launch_net_pair(h, c.B, ids, logp, c.hproj, c.t, c.cb, c.oi, c.status, st);
   // nodes: x = fold[id] + hproj + slot + rank, then x += W_c2 c1 + b_c2
   LL_TRY(launch_node_build(h, c.B, ids, logp, c.hproj, c.c1, adt, c.x, c.status, st));
   GemmArgs g = c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D);
@@ -556,6 +559,7 @@ lilicorr_status_t lilicorr_head_create(const lilicorr_head_desc* desc, const voi
   embed_dev = nullptr;
   h->net_maps = net_fused_maps_create(h);
   h->cluster_maps = net_cluster_maps_create(h);
+  h->pair_maps = net_pair_maps_create(h);
   *out = h;
   return LILICORR_OK;
 }
@@ -568,6 +572,7 @@ lilicorr_status_t lilicorr_head_destroy(lilicorr_head* h) {
   cudaError_t e = cudaFree(h->pool);
   net_fused_maps_free(h->net_maps);
   net_cluster_maps_free(h->cluster_maps);
+  net_pair_maps_free(h->pair_maps);
   if (h->side) cudaStreamDestroy(h->side);
   if (h->side2) cudaStreamDestroy(h->side2);
   if (h->ev_fork) cudaEventDestroy(h->ev_fork);
@@ -867,7 +872,8 @@ lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, flo
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode) {
   g_fused_enabled = mode < 0 ? 0 : mode > 3 ? 3 : mode;
   if (!head) return 0;
-  return (mode == 3 ? head->cluster_maps : head->net_maps) ? 1 : 0;
+  if (mode == 3) return head->cluster_maps ? 1 : 0;
+  return (head->net_maps || head->pair_maps) ? 1 : 0;
 }
 
 uint64_t lilicorr_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }

@@ -189,6 +189,7 @@ struct lilicorr_head {
   const void* anc_w; const float* anc_b;
   void* net_maps;             // tensor maps of the fused scoring network, or null
   void* cluster_maps;         // tensor maps of the cluster scoring network, or null
+  void* pair_maps;            // tensor maps of the two-CTA network (129-256 nodes), or null
 };
 
 namespace lilicorr {
@@ -284,6 +285,14 @@ void net_fused_maps_free(void* maps);
 lilicorr_status_t launch_net_fused(const lilicorr_head* h, int B, const int32_t* ids,
                                    const float* logp, const float* hproj, const float* t,
                                    const float* cb, float* oi, uint32_t* status, cudaStream_t st);
+// the same network for 129-256 nodes per sequence on a cluster of two CTAs, one 128-node
+// tile each (net_pair.cu)
+bool net_pair_supported(const lilicorr_head_desc& d);
+void* net_pair_maps_create(const lilicorr_head* h);
+void net_pair_maps_free(void* p);
+lilicorr_status_t launch_net_pair(const lilicorr_head* h, int B, const int32_t* ids,
+                                  const float* logp, const float* hproj, const float* t,
+                                  const float* cb, float* oi, uint32_t* status, cudaStream_t st);
 // the same network on a cluster of four CTAs per sequence (net_cluster.cu)
 bool net_cluster_supported(const lilicorr_head_desc& d);
 void* net_cluster_maps_create(const lilicorr_head* h);

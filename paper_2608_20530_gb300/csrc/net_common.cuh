@@ -387,5 +387,140 @@ __device__ __forceinline__ void head_attention(uint32_t qb, int LK, int K, const
   inv1 = 1.0f / l1;
 }
 
+
+// The attention core above over a range of keys, unnormalised, for kernels that split
+// the keys of one head over two warps and merge the halves afterwards: q at qb (local
+// query rows q0..q0+15), k and v of every key at kb / vb (rows = key index, qkv_off
+// layout), keys [key0, key0 + nkeys) with keys at or past LK masked (the first 64-key
+// block of the range must hold at least one unmasked key). qoff: the node index of local
+// query row 0 (for its slot). Out: o[nb][e] as above, the two rows' running maxima m0, m1
+// (log2 units) and sums l0, l1 of 2^(s - m) over the range (summed over the row's lanes).
+__device__ __forceinline__ void head_attention_part(uint32_t qb, uint32_t kb, uint32_t vb, int key0,
+                                                    int nkeys, int LK, int K,
+                                                    const uint8_t* s_slot, const float* sd,
+                                                    float same_l2, int q0, int qoff, int lane,
+                                                    float (&o)[4][4], float& m0, float& m1,
+                                                    float& l0, float& l1) {
+  constexpr int KB = 64, NB = KB / 8;
+  const int g8 = lane >> 2, t4 = lane & 3;
+  const float qscale = rsqrtf(32.f) * 1.4426950408889634f;   // 1/sqrt(head width), log2 units
+  const bool k8 = (K & 7) == 0;
+  uint32_t qa[2][4];
+#pragma unroll
+  for (int ks = 0; ks < 2; ++ks)
+    ldsm_x4(qb + qkv_off(q0 + (lane & 15), ks * 2 + (lane >> 4)), qa[ks]);
+  const int si0 = s_slot[qoff + q0 + g8], si1 = s_slot[qoff + q0 + g8 + 8];
+  m0 = -INFINITY;
+  m1 = -INFINITY;
+  l0 = 0.f;
+  l1 = 0.f;
+#pragma unroll
+  for (int nb = 0; nb < 4; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
+#pragma unroll 1
+  for (int kb0 = key0; kb0 < key0 + nkeys; kb0 += KB) {
+    float s4[NB][4];
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb) s4[nb][0] = s4[nb][1] = s4[nb][2] = s4[nb][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+      for (int nb = 0; nb < NB; nb += 2) {
+        uint32_t bf[4];
+        const int key = kb0 + nb * 8 + (lane & 7) + ((lane >> 4) << 3);
+        ldsm_x4(kb + qkv_off(key, ks * 2 + ((lane >> 3) & 1)), bf);
+        mma_bf16_16816(s4[nb], qa[ks], bf[0], bf[1]);
+        mma_bf16_16816(s4[nb + 1], qa[ks], bf[2], bf[3]);
+      }
+    float bm0 = -INFINITY, bm1 = -INFINITY;
+    if (k8) {
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb) {
+        const int jt = kb0 + nb * 8;
+        const bool in = jt < LK;
+        const int sj = s_slot[in ? jt : 0];
+        const float b0 = sd[sj - si0] + (si0 == sj ? same_l2 : 0.f);
+        const float b1 = sd[sj - si1] + (si1 == sj ? same_l2 : 0.f);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float v = in ? fmaf(s4[nb][e], qscale, e < 2 ? b0 : b1) : -INFINITY;
+          s4[nb][e] = v;
+          if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+        }
+      }
+    } else {
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb) {
+        const int j0 = kb0 + nb * 8 + 2 * t4;
+        const uint32_t sp = *reinterpret_cast<const uint16_t*>(s_slot + j0);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int jj = j0 + (e & 1);
+          const int sj = (e & 1) ? (int)(sp >> 8) : (int)(sp & 255u);
+          const int si = e < 2 ? si0 : si1;
+          const float v = jj < LK
+                              ? s4[nb][e] * qscale + sd[sj - si] + (si == sj ? same_l2 : 0.f)
+                              : -INFINITY;
+          s4[nb][e] = v;
+          if (e < 2) bm0 = fmaxf(bm0, v); else bm1 = fmaxf(bm1, v);
+        }
+      }
+    }
+    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
+    bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
+    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
+    bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
+    const float mn0 = fmaxf(m0, bm0), mn1 = fmaxf(m1, bm1);
+    const float c0 = ex2f(m0 - mn0), c1 = ex2f(m1 - mn1);   // 0 on the first block
+    m0 = mn0;
+    m1 = mn1;
+    l0 *= c0;
+    l1 *= c1;
+#pragma unroll
+    for (int nb = 0; nb < 4; ++nb) {
+      o[nb][0] *= c0; o[nb][1] *= c0;
+      o[nb][2] *= c1; o[nb][3] *= c1;
+    }
+    uint32_t pa[NB / 2][4];
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb) {
+      const uint32_t h01 = ex2_h2(pack_h2(s4[nb][0] - mn0, s4[nb][1] - mn0));
+      const uint32_t h23 = ex2_h2(pack_h2(s4[nb][2] - mn1, s4[nb][3] - mn1));
+      const float2 f01 = h2_to_f2(h01), f23 = h2_to_f2(h23);
+      l0 += f01.x + f01.y;
+      l1 += f23.x + f23.y;
+      const int kk = nb >> 1;
+      if ((nb & 1) == 0) {
+        pa[kk][0] = h01;
+        pa[kk][1] = h23;
+      } else {
+        pa[kk][2] = h01;
+        pa[kk][3] = h23;
+      }
+    }
+#pragma unroll
+    for (int kk = 0; kk < NB / 2; ++kk)
+#pragma unroll
+      for (int nb = 0; nb < 4; nb += 2) {
+        uint32_t vf[4];
+        const int key = kb0 + kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        ldsm_x4_t(vb + qkv_off(key, nb + (lane >> 4)), vf);
+        mma_f16_16816(o[nb], pa[kk], vf[0], vf[1]);
+        mma_f16_16816(o[nb + 1], pa[kk], vf[2], vf[3]);
+      }
+  }
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+}
+
+// one 16-byte store into a peer's shared memory (peer address), ordinary (weak) semantics;
+// a later release arrival on the peer's barrier publishes it
+__device__ __forceinline__ void st_peer_v4(uint32_t raddr, const uint4& v) {
+  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(raddr), "r"(v.x),
+               "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
 }  // namespace net
 }  // namespace lilicorr
