@@ -399,7 +399,8 @@ def roofline_fracs(wl, B, us_call, us_topk, pk):
     }
 
 
-def bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams, min_bytes=6e8, reps=5):
+def bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams, d2h_stream, min_bytes=6e8,
+                  reps=5):
     """One batched workload (one tier) through select_block: device-timed calls over
     distinct resident batches (inputs larger than L2), the top-K pass alone, and the
     same calls end to end from pinned host buffers."""
@@ -437,7 +438,7 @@ def bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams, min_by
     n_e2e = max(nb, 4)
     eg = pipelined_e2e_graph(
         lambda x, tok: ll.select_block(head, x[0], x[1], x[2], ws=ws, tokens=tok),
-        h_in, d_in, h_tok, d_tok, [j % nb for j in range(n_e2e)], copy_streams)
+        h_in, d_in, h_tok, d_tok, [j % nb for j in range(n_e2e)], copy_streams, d2h_stream)
     us_e2e = time_replays([eg], stream, max(2, reps // 2), warm=1) * 1e3 / n_e2e
     d_l, d_h, d_t = d_in[0]
     if ws.status() != 0 or tk_ws.status() != 0:
@@ -458,21 +459,23 @@ def bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams, min_by
     return out
 
 
-def pipelined_e2e_graph(select, h_in, d_in, h_tok, d_tok, order, copy_streams):
+def pipelined_e2e_graph(select, h_in, d_in, h_tok, d_tok, order, copy_streams, d2h_stream):
     """One CUDA graph of len(order) end-to-end calls: call j copies host item order[j]
     (pinned tensors h_in[k][i]) into device buffer set j % 2 on the copy streams, runs
     ``select(inputs, tokens)`` on the capturing stream once its copies have landed, and
-    copies the tokens back to h_tok[i]. The copies of call j + 1 run while call j computes
-    (a buffer set is refilled only after the call two back has finished with it); the
-    logits, the largest input, are split across the copy streams."""
+    copies the tokens back to h_tok[i] on d2h_stream. The copies of call j + 1 run while
+    call j computes (a buffer set is refilled, and a token buffer rewritten, only after the
+    call two back has finished with it); the logits, the largest input, are split across
+    the copy streams."""
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
         s0 = torch.cuda.current_stream()
         start = torch.cuda.Event()
         start.record(s0)
-        for cs in copy_streams:
+        for cs in copy_streams + [d2h_stream]:
             cs.wait_event(start)
         done = []
+        fetched = []
         nc = len(copy_streams)
         for j, i in enumerate(order):
             b = j % 2
@@ -495,12 +498,19 @@ def pipelined_e2e_graph(select, h_in, d_in, h_tok, d_tok, order, copy_streams):
                     landed.append(e)
             for e in landed:
                 s0.wait_event(e)
+            if j >= 2:
+                s0.wait_event(fetched[j - 2])       # token buffer b has been read back
             select(d_in[b], d_tok[b])
-            h_tok[i].copy_(d_tok[b], non_blocking=True)
             e = torch.cuda.Event()
             e.record(s0)
             done.append(e)
-        for cs in copy_streams:
+            with torch.cuda.stream(d2h_stream):
+                d2h_stream.wait_event(e)
+                h_tok[i].copy_(d_tok[b], non_blocking=True)
+                f = torch.cuda.Event()
+                f.record(d2h_stream)
+                fetched.append(f)
+        for cs in copy_streams + [d2h_stream]:
             e = torch.cuda.Event()
             e.record(cs)
             s0.wait_event(e)
@@ -619,9 +629,11 @@ def run_ours(args, world, rank, local, pool):
     d_in = [[torch.empty_like(t[0]) for t in (logits, hidden, target)] for _ in range(2)]
     d_tok = [torch.empty((B, wl.L), dtype=torch.int32, device=dev) for _ in range(2)]
     copy_streams = [torch.cuda.Stream() for _ in range(args.copy_streams)]
+    d2h_stream = torch.cuda.Stream()
     sel = lambda x, tok: ll.select_block(head, x[0], x[1], x[2], ws=ws, tokens=tok)
     e2e_graphs = [pipelined_e2e_graph(sel, h_in, d_in, h_tokens, d_tok,
-                                      [(k * G + j) % nh for j in range(G)], copy_streams)
+                                      [(k * G + j) % nh for j in range(G)], copy_streams,
+                                      d2h_stream)
                   for k in range(-(-nh // G))]
     n_e2e_replays = -(-nblk // G)
     e2e_calls = n_e2e_replays * G
@@ -786,7 +798,8 @@ def run_ours(args, world, rank, local, pool):
         by_workload = {}
         for name, tier in BATCHED:
             key = name if not workloads.WORKLOADS[name].tiers else f"{name}.tau{workloads.WORKLOADS[name].tiers[tier]}"
-            by_workload[key] = bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams)
+            by_workload[key] = bench_batched(ll, name, tier, dev, stream, E, pk, rank, copy_streams,
+                                             d2h_stream)
         by_workload["clocks"] = bclk.stop()
         by_workload["note"] = ("each: select_block over distinct resident batches (>= 0.6 GB of "
                                "logits, larger than L2) in one CUDA graph, CUDA events; topk_* = "
@@ -809,9 +822,10 @@ def run_ours(args, world, rank, local, pool):
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
-                "note": f"pinned host blocks cycled ({nh} distinct); each call's copies (logits "
-                        f"split over {args.copy_streams} copy streams) captured with it, "
-                        f"overlapping the previous call's compute"},
+                "note": f"pinned host blocks cycled ({nh} distinct); each call's input copies "
+                        f"(logits split over {args.copy_streams} copy streams) and token read-back "
+                        f"(its own stream) captured with it, overlapping the neighbouring calls' "
+                        f"compute"},
         "gpu_launches": launches_per_call * nblk * args.steps,
         "roofline": roofline,
         "by_workload": by_workload,

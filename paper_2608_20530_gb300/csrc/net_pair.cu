@@ -18,7 +18,8 @@
 // row-worker warps then take 16 queries each over one half of the keys (warp w: queries
 // 16(w % 8).., keys 128(w / 8)..), and the two halves' online-softmax states (maxima,
 // sums, unnormalised outputs) merge through shared memory: once every warp is done with the
-// head's keys and values, the second-half warp parks its state in their place and the
+// head's q, k and v, the buffer opens to the peer's rows of the next head, and the second-half
+// warp parks its state (outputs as fp16) in the q rows and the 8 KB after v, where the
 // first-half warp of the same queries combines it and writes the head's output. (A hand-off
 // of the same state through tensor-memory columns, second-half warp storing and first-half
 // warp loading the same lanes after tcgen05.wait::st, the thread-sync fences and a named
@@ -610,7 +611,7 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
             // first head of a layer, with the FFN's use of the buffer): the peer may now write
             // its rows of head hn here
             rw_bar();
-            if (lane == 0) mbar_arrive_peer(peer_addr(smem_u32(&kv_open[hn]), peer));
+            if (hh == 0 && lane == 0) mbar_arrive_peer(peer_addr(smem_u32(&kv_open[hn]), peer));
             // q (columns of part 0), k (part 1, bf16) and v (part 2, fp16) of head hh, biases
             // added, by column groups 0, 1, 2; the k and v rows go to the peer as well, once
             // the peer's buffer is open for this head
@@ -645,29 +646,41 @@ __global__ void __launch_bounds__(NF_THREADS, 1)
             head_attention_part(smem_u32(hq + Q_OFF), smem_u32(hq + K_OFF), smem_u32(hq + V_OFF),
                                 NF_M * kh, NF_M, LK, K, s_slot, s_dist + hh * nd + (L - 1),
                                 s_same[hh], 16 * wr16, nbase, lane, o, m0, m1, l0, l1);
-            // merge the two key halves: once every warp is done with k and v (this CTA's alone
-            // until it opens the buffer for the next head), the second-half warp parks its
-            // state there (value j of thread (pair wr16, lane) at float j * 256 + 32 wr16 + lane)
-            // and the first-half warp of the same queries combines it with its own
-            float* park = reinterpret_cast<float*>(hq + K_OFF);
+            // every warp is done with q, k and v of head hh: k and v may take the peer's rows
+            // of the next head of the layer while the two key halves merge. The second-half
+            // warp parks its state (outputs as fp16 pairs: |o| <= the sum of the half's
+            // weights times max |v|, far inside fp16's range; then its maxima and sums) in the
+            // q rows and the free 8 KB after v: word j of thread (pair wr16, lane) at
+            // park[j][32 wr16 + lane]; the first-half warp of the same queries combines.
             rw_bar();
+            if (hh < NF_NH - 1 && lane == 0)
+              mbar_arrive_peer(peer_addr(smem_u32(&kv_open[hn + 1]), peer));
+            uint32_t* park_o = reinterpret_cast<uint32_t*>(hq + Q_OFF);           // 8 words
+            float* park_s = reinterpret_cast<float*>(hq + V_OFF + 16384);         // 4 words
+            const int slot_ = 32 * wr16 + lane;
             if (kh == 1) {
 #pragma unroll
-              for (int nb = 0; nb < 4; ++nb)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) park[(4 * nb + i) * 256 + 32 * wr16 + lane] = o[nb][i];
-              park[16 * 256 + 32 * wr16 + lane] = m0;
-              park[17 * 256 + 32 * wr16 + lane] = m1;
-              park[18 * 256 + 32 * wr16 + lane] = l0;
-              park[19 * 256 + 32 * wr16 + lane] = l1;
+              for (int nb = 0; nb < 4; ++nb) {
+                park_o[(2 * nb) * 256 + slot_] = pack_h2(o[nb][0], o[nb][1]);
+                park_o[(2 * nb + 1) * 256 + slot_] = pack_h2(o[nb][2], o[nb][3]);
+              }
+              park_s[0 * 256 + slot_] = m0;
+              park_s[1 * 256 + slot_] = m1;
+              park_s[2 * 256 + slot_] = l0;
+              park_s[3 * 256 + slot_] = l1;
             }
             rw_bar();
             if (kh == 0) {
               float ot[16], mt[4];
 #pragma unroll
-              for (int j = 0; j < 16; ++j) ot[j] = park[j * 256 + 32 * wr16 + lane];
+              for (int nb = 0; nb < 4; ++nb) {
+                const float2 a01 = h2_to_f2(park_o[(2 * nb) * 256 + slot_]);
+                const float2 a23 = h2_to_f2(park_o[(2 * nb + 1) * 256 + slot_]);
+                ot[4 * nb + 0] = a01.x; ot[4 * nb + 1] = a01.y;
+                ot[4 * nb + 2] = a23.x; ot[4 * nb + 3] = a23.y;
+              }
 #pragma unroll
-              for (int j = 0; j < 4; ++j) mt[j] = park[(16 + j) * 256 + 32 * wr16 + lane];
+              for (int j = 0; j < 4; ++j) mt[j] = park_s[j * 256 + slot_];
               const float M0 = fmaxf(m0, mt[0]), M1 = fmaxf(m1, mt[1]);
               const float a0 = ex2f(m0 - M0), b0 = ex2f(mt[0] - M0);
               const float a1 = ex2f(m1 - M1), b1 = ex2f(mt[1] - M1);

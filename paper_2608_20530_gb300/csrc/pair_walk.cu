@@ -6,10 +6,12 @@
 // one small matrix product per slot pair, and the walk commits left to right
 // c_s = argmax_k phi(s-1, c_{s-1}, k), touching no weights.
 //
-// pair_rows_kernel: grid (B, L). CTA (b, j) scores the anchor row (j = 0) or the
-// slot pair (j-1, j): it stages slot j's K in vectors and their norms in shared
-// memory, every warp takes rows of the earlier slot and forms K dot products by
-// lane-strided loads and a shuffle reduction. With the walk fused, the last CTA
+// pair_block_kernel: grid (B, L). CTA (b, j) scores the anchor row (j = 0) or the slot
+// pair (j-1, j): both slots' vectors are staged in shared memory and each thread forms
+// whole dot products (one output at a time). pair_rows_kernel, the same grid for vectors
+// too long to stage twice: it stages slot j's K in vectors and their norms, every warp
+// takes rows of the earlier slot and forms K dot products by lane-strided loads and a
+// shuffle reduction. With the walk fused, the last CTA
 // of a sequence to finish (atomic ticket, nobody waits) loads the sequence's
 // scores into shared memory and walks them.
 // walk_kernel: grid B, the walk alone over given scores.
@@ -110,6 +112,113 @@ __device__ __forceinline__ void run_walk(const PairWalkArgs& a, const float* A, 
     if (a.choice) a.choice[o] = c;
     if (a.tokens) a.tokens[o] = a.ids[o * a.K + c];
   }
+}
+
+// The walk after the pair scores: the last CTA of a sequence to finish (atomic ticket,
+// nobody waits) stages the sequence's scores in shared memory and walks them.
+__device__ __forceinline__ void walk_after_pairs(const PairWalkArgs& a, float* sm, int* s_last,
+                                                 uint8_t* s_back, uint8_t* s_path) {
+  const int b = blockIdx.x, L = a.L, K = a.K;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) *s_last = atomicAdd(&a.counters[b], 1u) == (uint32_t)(L - 1);
+  __syncthreads();
+  if (!*s_last) return;
+  __threadfence();
+  const int n_scores = K + (L - 1) * K * K;
+  const float* gA = a.A + (size_t)b * K;
+  const float* gP = a.P + (size_t)b * (L - 1) * K * K;
+  const float* A = gA;
+  const float* P = gP;
+  if (a.scores_in_smem) {                       // reuse the staging buffer for the scores
+    stage_scores(sm, gA, gP, K, n_scores);
+    __syncthreads();
+    A = sm;
+    P = sm + K;
+  }
+  if ((threadIdx.x >> 5) == 0) {
+    run_walk(a, A, P, b, s_back, s_path);
+    if ((threadIdx.x & 31) == 0) a.counters[b] = 0u;   // leave the workspace reusable
+  }
+}
+
+// Row stride (floats) of the staged vectors: 16-byte aligned rows whose 16-byte pieces
+// start on different banks for consecutive rows.
+__host__ __device__ __forceinline__ int pw_stride(int d) { return (d + 3) / 4 * 4 + 4; }
+
+// CTA (b, j): the slot pair (j - 1, j), or the anchor row (j = 0). Both slots' vectors
+// (K in vectors of slot j, K out vectors of slot j - 1 or the anchor's one) are staged in
+// shared memory by asynchronous copies, all issued before one wait; each warp takes the
+// norms of some rows; then thread t forms whole dot products, one output (k, k') at a time,
+// reading both rows from shared memory (no cross-lane reductions) and storing the cosine.
+__global__ void __launch_bounds__(PW_THREADS) pair_block_kernel(PairWalkArgs a) {
+  pdl_wait();
+  extern __shared__ float sm[];
+  __shared__ int s_last;
+  __shared__ float s_norm[2 * LILICORR_MAX_K];
+  __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
+  __shared__ uint8_t s_path[LILICORR_MAX_L];
+  const int b = blockIdx.x, j = blockIdx.y;
+  const int L = a.L, K = a.K, d = a.d, ds = pw_stride(d);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = PW_THREADS / 32;
+  const int nrows = j == 0 ? 1 : K;                 // vectors of the earlier slot (or anchor)
+  const float* inb = a.in + (size_t)(b * L + j) * K * a.ld_vec;
+  const float* outb = j == 0 ? a.anchor + (size_t)b * d
+                             : a.out + (size_t)(b * L + j - 1) * K * a.ld_vec;
+  const int ldo = j == 0 ? d : a.ld_vec;
+  const bool v4 = ((d | a.ld_vec) & 3) == 0 && (reinterpret_cast<uintptr_t>(a.in) & 15) == 0 &&
+                  (reinterpret_cast<uintptr_t>(a.out) & 15) == 0 &&
+                  (reinterpret_cast<uintptr_t>(a.anchor) & 15) == 0;
+  // rows 0 .. K-1: in vectors of slot j; rows K .. K+nrows-1: out vectors (or the anchor)
+  if (v4) {
+    const int dv = d >> 2;
+    for (int i = threadIdx.x; i < (K + nrows) * dv; i += PW_THREADS) {
+      const int row = i / dv, c = 4 * (i - row * dv);
+      const float* src = row < K ? inb + (size_t)row * a.ld_vec + c : outb + (size_t)(row - K) * ldo + c;
+      cp16(sm + (size_t)row * ds + c, src);
+    }
+    cp_wait_all();
+  } else {
+    for (int i = threadIdx.x; i < (K + nrows) * d; i += PW_THREADS) {
+      const int row = i / d, c = i - row * d;
+      sm[(size_t)row * ds + c] = row < K ? inb[(size_t)row * a.ld_vec + c]
+                                         : outb[(size_t)(row - K) * ldo + c];
+    }
+  }
+  __syncthreads();
+  for (int v = warp; v < K + nrows; v += nw) {
+    float ss = 0.f;
+    for (int c = lane; c < d; c += 32) ss = fmaf(sm[(size_t)v * ds + c], sm[(size_t)v * ds + c], ss);
+    ss = warp_sum(ss);
+    if (lane == 0) s_norm[v] = fmaxf(sqrtf(ss), UNIT_EPS);
+  }
+  __syncthreads();
+  for (int o = threadIdx.x; o < nrows * K; o += PW_THREADS) {
+    const int r = o / K, k2 = o - r * K;
+    const float* x = sm + (size_t)(K + r) * ds;
+    const float* y = sm + (size_t)k2 * ds;
+    float acc0 = 0.f, acc1 = 0.f;
+    int c = 0;
+    if ((d & 3) == 0) {
+      for (; c < d; c += 8) {
+        const float4 x0 = *reinterpret_cast<const float4*>(x + c);
+        const float4 y0 = *reinterpret_cast<const float4*>(y + c);
+        acc0 = fmaf(x0.x, y0.x, fmaf(x0.y, y0.y, fmaf(x0.z, y0.z, fmaf(x0.w, y0.w, acc0))));
+        if (c + 4 < d) {
+          const float4 x1 = *reinterpret_cast<const float4*>(x + c + 4);
+          const float4 y1 = *reinterpret_cast<const float4*>(y + c + 4);
+          acc1 = fmaf(x1.x, y1.x, fmaf(x1.y, y1.y, fmaf(x1.z, y1.z, fmaf(x1.w, y1.w, acc1))));
+        }
+      }
+    } else {
+      for (; c < d; ++c) acc0 = fmaf(x[c], y[c], acc0);
+    }
+    const float v = (acc0 + acc1) / (s_norm[K + r] * s_norm[k2]);
+    if (j == 0) a.A[(size_t)b * K + k2] = v;
+    else a.P[((size_t)b * (L - 1) + (j - 1)) * K * K + (size_t)r * K + k2] = v;
+  }
+  if (!a.do_walk) return;
+  walk_after_pairs(a, sm, &s_last, s_back, s_path);
 }
 
 __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
@@ -220,29 +329,7 @@ __global__ void __launch_bounds__(PW_THREADS) pair_rows_kernel(PairWalkArgs a) {
     }
   }
   if (!a.do_walk) return;
-
-  // the last CTA of this sequence walks
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(&a.counters[b], 1u) == (uint32_t)(L - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  const int n_scores = K + (L - 1) * K * K;
-  const float* gA = a.A + (size_t)b * K;
-  const float* gP = a.P + (size_t)b * (L - 1) * K * K;
-  const float* A = gA;
-  const float* P = gP;
-  if (a.scores_in_smem) {                       // reuse the staging buffer for the scores
-    stage_scores(sm, gA, gP, K, n_scores);
-    __syncthreads();
-    A = sm;
-    P = sm + K;
-  }
-  if (warp == 0) {
-    run_walk(a, A, P, b, s_back, s_path);
-    if (lane == 0) a.counters[b] = 0u;          // leave the workspace reusable
-  }
+  walk_after_pairs(a, sm, &s_last, s_back, s_path);
 }
 
 __global__ void __launch_bounds__(PW_THREADS) walk_kernel(PairWalkArgs a) {
@@ -279,6 +366,16 @@ lilicorr_status_t launch_pair_walk(const PairWalkArgs& in, cudaStream_t st) {
   static bool cfg_pair[64] = {false}, cfg_walk[64] = {false};
   if (a.do_pairs) {
     if (a.do_walk && !a.counters) return LILICORR_ERR_ARG;
+    // both slots' vectors staged: when that stays within 100 KB (two CTAs per SM at least)
+    const size_t block_smem = sizeof(float) * (size_t)2 * a.K * pw_stride(a.d);
+    if (block_smem <= 100 * 1024) {
+      static bool cfg_block[64] = {false};
+      size_t smem = block_smem;
+      if (a.do_walk && a.scores_in_smem && score_bytes > smem) smem = score_bytes;
+      LL_TRY(allow_max_dynamic_smem(pair_block_kernel, cfg_block));
+      LL_TRY(launch_k(pair_block_kernel, dim3(a.B, a.L), PW_THREADS, smem, st, a));
+      return LILICORR_OK;
+    }
     size_t smem = pair_walk_smem_bytes(a.L, a.K, a.d);
     if (smem > PW_SMEM_MAX) return LILICORR_ERR_SHAPE;
     if (a.do_walk && a.scores_in_smem && score_bytes > smem) smem = score_bytes;
