@@ -64,6 +64,9 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-by-workload", dest="by_workload", action="store_false",
                    help="skip the batched workloads' section of the default run")
+    p.add_argument("--no-extras", action="store_true",
+                   help="time the selection only (no Viterbi, diagnostics, walk, vocabulary-shard "
+                        "or LM-head sections): for short profiling runs")
     p.add_argument("--no-cpu-baseline", action="store_true")
     return p.parse_args()
 
@@ -667,7 +670,7 @@ def run_ours(args, world, rank, local, pool):
     # sample of the blocks, both walks captured alike and timed back to back
     nv = min(nblk, 100)
     walk_ms = {}
-    for walk in ("greedy", "viterbi"):
+    for walk in (("greedy", "viterbi") if not args.no_extras else ()):
         gl = [graph_of([lambda i=i: ll.select_block(head, logits[i], hidden[i], target[i], ws=ws,
                                                      tokens=tokens[i], walk=walk)
                         for i in range(i0, min(i0 + G, nv))]) for i0 in range(0, nv, G)]
@@ -675,12 +678,13 @@ def run_ours(args, world, rank, local, pool):
                             for k in range(3)) / nv
     if ws.status() != 0:
         raise RuntimeError("device status set by the walk comparison")
-    walk = walk_latency(ll, head, logits[0], hidden[0], target[0], ws, B, stream)
+    walk = (walk_latency(ll, head, logits[0], hidden[0], target[0], ws, B, stream)
+            if not args.no_extras else None)
 
     # ---- diagnostics of the chosen blocks (Eq. "localar" probabilities and gaps along the
     # walk; coverage / oracle prefix / accepted prefix against the planted tokens)
     diag = None
-    if planted is not None:
+    if planted is not None and not args.no_extras:
         nd = min(nblk, 100)
         prefix_sum = acc_sum = 0
         for i in range(nd):
@@ -728,35 +732,37 @@ def run_ours(args, world, rank, local, pool):
     # ---- the vocabulary-sharded pass (a tensor-parallel LM head's logits), simulated on
     # this GPU: P contiguous vocabulary slices, each summarised into per-row records
     # (what one rank computes), then the merge of the gathered records
-    P = 4
-    sl = [flat[0][:, a:b].contiguous() for a, b in shards.bounds(wl.V, P)]
-    sws = [ll.Workspace(ll.lib().lilicorr_topk_lse_partial_workspace_bytes(rows, t.shape[1], wl.K))
-           for t in sl]
-    recs = torch.stack([ll.topk_lse_partial(t, wl.K, a, ws=w)
-                        for t, (a, _), w in zip(sl, shards.bounds(wl.V, P), sws)])
-    torch.cuda.synchronize()
-
     def timed(fn, n=20):
         fn()
         torch.cuda.synchronize()
         return time_replays([graph_of([fn] * n)], stream, 1, warm=1) * 1e3 / n
 
-    part_us = timed(lambda: ll.topk_lse_partial(sl[0], wl.K, 0, ws=sws[0]))
-    merge_us = timed(lambda: ll.topk_lse_merge(recs, wl.K))
-    sharded = {"shards": P, "partial_us_per_rank": round(part_us, 2),
-               "merge_us": round(merge_us, 2),
-               "gather_bytes_per_rank": rows * ll.topk_partial_bytes(wl.K),
-               "note": "one rank's slice (V/%d columns of every row) and the merge of %d "
-                       "ranks' records, both on this GPU; the all-gather itself is not timed"
-                       % (P, P)}
-    del sl, sws, recs
+    sharded = lm_head = None
+    P = 4
+    if args.no_extras:
+        P = 0                                   # the sections below are skipped
+    sl = [flat[0][:, a:b].contiguous() for a, b in shards.bounds(wl.V, P)] if P else []
+    if P:
+        sws = [ll.Workspace(ll.lib().lilicorr_topk_lse_partial_workspace_bytes(rows, t.shape[1], wl.K))
+               for t in sl]
+        recs = torch.stack([ll.topk_lse_partial(t, wl.K, a, ws=w)
+                            for t, (a, _), w in zip(sl, shards.bounds(wl.V, P), sws)])
+        torch.cuda.synchronize()
+        part_us = timed(lambda: ll.topk_lse_partial(sl[0], wl.K, 0, ws=sws[0]))
+        merge_us = timed(lambda: ll.topk_lse_merge(recs, wl.K))
+        sharded = {"shards": P, "partial_us_per_rank": round(part_us, 2),
+                   "merge_us": round(merge_us, 2),
+                   "gather_bytes_per_rank": rows * ll.topk_partial_bytes(wl.K),
+                   "note": "one rank's slice (V/%d columns of every row) and the merge of %d "
+                           "ranks' records, both on this GPU; the all-gather itself is not timed"
+                           % (P, P)}
+        del sl, sws, recs
 
     # ---- the LM-head projection fused with the top-K pass (logits never written): this
     # workload's drafter hidden states against a random bf16 vocabulary projection of the
     # workload's shape, next to the unfused pair (cuBLAS bf16 product writing the logits,
     # then the top-K pass)
-    lm_head = None
-    if wl.dtype == "bf16":
+    if wl.dtype == "bf16" and not args.no_extras:
         gW = torch.Generator(device=dev).manual_seed(1_000_033)
         Wv = (0.02 * torch.randn((wl.V, wl.H), generator=gW, device=dev)).to(torch.bfloat16)
         hrows = hidden[0].reshape(rows, wl.H)
@@ -830,10 +836,11 @@ def run_ours(args, world, rank, local, pool):
         "roofline": roofline,
         "by_workload": by_workload,
         "diagnostics": diag,
-        "walk_viterbi": {"us_per_call": round(walk_ms["viterbi"] * 1e3, 2),
-                         "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
-                         "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
-                         "sample": f"{nv} calls of this workload, best of 3"},
+        "walk_viterbi": ({"us_per_call": round(walk_ms["viterbi"] * 1e3, 2),
+                          "greedy_us_per_call": round(walk_ms["greedy"] * 1e3, 2),
+                          "block_rate_cost": round(walk_ms["viterbi"] / walk_ms["greedy"] - 1, 4),
+                          "sample": f"{nv} calls of this workload, best of 3"}
+                         if walk_ms else None),
         "walk": walk,
         "vocab_sharded": sharded,
         "lm_head_fused": lm_head,
