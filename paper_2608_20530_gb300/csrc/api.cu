@@ -150,7 +150,7 @@ WsLayout ws_layout(const lilicorr_head_desc& d, int B) {
   auto take = [&](size_t bytes) { size_t r = o; o = align_up(o + bytes, 256); return r; };
   w.status = take(256);
   w.counters = take(R * 4);
-  w.partials = take(R * p.splits * p.rec_bytes);
+  w.partials = take(R * p.pieces * p.rec_bytes);
   w.ids = take(N * 4); w.logp = take(N * 4); w.lse = take(R * 4);
   w.hproj = take(R * d.D * 4);
   w.tn = take((size_t)B * d.H * 4);

@@ -199,6 +199,7 @@ struct TopkPlan {
   int splits;          // CTAs per row
   int threads;         // threads per CTA
   int chunk_vecs;      // 16-byte vectors per split
+  int pieces;          // partial records per row in the workspace
   size_t rec_bytes;    // bytes of one partial record
 };
 TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt);

@@ -83,6 +83,13 @@ __device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
   return d;
 }
 
+// Barrier of the NT threads of a CTA (named barrier 1; the same threads as
+// __syncthreads).
+template <int NT>
+__device__ __forceinline__ void csync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(NT) : "memory");
+}
+
 // Rank counting: each key of keys[0..n) (distinct apart from zeros, which mean "empty")
 // counts the keys larger than itself and, if that rank is below K, lands in out[rank].
 // Run by `nthreads` threads with indices t; out[0..K) must be zeroed beforehand and
@@ -101,7 +108,8 @@ __device__ __forceinline__ void rank_place(const uint64_t* keys, int n, int K, u
 // K largest of groups[g][0..K) for g < ngroups (each group sorted descending, zeros =
 // empty), CTA-wide. Every group's K-th key bounds the answer's K-th from below, so only
 // keys >= the largest such bound survive; they are compacted and rank-counted.
-// surv: scratch of TK_MERGE_MAX keys; out[0..K) receives the result. All NT threads call.
+// surv: scratch of TK_MERGE_MAX keys; out[0..K) receives the result. All NT reducing
+// threads call.
 template <int NT>
 __device__ void cta_select(const uint64_t* groups, int ngroups, int stride, int K, uint64_t* surv,
                            int* s_count, uint64_t* s_bound, uint64_t* out) {
@@ -120,15 +128,15 @@ __device__ void cta_select(const uint64_t* groups, int ngroups, int stride, int 
     if (lane == 0) { *s_bound = b; *s_count = 0; }
   }
   for (int i = tid; i < K; i += NT) out[i] = 0ull;
-  __syncthreads();
+  csync<NT>();
   const uint64_t bound = *s_bound;
   for (int i = tid; i < ngroups * K; i += NT) {
     const uint64_t k = groups[(size_t)(i / K) * stride + i % K];
     if (k != 0ull && k >= bound) surv[atomicAdd(s_count, 1)] = k;
   }
-  __syncthreads();
+  csync<NT>();
   rank_place(surv, *s_count, K, out, tid, NT);
-  __syncthreads();
+  csync<NT>();
 }
 
 template <int N>
@@ -211,12 +219,36 @@ __device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
 // rank counting once it holds 2K keys (or when it would overflow).
 constexpr int TK_CAP = 96;
 
+// Every warp meets its elements in increasing id order (its share of each batch lies
+// above its share of the batch before; the split kernel's scalar head comes first and its
+// tail last). So once the buffer holds K keys, a later element whose value equals the
+// K-th key's loses that tie, and the warp's own filter may sit just above that value:
+// then a run of equal values costs one compaction, not one append per element. Other
+// warps meet elements on both sides of this warp's ids, so what the warp publishes (to
+// the CTA-wide bound and to the final selection) is the plain bound, publish_bound().
 struct WarpCand {
   uint64_t* buf;       // [TK_CAP] in shared memory
-  uint64_t* tmp;       // [LILICORR_MAX_K] scratch of the compaction
+  uint64_t* tmp;       // [LILICORR_MAX_K] scratch of the compaction; tmp[K - 1] holds the
+                       // K-th key of the last compaction (0: none yet)
   int n;               // keys in buf (warp-uniform)
-  float thr;           // value bound (warp-uniform, never decreases)
+  float thr;           // the warp's filter (warp-uniform, never decreases)
 };
+
+// Smallest float above v (+inf stays +inf).
+__device__ __forceinline__ float next_up(float v) {
+  if (v == 0.f) return __uint_as_float(1u);
+  const uint32_t b = __float_as_uint(v);
+  if (b == 0x7F800000u) return v;
+  return __uint_as_float((b & 0x80000000u) ? b - 1u : b + 1u);
+}
+
+// The warp's bound without the tie step: a value no element of the CTA's top-K lies below.
+__device__ __forceinline__ float publish_bound(const WarpCand& w, int K) {
+  const uint64_t kth = w.tmp[K - 1];
+  if (kth == 0ull) return w.thr;
+  const float kv = key_value(kth);
+  return w.thr == next_up(kv) ? kv : w.thr;
+}
 
 __device__ __forceinline__ void warp_compact(WarpCand& w, int K, int lane) {
   __syncwarp();
@@ -234,12 +266,33 @@ __device__ __forceinline__ void warp_compact(WarpCand& w, int K, int lane) {
   __syncwarp();
   if (lane < K) w.buf[lane] = mine;
   w.n = min(w.n, K);
-  if (kth) w.thr = fmaxf(w.thr, key_value(kth));
+  if (kth) {
+    const float kv = key_value(kth);
+    if (w.thr <= kv) w.thr = next_up(kv);      // equal values to come lose the tie
+  }
   __syncwarp();
 }
 
-// Append this lane's N values (ids id0 + j) that reach the bound. Warp-collective: one
-// ballot round per hot element of the busiest lane.
+// This lane's hot values among x[0..N) (ids id0 + j), exactly: at or above the plain bound
+// and with a key above the buffer's K-th key (a value equal to that key's needs a lower
+// id). For the rest of a vector after a compaction in its middle, whose lanes hold ids on
+// both sides of the new K-th key.
+template <int N>
+__device__ __forceinline__ uint32_t hot_mask_exact(const WarpCand& w, const float (&x)[N],
+                                                   uint32_t id0, bool valid, int K) {
+  const uint64_t kth = w.tmp[K - 1];
+  const float kv = key_value(kth);                // NaN for kth == 0: no tie to break
+  const uint32_t kid = (uint32_t)key_id(kth);
+  const float lo = publish_bound(w, K);
+  uint32_t hm = 0u;
+#pragma unroll
+  for (int j = 0; j < N; ++j)
+    hm |= (valid && x[j] >= lo && (x[j] != kv || id0 + (uint32_t)j < kid)) ? (1u << j) : 0u;
+  return hm;
+}
+
+// Append this lane's values that reach the filter. Warp-collective: one ballot round per
+// hot element of the busiest lane.
 template <int N>
 __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], uint32_t id0,
                                             bool valid, int K, int lane) {
@@ -249,8 +302,7 @@ __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], ui
   while (__any_sync(FULL, hm != 0u)) {
     if (w.n + 32 > TK_CAP) {
       warp_compact(w, K, lane);
-#pragma unroll
-      for (int j = 0; j < N; ++j) hm &= (x[j] >= w.thr) ? ~0u : ~(1u << j);
+      hm &= hot_mask_exact<N>(w, x, id0, valid, K);
       if (!__any_sync(FULL, hm != 0u)) break;
     }
     const bool has = hm != 0u;
@@ -267,7 +319,8 @@ __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], ui
 
 // A batch: TK_UNROLL 16-byte vectors per thread (vectors it + u*NT + tid, NT threads).
 // CHECK = false: every vector is inside the chunk (no predicates); otherwise vectors past
-// v_end read as -inf, which adds nothing to the sum and never becomes a candidate.
+// v_end read as -inf, which adds nothing to the sum and never becomes a candidate (the
+// reduction below also skips vectors outside [v_lo, v_end) as candidates).
 template <typename T, int NT, bool CHECK>
 __device__ __forceinline__ void load_batch(const uint4* __restrict__ vp, int it, int v_end, int tid,
                                            uint4 (&raw)[TK_UNROLL]) {
@@ -309,8 +362,8 @@ __device__ __forceinline__ void exp_vec(const uint4& r, uint64_t l2, uint64_t nm
 // the candidates, which the warp looks at only if some lane's batch maximum reaches the
 // bound. s_wtop[warp]: the warps' published r-th largest lane maxima (r = ceil(K / warps)).
 template <typename T, int NT, bool CHECK>
-__device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int it, int v_end,
-                                              uint32_t id_base, int K, int tid, int lane,
+__device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int it, int v_lo,
+                                              int v_end, uint32_t id_base, int K, int tid, int lane,
                                               float& m, float& s, WarpCand& w,
                                               uint32_t* s_cta_thr, float* s_wtop) {
   constexpr int VEC = Vec<T>::N;
@@ -337,7 +390,7 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int
     unpack2(a1, p2, p3);
     s += (p0 + p1) + (p2 + p3);
   }
-  // candidates: only when some lane's batch maximum reaches the current bound
+  // candidates: only when some lane's batch maximum reaches the current filter
   w.thr = fmaxf(w.thr, unord32(*(volatile uint32_t*)s_cta_thr));
   if (!__any_sync(FULL, bmax >= w.thr)) return;
   {
@@ -371,11 +424,12 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int
     const int v = it + u * NT + tid;
     float x[VEC];
     Vec<T>::unpack(raw[u], x);
-    warp_append<VEC>(w, x, id_base + (uint32_t)(v * VEC), !CHECK || v < v_end, K, lane);
+    warp_append<VEC>(w, x, id_base + (uint32_t)(v * VEC), !CHECK || (v >= v_lo && v < v_end), K,
+                     lane);
   }
   if (w.n >= 2 * K) {                                  // the buffer's K-th key bounds it
     warp_compact(w, K, lane);
-    if (lane == 0) atomicMax(s_cta_thr, ord32(w.thr));
+    if (lane == 0) atomicMax(s_cta_thr, ord32(publish_bound(w, K)));
   }
 }
 
@@ -394,14 +448,28 @@ __device__ __forceinline__ void stream_chunk(const uint4* __restrict__ vp, int v
 #pragma unroll 1
   for (int it = v_begin; it < full_end; it += STEP) {
     if (it + STEP < full_end) load_batch<T, NT, false>(vp, it + STEP, v_end, tid, nxt);
-    process_batch<T, NT, false>(cur, it, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr, s_wtop);
+    process_batch<T, NT, false>(cur, it, it, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr,
+                                s_wtop);
 #pragma unroll
     for (int u = 0; u < TK_UNROLL; ++u) cur[u] = nxt[u];
   }
   if (full_end < v_end) {
     load_batch<T, NT, true>(vp, full_end, v_end, tid, cur);
-    process_batch<T, NT, true>(cur, full_end, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr,
-                               s_wtop);
+    process_batch<T, NT, true>(cur, full_end, full_end, v_end, id_base, K, tid, lane, m, s, w,
+                               s_cta_thr, s_wtop);
+  }
+}
+
+// Elements [e_begin, e_end) of row rp, one per lane (the few outside the 16-byte vectors).
+template <typename T>
+__device__ __forceinline__ void scalar_part(const T* rp, int e_begin, int e_end, int K, int lane,
+                                            float& m, float& s, WarpCand& w) {
+  for (int base = e_begin; base < e_end; base += 32) {
+    const int e = base + lane;
+    const bool valid = e < e_end;
+    float x[1] = {valid ? Vec<T>::scalar(rp, e) : -INFINITY};
+    lse_update<1>(m, s, x, valid);
+    warp_append<1>(w, x, (uint32_t)(valid ? e : 0), valid, K, lane);
   }
 }
 
@@ -446,6 +514,124 @@ __device__ __forceinline__ void write_row(int row, int K, float m, float s, cons
   }
 }
 
+// Shared memory of one CTA's row reduction.
+template <int NW>
+struct TkShared {
+  uint64_t buf[NW][TK_CAP];             // the warps' candidates
+  uint64_t tmp[NW][LILICORR_MAX_K];
+  uint64_t keys[TK_MERGE_MAX];          // the pieces' lists (merging CTA)
+  uint64_t merge[TK_MERGE_MAX];
+  uint64_t top[LILICORR_MAX_K];
+  uint64_t bound;
+  float m[NW], s[NW];
+  float wtop[NW];                       // the warps' r-th largest lane maxima
+  uint32_t cta_thr;                     // CTA-wide value bound (order image)
+  int last, count;
+};
+
+// Close this CTA's piece of row `row` (all NT reducing threads, same arguments): the
+// piece's (max, sum exp) and top-K from the warps' states, then either the row's outputs
+// (its only piece) or the piece's partial record and a ticket. The CTA that takes the
+// row's last ticket (atomic, no waiting) merges the `npieces` records (row_recs,
+// rec_bytes apart) and writes the row.
+template <int NT>
+__device__ void finish_piece(TkShared<NT / 32>& sh, WarpCand& w, float m, float s, int row, int K,
+                             int npieces, int piece, unsigned char* row_recs, size_t rec_bytes,
+                             uint32_t* counters, const PartialOut& pout, int32_t* ids,
+                             float* logp, float* lse, uint32_t* status) {
+  constexpr int NW = NT / 32;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // (max, sum) of the warp, then of the CTA
+  const float wm = warp_max(m);
+  float ws = (m == -INFINITY) ? 0.f : s * ex2((m - wm) * LOG2E);
+  ws = warp_sum(ws);
+  const float pb = publish_bound(w, K);
+  if (lane == 0) {
+    sh.m[warp] = wm;
+    sh.s[warp] = ws;
+    atomicMax(&sh.cta_thr, ord32(pb));
+  }
+  // CTA top-K: keys of every warp's buffer at or above the CTA-wide bound, rank-counted
+  // (the bound never exceeds the CTA's K-th value, so the K largest keys all survive)
+  if (tid == 0) sh.count = 0;
+  for (int i = tid; i < LILICORR_MAX_K; i += NT) sh.top[i] = 0ull;
+  csync<NT>();
+  {
+    const float bound = unord32(sh.cta_thr);
+    const int nw = w.n;
+    for (int i = lane; i < nw; i += 32) {
+      const uint64_t k = w.buf[i];
+      if (key_value(k) >= bound) {
+        const int pos = atomicAdd(&sh.count, 1);
+        if (pos < TK_MERGE_MAX) sh.merge[pos] = k;
+      }
+    }
+  }
+  csync<NT>();
+  if (sh.count > TK_MERGE_MAX) {
+    // more survivors than the merge area holds (only with massive ties at the bound):
+    // compact every warp's buffer to its own top-K first, then merge those
+    warp_compact(w, K, lane);
+    if (lane < LILICORR_MAX_K) sh.keys[warp * LILICORR_MAX_K + lane] = lane < w.n ? w.buf[lane] : 0ull;
+    csync<NT>();
+    cta_select<NT>(sh.keys, NW, LILICORR_MAX_K, K, sh.merge, &sh.count, &sh.bound, sh.top);
+  } else {
+    rank_place(sh.merge, sh.count, K, sh.top, tid, NT);
+    csync<NT>();
+  }
+
+  float cm = -INFINITY, cs = 0.f;
+  if (warp == 0) {
+    const float pm = lane < NW ? sh.m[lane] : -INFINITY;
+    const float ps = lane < NW ? sh.s[lane] : 0.f;
+    cm = warp_max(pm);
+    cs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - cm) * LOG2E));
+  }
+  if (npieces == 1) {
+    if (warp == 0) write_row(row, K, cm, cs, sh.top, pout, ids, logp, lse, status, lane);
+    return;
+  }
+
+  // publish this piece's record, then take a ticket
+  Rec* rec = reinterpret_cast<Rec*>(row_recs + (size_t)piece * rec_bytes);
+  if (warp == 0) {
+    if (lane == 0) { rec->m = cm; rec->s = cs; }
+    if (lane < K) rec->keys[lane] = sh.top[lane];
+    __threadfence();
+  }
+  csync<NT>();
+  if (tid == 0) {
+    const uint32_t ticket = atomicAdd(&counters[row], 1u);
+    sh.last = (ticket == (uint32_t)(npieces - 1));
+  }
+  csync<NT>();
+  if (!sh.last) return;
+  __threadfence();
+
+  // last CTA of the row: merge all pieces (their lists staged in shared memory)
+  const int n = npieces * K;
+  for (int i = tid; i < n; i += NT) {
+    const Rec* r = reinterpret_cast<const Rec*>(row_recs + (size_t)(i / K) * rec_bytes);
+    sh.keys[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
+  }
+  csync<NT>();
+  cta_select<NT>(sh.keys, npieces, K, K, sh.merge, &sh.count, &sh.bound, sh.top);
+  if (warp == 0) {
+    float pm = -INFINITY, ps = 0.f;
+    for (int i = lane; i < npieces; i += 32) {
+      const Rec* r = reinterpret_cast<const Rec*>(row_recs + (size_t)i * rec_bytes);
+      const float rm = __ldcg(&r->m), rs = __ldcg(&r->s);
+      if (rm == -INFINITY) continue;
+      if (rm > pm) { ps = ps * ex2((pm - rm) * LOG2E) + rs; pm = rm; }
+      else ps += rs * ex2((rm - pm) * LOG2E);
+    }
+    const float gm = warp_max(pm);
+    const float gs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - gm) * LOG2E));
+    if (lane == 0) counters[row] = 0u;             // leave the workspace reusable
+    write_row(row, K, gm, gs, sh.top, pout, ids, logp, lse, status, lane);
+  }
+}
+
 template <typename T, int NT>
 __global__ void __launch_bounds__(NT, 1024 / NT)
 topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chunk_vecs,
@@ -455,16 +641,7 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   pdl_wait();
   constexpr int VEC = Vec<T>::N;
   constexpr int NW = NT / 32;
-  __shared__ uint64_t s_buf[NW][TK_CAP];         // the warps' candidates
-  __shared__ uint64_t s_tmp[NW][LILICORR_MAX_K];
-  __shared__ uint64_t s_keys[TK_MERGE_MAX];       // the splits' lists (last CTA)
-  __shared__ uint64_t s_merge[TK_MERGE_MAX];
-  __shared__ uint64_t s_top[LILICORR_MAX_K];
-  __shared__ float s_m[NW], s_s[NW];
-  __shared__ uint32_t s_cta_thr;                // CTA-wide value bound (order image)
-  __shared__ float s_wtop[NW];                  // the warps' r-th largest lane maxima
-  __shared__ int s_last, s_count;
-  __shared__ uint64_t s_bound;
+  __shared__ TkShared<NW> sh;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int split = blockIdx.x;
@@ -479,120 +656,31 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
   const int v_end = min(v_begin + chunk_vecs, nvec);
 
   WarpCand w;
-  w.buf = s_buf[warp];
-  w.tmp = s_tmp[warp];
+  w.buf = sh.buf[warp];
+  w.tmp = sh.tmp[warp];
   w.n = 0;
   w.thr = -INFINITY;
-  if (tid == 0) s_cta_thr = ord32(-INFINITY);
-  if (tid < NW) s_wtop[tid] = -INFINITY;
+  if (lane == 0) w.tmp[K - 1] = 0ull;
+  if (tid == 0) sh.cta_thr = ord32(-INFINITY);
+  if (tid < NW) sh.wtop[tid] = -INFINITY;
   __syncthreads();
 
   float m = -INFINITY, s = 0.f;
 
-  // scalar head [0, e0) and tail [e0 + nvec*VEC, V): warp 0 of split 0, one element per lane
-  if (split == 0 && warp == 0) {
-    const int tail0 = e0 + nvec * VEC;
-    const int nscalar = e0 + (V - tail0);
-    for (int base = 0; base < nscalar; base += 32) {
-      const int i = base + lane;
-      const bool valid = i < nscalar;
-      const int e = valid ? (i < e0 ? i : tail0 + (i - e0)) : 0;
-      float x[1] = {valid ? Vec<T>::scalar(rp, e) : -INFINITY};
-      lse_update<1>(m, s, x, valid);
-      warp_append<1>(w, x, (uint32_t)e, valid, K, lane);
-    }
-  }
+  // scalar head [0, e0), before the vectors, and scalar tail [e0 + nvec*VEC, V), after
+  // them: warp 0 of split 0, one element per lane (so that warp meets its ids in order)
+  const int tail0 = e0 + nvec * VEC;
+  const bool scalars = split == 0 && warp == 0;
+  if (scalars) scalar_part<T>(rp, 0, e0, K, lane, m, s, w);
 
   // main stream: batches of 16-byte vectors, the next one's loads in flight
   const uint4* vp = reinterpret_cast<const uint4*>(rp + e0);
-  stream_chunk<T, NT>(vp, v_begin, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &s_cta_thr, s_wtop);
-
-  // (max, sum) of the warp, then of the CTA
-  const float wm = warp_max(m);
-  float ws = (m == -INFINITY) ? 0.f : s * ex2((m - wm) * LOG2E);
-  ws = warp_sum(ws);
-  if (lane == 0) { s_m[warp] = wm; s_s[warp] = ws; }
-  // CTA top-K: keys of every warp's buffer at or above the CTA-wide bound, rank-counted.
-  // (the bound never exceeds the CTA's K-th value, so the K largest keys all survive)
-  if (lane == 0) atomicMax(&s_cta_thr, ord32(w.thr));
-  if (tid == 0) s_count = 0;
-  for (int i = tid; i < LILICORR_MAX_K; i += NT) s_top[i] = 0ull;
-  __syncthreads();
-  {
-    const float bound = unord32(s_cta_thr);
-    const int nw = w.n;
-    for (int i = lane; i < nw; i += 32) {
-      const uint64_t k = w.buf[i];
-      if (key_value(k) >= bound) {
-        const int pos = atomicAdd(&s_count, 1);
-        if (pos < TK_MERGE_MAX) s_merge[pos] = k;
-      }
-    }
-  }
-  __syncthreads();
-  if (s_count > TK_MERGE_MAX) {
-    // more survivors than the merge area holds (only with massive ties at the bound):
-    // compact every warp's buffer to its own top-K first, then merge those
-    warp_compact(w, K, lane);
-    if (lane < LILICORR_MAX_K) s_keys[warp * LILICORR_MAX_K + lane] = lane < w.n ? w.buf[lane] : 0ull;
-    __syncthreads();
-    cta_select<NT>(s_keys, NW, LILICORR_MAX_K, K, s_merge, &s_count, &s_bound, s_top);
-  } else {
-    rank_place(s_merge, s_count, K, s_top, tid, NT);
-    __syncthreads();
-  }
-
-  float cm = -INFINITY, cs = 0.f;
-  if (warp == 0) {
-    const float pm = lane < NW ? s_m[lane] : -INFINITY;
-    const float ps = lane < NW ? s_s[lane] : 0.f;
-    cm = warp_max(pm);
-    cs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - cm) * LOG2E));
-  }
-
-  if (splits == 1) {
-    if (warp == 0) write_row(row, K, cm, cs, s_top, pout, ids, logp, lse, status, lane);
-    return;
-  }
-
-  // publish this split's partial record, then take a ticket
-  Rec* rec = reinterpret_cast<Rec*>(partials + ((size_t)row * splits + split) * rec_bytes);
-  if (warp == 0) {
-    if (lane == 0) { rec->m = cm; rec->s = cs; }
-    if (lane < K) rec->keys[lane] = s_top[lane];
-    __threadfence();
-  }
-  __syncthreads();
-  if (tid == 0) {
-    const uint32_t ticket = atomicAdd(&counters[row], 1u);
-    s_last = (ticket == (uint32_t)(splits - 1));
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-
-  // last CTA of the row: merge all splits (their lists staged in shared memory)
-  const int n = splits * K;
-  for (int i = tid; i < n; i += NT) {
-    const Rec* r = reinterpret_cast<const Rec*>(partials + ((size_t)row * splits + i / K) * rec_bytes);
-    s_keys[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&r->keys[i % K]));
-  }
-  __syncthreads();
-  cta_select<NT>(s_keys, splits, K, K, s_merge, &s_count, &s_bound, s_top);
-  if (warp == 0) {
-    float pm = -INFINITY, ps = 0.f;
-    for (int i = lane; i < splits; i += 32) {
-      const Rec* r = reinterpret_cast<const Rec*>(partials + ((size_t)row * splits + i) * rec_bytes);
-      const float rm = __ldcg(&r->m), rs = __ldcg(&r->s);
-      if (rm == -INFINITY) continue;
-      if (rm > pm) { ps = ps * ex2((pm - rm) * LOG2E) + rs; pm = rm; }
-      else ps += rs * ex2((rm - pm) * LOG2E);
-    }
-    const float gm = warp_max(pm);
-    const float gs = warp_sum(pm == -INFINITY ? 0.f : ps * ex2((pm - gm) * LOG2E));
-    if (lane == 0) counters[row] = 0u;             // leave the workspace reusable
-    write_row(row, K, gm, gs, s_top, pout, ids, logp, lse, status, lane);
-  }
+  stream_chunk<T, NT>(vp, v_begin, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &sh.cta_thr,
+                      sh.wtop);
+  if (scalars) scalar_part<T>(rp, tail0, V, K, lane, m, s, w);
+  finish_piece<NT>(sh, w, m, s, row, K, splits, split,
+                   partials + (size_t)row * splits * rec_bytes, rec_bytes, counters, pout, ids,
+                   logp, lse, status);
 }
 
 // Merge of P vocabulary shards' partial records of one row (one CTA per row): the union
@@ -662,13 +750,14 @@ TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   p.splits = splits;
   p.threads = threads;
   p.chunk_vecs = ceil_div(max(nvec, 1), splits);
+  p.pieces = splits;
   p.rec_bytes = align_up(8 + 8 * (size_t)K, 16);
   return p;
 }
 
 size_t topk_ws_bytes(int rows, int V, int K, lilicorr_dtype_t dt) {
   const TopkPlan p = topk_plan(rows, V, K, dt);
-  return 256 + align_up((size_t)rows * 4, 256) + align_up((size_t)rows * p.splits * p.rec_bytes, 256);
+  return 256 + align_up((size_t)rows * 4, 256) + align_up((size_t)rows * p.pieces * p.rec_bytes, 256);
 }
 
 lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int rows, int V, int K,
@@ -678,8 +767,8 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
   const PartialOut pout{static_cast<unsigned char*>(partial_out), id_offset};
   if (rows == 0) return LILICORR_OK;
   const TopkPlan p = topk_plan(rows, V, K, dt);
-  dim3 grid(p.splits, rows);
   unsigned char* part = static_cast<unsigned char*>(partials);
+  dim3 grid(p.splits, rows);
   if (dt == LILICORR_BF16) {
     const uint16_t* x = static_cast<const uint16_t*>(logits);
     if (p.threads == TK_THREADS_MANY)

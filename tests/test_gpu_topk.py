@@ -135,6 +135,37 @@ def test_ties_zero_signs_and_minus_inf(dtype):
     _check_rows(x, 16, ids, logp, lse, range(6))
 
 
+@pytest.mark.parametrize("dtype,rows,V", [("bf16", 4, 151936), ("bf16", 512, 151936),
+                                          ("bf16", 3, 151937), ("f32", 6, 151937)])
+def test_full_width_tie_rows(dtype, rows, V):
+    """Vocabulary-wide runs of equal values: the K lowest ids among the tied maxima win,
+    on rows split over several CTAs (few rows) and on one CTA per row (512 rows), and with
+    rows that start off a 16-byte boundary (V odd), whose scalar head holds the lowest
+    ids and scalar tail the highest."""
+    K = 8
+    rng = np.random.default_rng(rows + V)
+    x = (rng.standard_normal((rows, V)) * 3).astype(np.float32)
+    special = [
+        np.full(V, 0.5, np.float32),                                    # all equal
+        np.where(np.arange(V) % 3 == 0, 0.0, -0.0).astype(np.float32),  # -0 == +0
+        (np.arange(V) % 7).astype(np.float32),                          # 21,706 tied maxima
+        np.round(rng.standard_normal(V) * 8) * 0.25,                    # quantised
+        np.full(V, -1.0, np.float32),                                   # maximum at the end
+        np.full(V, 2.0, np.float32),                                    # minimum at the start
+    ]
+    special[1][V // 2] = -1.0
+    special[4][-1] = 1.0
+    special[5][0] = 1.0
+    for r in range(min(rows, len(special))):
+        x[r] = special[r]
+    if dtype == "bf16":
+        x = workloads.round_to_bf16(x)
+    ids, logp, lse, st = _run(x, K, dtype)
+    assert st == 0
+    _check_rows(x, K, ids, logp, lse, list(range(min(rows, len(special)))) +
+                list(range(len(special), rows, 50)))
+
+
 @pytest.mark.parametrize("bad", ["nan", "all_minus_inf", "plus_inf"])
 def test_nonfinite_rows_set_device_status(bad):
     x = np.random.default_rng(0).standard_normal((4, 3000)).astype(np.float32)
