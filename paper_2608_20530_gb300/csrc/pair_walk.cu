@@ -7,9 +7,10 @@
 // c_s = argmax_k phi(s-1, c_{s-1}, k), touching no weights.
 //
 // pair_block_kernel: grid (B, L). CTA (b, j) scores the anchor row (j = 0) or the slot
-// pair (j-1, j): both slots' vectors are staged in shared memory and each thread forms
-// whole dot products (one output at a time). pair_rows_kernel, the same grid for vectors
-// too long to stage twice: it stages slot j's K in vectors and their norms, every warp
+// pair (j-1, j): both slots' vectors are staged in shared memory and the outputs are
+// formed in 4 x 4 blocks, 16 lanes per block. pair_rows_kernel, the same grid for vectors
+// too long to stage twice (or rows off 16-byte boundaries): it stages slot j's K in
+// vectors and their norms, every warp
 // takes rows of the earlier slot and forms K dot products by lane-strided loads and a
 // shuffle reduction. With the walk fused, the last CTA
 // of a sequence to finish (atomic ticket, nobody waits) loads the sequence's
@@ -142,80 +143,179 @@ __device__ __forceinline__ void walk_after_pairs(const PairWalkArgs& a, float* s
   }
 }
 
-// Row stride (floats) of the staged vectors: 16-byte aligned rows whose 16-byte pieces
-// start on different banks for consecutive rows.
-__host__ __device__ __forceinline__ int pw_stride(int d) { return (d + 3) / 4 * 4 + 4; }
+// pair_block_kernel's staging: rows padded to a multiple of 4 per slot, row stride d + 4.
+__host__ __device__ __forceinline__ int pb_rows(int K) { return (K + 3) / 4 * 4; }
+__host__ __device__ __forceinline__ size_t pb_smem_bytes(int K, int d) {
+  return sizeof(float) * (size_t)2 * pb_rows(K) * (d + 4);
+}
 
-// CTA (b, j): the slot pair (j - 1, j), or the anchor row (j = 0). Both slots' vectors
-// (K in vectors of slot j, K out vectors of slot j - 1 or the anchor's one) are staged in
-// shared memory by asynchronous copies, all issued before one wait; each warp takes the
-// norms of some rows; then thread t forms whole dot products, one output (k, k') at a time,
-// reading both rows from shared memory (no cross-lane reductions) and storing the cosine.
+__device__ __forceinline__ float dot4(const float4& x, const float4& y, float acc) {
+  return fmaf(x.x, y.x, fmaf(x.y, y.y, fmaf(x.z, y.z, fmaf(x.w, y.w, acc))));
+}
+
+// Dot products of the 4 x 4 block of rows x (xr..xr+3, the earlier slot) and y (yr..yr+3,
+// slot j) over the 16-byte columns f = split, split + 16, ... within [f0, f1); the thread's
+// squared norms of those rows alongside when nx / ny are asked for.
+__device__ __forceinline__ void block_dots(const float* sm, int ds, int xr, int yr, int f0, int f1,
+                                           int split, bool want_nx, bool want_ny,
+                                           float (&acc)[4][4], float (&nx)[4], float (&ny)[4]) {
+  for (int f = f0 + split; f < f1; f += 16) {
+    float4 xv[4], yv[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      xv[r] = *reinterpret_cast<const float4*>(sm + (size_t)(xr + r) * ds + 4 * f);
+      yv[r] = *reinterpret_cast<const float4*>(sm + (size_t)(yr + r) * ds + 4 * f);
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = dot4(xv[r], yv[c], acc[r][c]);
+    if (want_nx)
+#pragma unroll
+      for (int r = 0; r < 4; ++r) nx[r] = dot4(xv[r], xv[r], nx[r]);
+    if (want_ny)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) ny[c] = dot4(yv[c], yv[c], ny[c]);
+  }
+}
+
+// Sum over the 16 lanes that share a block (lanes 0-15 or 16-31 of the warp).
+template <int N>
+__device__ __forceinline__ void sum16(float (&v)[N]) {
+#pragma unroll
+  for (int o = 1; o < 16; o <<= 1)
+#pragma unroll
+    for (int i = 0; i < N; ++i) v[i] += __shfl_xor_sync(0xffffffffu, v[i], o);
+}
+
+// CTA (b, j): the slot pair (j - 1, j), or the anchor row (j = 0). The K in vectors of slot
+// j (rows 0 .. K-1) and the earlier slot's out vectors or the anchor (rows R ..) are staged
+// in shared memory by asynchronous copies in two column halves, so the products of the
+// first half run while the second lands. The nrows x K outputs go in 4 x 4 blocks: thread t
+// takes block t / 16 and the 16-byte columns t % 16, t % 16 + 16, ... of every row, so the
+// 16 lanes of a block read 256 consecutive bytes of a row (no bank conflicts) and each
+// loaded piece feeds four products; the 16 partial sums meet by shuffles. The row norms
+// come out of the same pass (blocks of the first row / column group).
 __global__ void __launch_bounds__(PW_THREADS) pair_block_kernel(PairWalkArgs a) {
   pdl_wait();
   extern __shared__ float sm[];
   __shared__ int s_last;
-  __shared__ float s_norm[2 * LILICORR_MAX_K];
+  __shared__ float s_nx[LILICORR_MAX_K], s_ny[LILICORR_MAX_K];
   __shared__ uint8_t s_back[LILICORR_MAX_L * LILICORR_MAX_K];
   __shared__ uint8_t s_path[LILICORR_MAX_L];
   const int b = blockIdx.x, j = blockIdx.y;
-  const int L = a.L, K = a.K, d = a.d, ds = pw_stride(d);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = PW_THREADS / 32;
+  const int L = a.L, K = a.K, d = a.d, ds = d + 4, d4 = d >> 2;
+  const int R = pb_rows(K);                         // first row of the earlier slot
   const int nrows = j == 0 ? 1 : K;                 // vectors of the earlier slot (or anchor)
+  const int nbx = (nrows + 3) >> 2, nby = R >> 2, nblk = nbx * nby;
   const float* inb = a.in + (size_t)(b * L + j) * K * a.ld_vec;
   const float* outb = j == 0 ? a.anchor + (size_t)b * d
                              : a.out + (size_t)(b * L + j - 1) * K * a.ld_vec;
   const int ldo = j == 0 ? d : a.ld_vec;
-  const bool v4 = ((d | a.ld_vec) & 3) == 0 && (reinterpret_cast<uintptr_t>(a.in) & 15) == 0 &&
-                  (reinterpret_cast<uintptr_t>(a.out) & 15) == 0 &&
-                  (reinterpret_cast<uintptr_t>(a.anchor) & 15) == 0;
-  // rows 0 .. K-1: in vectors of slot j; rows K .. K+nrows-1: out vectors (or the anchor)
-  if (v4) {
-    const int dv = d >> 2;
-    for (int i = threadIdx.x; i < (K + nrows) * dv; i += PW_THREADS) {
-      const int row = i / dv, c = 4 * (i - row * dv);
-      const float* src = row < K ? inb + (size_t)row * a.ld_vec + c : outb + (size_t)(row - K) * ldo + c;
-      cp16(sm + (size_t)row * ds + c, src);
-    }
-    cp_wait_all();
-  } else {
-    for (int i = threadIdx.x; i < (K + nrows) * d; i += PW_THREADS) {
-      const int row = i / d, c = i - row * d;
-      sm[(size_t)row * ds + c] = row < K ? inb[(size_t)row * a.ld_vec + c]
-                                         : outb[(size_t)(row - K) * ldo + c];
-    }
-  }
-  __syncthreads();
-  for (int v = warp; v < K + nrows; v += nw) {
-    float ss = 0.f;
-    for (int c = lane; c < d; c += 32) ss = fmaf(sm[(size_t)v * ds + c], sm[(size_t)v * ds + c], ss);
-    ss = warp_sum(ss);
-    if (lane == 0) s_norm[v] = fmaxf(sqrtf(ss), UNIT_EPS);
-  }
-  __syncthreads();
-  for (int o = threadIdx.x; o < nrows * K; o += PW_THREADS) {
-    const int r = o / K, k2 = o - r * K;
-    const float* x = sm + (size_t)(K + r) * ds;
-    const float* y = sm + (size_t)k2 * ds;
-    float acc0 = 0.f, acc1 = 0.f;
-    int c = 0;
-    if ((d & 3) == 0) {
-      for (; c < d; c += 8) {
-        const float4 x0 = *reinterpret_cast<const float4*>(x + c);
-        const float4 y0 = *reinterpret_cast<const float4*>(y + c);
-        acc0 = fmaf(x0.x, y0.x, fmaf(x0.y, y0.y, fmaf(x0.z, y0.z, fmaf(x0.w, y0.w, acc0))));
-        if (c + 4 < d) {
-          const float4 x1 = *reinterpret_cast<const float4*>(x + c + 4);
-          const float4 y1 = *reinterpret_cast<const float4*>(y + c + 4);
-          acc1 = fmaf(x1.x, y1.x, fmaf(x1.y, y1.y, fmaf(x1.z, y1.z, fmaf(x1.w, y1.w, acc1))));
-        }
+  const int h4 = (d4 + 1) >> 1;                     // 16-byte columns of the first half
+  // stage both column halves (two commit groups), a warp per row and a lane per 16-byte
+  // column; padding rows read as zero
+  const int nr = R + 4 * nbx;
+  const int wp = threadIdx.x >> 5, ln = threadIdx.x & 31;
+  for (int h = 0; h < 2; ++h) {
+    const int f0 = h ? h4 : 0, f1 = h ? d4 : h4;
+    for (int row = wp; row < nr; row += PW_THREADS / 32) {
+      const bool in_row = row < R;
+      const int k = in_row ? row : row - R;
+      float* dst = sm + (size_t)row * ds;
+      if (k < (in_row ? K : nrows)) {
+        const float* src = in_row ? inb + (size_t)k * a.ld_vec : outb + (size_t)k * ldo;
+        for (int f = f0 + ln; f < f1; f += 32) cp16(dst + 4 * f, src + 4 * f);
+      } else {
+        for (int f = f0 + ln; f < f1; f += 32)
+          *reinterpret_cast<float4*>(dst + 4 * f) = make_float4(0.f, 0.f, 0.f, 0.f);
       }
-    } else {
-      for (; c < d; ++c) acc0 = fmaf(x[c], y[c], acc0);
     }
-    const float v = (acc0 + acc1) / (s_norm[K + r] * s_norm[k2]);
-    if (j == 0) a.A[(size_t)b * K + k2] = v;
-    else a.P[((size_t)b * (L - 1) + (j - 1)) * K * K + (size_t)r * K + k2] = v;
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+
+  const int split = threadIdx.x & 15;
+  float* outp = j == 0 ? a.A + (size_t)b * K
+                       : a.P + ((size_t)b * (L - 1) + (j - 1)) * K * K;
+  // this lane's output of a reduced block: row 4 bx + split / 4, column 4 by + split % 4
+  auto put = [&](int bx, int by, const float (&acc)[4][4]) {
+    float v = 0.f;
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v = split == 4 * r + c ? acc[r][c] : v;
+    const int r = 4 * bx + (split >> 2), k2 = 4 * by + (split & 3);
+    if (r < nrows && k2 < K) outp[(size_t)r * K + k2] = v / (s_nx[r] * s_ny[k2]);
+  };
+  auto put_norms = [&](int bx, int by, const float (&nx)[4], const float (&ny)[4]) {
+    if (split != 0) return;
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      if (by == 0 && 4 * bx + r < nrows) s_nx[4 * bx + r] = fmaxf(sqrtf(nx[r]), UNIT_EPS);
+      if (bx == 0 && 4 * by + r < K) s_ny[4 * by + r] = fmaxf(sqrtf(ny[r]), UNIT_EPS);
+    }
+  };
+
+  if (nblk <= PW_THREADS / 16) {
+    // one block per thread (K <= 16): the first half's products while the second lands
+    const int blk = threadIdx.x >> 4;
+    const bool active = blk < nblk;
+    const int bx = active ? blk / nby : 0, by = active ? blk % nby : 0;
+    float acc[4][4] = {}, nx[4] = {}, ny[4] = {};
+    asm volatile("cp.async.wait_group 1;" ::: "memory");
+    __syncthreads();
+    if (active) block_dots(sm, ds, R + 4 * bx, 4 * by, 0, h4, split, by == 0, bx == 0, acc, nx, ny);
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    if (active) block_dots(sm, ds, R + 4 * bx, 4 * by, h4, d4, split, by == 0, bx == 0, acc, nx, ny);
+    sum16(nx);
+    sum16(ny);
+    if (active) put_norms(bx, by, nx, ny);
+    float flat[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) flat[i] = acc[i >> 2][i & 3];
+    sum16(flat);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) acc[i >> 2][i & 3] = flat[i];
+    __syncthreads();                               // the norms
+    if (active) put(bx, by, acc);
+  } else {
+    // more blocks than the CTA holds at once (K > 16): norms first, then block after block
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    for (int blk0 = 0; blk0 < nbx + nby; blk0 += PW_THREADS / 16) {
+      // norms of row group blk (x rows for blk < nbx, else y rows), as blocks with bx or by 0
+      // (the loop is warp-uniform: the sums below take every lane)
+      const int blk = blk0 + (threadIdx.x >> 4);
+      const bool act = blk < nbx + nby;
+      float acc[4][4] = {}, nx[4] = {}, ny[4] = {};
+      const bool xs = blk < nbx;
+      const int bx = xs ? blk : 0, by = xs ? 0 : (act ? blk - nbx : 0);
+      if (act) block_dots(sm, ds, R + 4 * bx, 4 * by, 0, d4, split, xs, !xs, acc, nx, ny);
+      sum16(nx);
+      sum16(ny);
+      if (act && split == 0)
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          if (xs && 4 * bx + r < nrows) s_nx[4 * bx + r] = fmaxf(sqrtf(nx[r]), UNIT_EPS);
+          if (!xs && 4 * by + r < K) s_ny[4 * by + r] = fmaxf(sqrtf(ny[r]), UNIT_EPS);
+        }
+    }
+    __syncthreads();
+    for (int blk0 = 0; blk0 < nblk; blk0 += PW_THREADS / 16) {
+      const int blk = blk0 + (threadIdx.x >> 4);
+      const bool active = blk < nblk;                // warp-uniform: 2 blocks per warp
+      const int bx = active ? blk / nby : 0, by = active ? blk % nby : 0;
+      float acc[4][4] = {}, nx[4], ny[4];
+      if (active) block_dots(sm, ds, R + 4 * bx, 4 * by, 0, d4, split, false, false, acc, nx, ny);
+      float flat[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) flat[i] = acc[i >> 2][i & 3];
+      sum16(flat);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) acc[i >> 2][i & 3] = flat[i];
+      if (active) put(bx, by, acc);
+    }
   }
   if (!a.do_walk) return;
   walk_after_pairs(a, sm, &s_last, s_back, s_path);
@@ -366,9 +466,12 @@ lilicorr_status_t launch_pair_walk(const PairWalkArgs& in, cudaStream_t st) {
   static bool cfg_pair[64] = {false}, cfg_walk[64] = {false};
   if (a.do_pairs) {
     if (a.do_walk && !a.counters) return LILICORR_ERR_ARG;
-    // both slots' vectors staged: when that stays within 100 KB (two CTAs per SM at least)
-    const size_t block_smem = sizeof(float) * (size_t)2 * a.K * pw_stride(a.d);
-    if (block_smem <= 100 * 1024) {
+    // both slots' vectors staged, 16-byte pieces: when the rows are 16-byte aligned and the
+    // staging stays within 100 KB (two CTAs per SM at least)
+    const size_t block_smem = pb_smem_bytes(a.K, a.d);
+    const bool v4 = ((a.d | a.ld_vec) & 3) == 0 && aligned16(a.in) && aligned16(a.out) &&
+                    aligned16(a.anchor);
+    if (v4 && block_smem <= 100 * 1024) {
       static bool cfg_block[64] = {false};
       size_t smem = block_smem;
       if (a.do_walk && a.scores_in_smem && score_bytes > smem) smem = score_bytes;

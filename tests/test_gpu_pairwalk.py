@@ -20,7 +20,8 @@ def _ll():
 @pytest.mark.parametrize("B,L,K,d,unit", [(1, 8, 4, 64, True), (3, 16, 8, 256, True),
                                           (2, 16, 16, 512, True), (5, 1, 3, 40, True),
                                           (2, 6, 32, 24, False), (4, 3, 1, 8, False),
-                                          (7, 15, 8, 1024, True)])
+                                          (7, 15, 8, 1024, True), (2, 5, 20, 36, True),
+                                          (3, 4, 32, 256, False)])
 def test_pair_scores_match_oracle(B, L, K, d, unit):
     ll = _ll()
     rng = np.random.default_rng(B * 100 + L * 10 + K + d)
