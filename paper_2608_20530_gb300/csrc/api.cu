@@ -169,6 +169,7 @@ WsLayout ws_layout(const lilicorr_head_desc& d, int B) {
   w.P = take((size_t)B * (d.L > 1 ? d.L - 1 : 0) * d.K * d.K * 4);
   w.choice = take(R * 4);
   w.pw_counters = take((size_t)B * 4);
+  w.ss = take(Np * SS_LD * 4);
   w.total = o;
   return w;
 }
@@ -197,7 +198,15 @@ GemmArgs gemm(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W, lili
 
 // Few rows: split-N CUDA-core kernel. bf16 operands: tensor cores. Otherwise the
 // tiled fp32 CUDA-core kernel (the fp32 head keeps fp32 arithmetic throughout).
+// The persistent tensor-core kernel is the one run_gemm picks for g.
+bool takes_gemm_tc(const GemmArgs& g) {
+  return !(g.M <= 64 || (g.a_dt == LILICORR_F32 && g.M <= 1024)) && !gemm_small_supported(g) &&
+         gemm_tc_supported(g);
+}
+
 lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
+  // a folded RMSNorm only exists in the persistent tensor-core kernel
+  if (g.c2 || g.ss_in) return takes_gemm_tc(g) ? launch_gemm_tc(g, st) : LILICORR_ERR_SHAPE;
   // few rows, or fp32 activations (the tensor-core kernels take bf16) at per-sequence row
   // counts: the split-N kernel spreads the weights over many CTAs
   if (g.M <= 64 || (g.a_dt == LILICORR_F32 && g.M <= 1024)) return launch_gemm_skinny(g, st);
@@ -215,7 +224,7 @@ struct HeadCall {
   bool tc_attn;                          // tensor-core attention core
   uint32_t* status;
   lilicorr_dtype_t tn_dt;                // normalised target state (an operand of W_t)
-  float *hproj, *t, *anc, *cb, *x, *oi;
+  float *hproj, *t, *anc, *cb, *x, *oi, *ss;
   void *tn, *c1, *xn, *qkv, *att, *hf, *u;
 
   HeadCall(const lilicorr_head* head, int b, void* ws, const WsLayout& w)
@@ -241,6 +250,7 @@ struct HeadCall {
     cb = at<float>(ws, w.cb);
     x = at<float>(ws, w.x);
     oi = at<float>(ws, w.oi);
+    ss = at<float>(ws, w.ss);
     c1 = at<void>(ws, w.c1);
     xn = at<void>(ws, w.xn);
     qkv = at<void>(ws, w.qkv);
@@ -253,6 +263,15 @@ struct HeadCall {
     GemmArgs g = gemm(A, a_dt, lda, W, wdt, ldw, C, c_dt, ldc, M, Nn, Kd);
     g.status = status;
     return g;
+  }
+  // RMSNorm folded around a product (App. A's pre-norm x / rms(x) * gain): the product
+  // writing the fp32 state also writes bf16(state * gain) into xn and its row sums of
+  // squares; the next product reads xn and scales its rows by 1 / rms.
+  void norm_out(GemmArgs& g, const float* gain) const {
+    g.c2 = xn; g.ldc2 = D; g.c2_gain = gain; g.ss_out = ss;
+  }
+  void norm_in(GemmArgs& g) const {
+    g.ss_in = ss; g.ss_slots = gemm_tc_ss_slots(N, D);
   }
 };
 
@@ -316,6 +335,28 @@ lilicorr_status_t join_prologue(const lilicorr_head* h, cudaStream_t st) {
   return LILICORR_OK;
 }
 
+// Whether every product around the chain's RMSNorms takes the persistent tensor-core
+// kernel (the only one that folds a norm): bf16 heads with more node rows than one tile.
+bool fold_norms(const HeadCall& c) {
+  const lilicorr_head* h = c.h;
+  const int D = c.D, F = c.F, N = c.N;
+  const lilicorr_dtype_t adt = c.adt, F32 = LILICORR_F32;
+  if (c.wdt != LILICORR_BF16) return false;
+  GemmArgs p[5] = {c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D),
+                   c.G(c.xn, adt, D, h->layer[0].wqkv, D, c.qkv, c.qkv_dt, 3 * D, N, 3 * D, D),
+                   c.G(c.att, adt, D, h->layer[0].wo, D, c.x, F32, D, N, D, D),
+                   c.G(c.xn, adt, D, h->layer[0].w1, D, c.hf, adt, F, N, F, D),
+                   c.G(c.hf, adt, F, h->layer[0].w2, F, c.x, F32, D, N, D, F)};
+  for (int i : {0, 2, 4}) {
+    p[i].residual = c.x; p[i].ldr = D;
+    c.norm_out(p[i], h->layer[0].an);
+  }
+  for (int i : {1, 3}) c.norm_in(p[i]);
+  for (const GemmArgs& g : p)
+    if (!takes_gemm_tc(g)) return false;
+  return true;
+}
+
 // Candidate-dependent part, after the prologue: nodes, the Transformer, fusion and the
 // out/in heads. Writes oi = [W_o u + b_o | W_i u + b_i] (not yet normalised).
 // With `tail`, the cluster kernel also forms the pair scores and walks; *tail_done says
@@ -348,13 +389,18 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
   GemmArgs g = c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D);
   g.bias = h->conf2_b;
   g.residual = c.x; g.ldr = D;
+  // the RMSNorms fold into the products around them when every one of those runs on the
+  // persistent tensor-core kernel; otherwise each is a kernel of its own
+  const bool fold = fold_norms(c);
+  if (fold) c.norm_out(g, h->layer[0].an);
   LL_TRY(run_gemm(g, st));
   // Transformer layers
   for (int i = 0; i < d.n_layers; ++i) {
     const HeadW& l = h->layer[i];
-    LL_TRY(launch_rmsnorm(c.x, N, D, l.an, c.xn, adt, st));
+    if (!fold) LL_TRY(launch_rmsnorm(c.x, N, D, l.an, c.xn, adt, st));
     g = c.G(c.xn, adt, D, l.wqkv, D, c.qkv, c.qkv_dt, 3 * D, N, 3 * D, D);
     g.bias = l.bqkv;
+    if (fold) c.norm_in(g);
     LL_TRY(run_gemm(g, st));
     if (c.tc_attn)
       LL_TRY(launch_attention_tc(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att, st));
@@ -364,15 +410,19 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
     g = c.G(c.att, adt, D, l.wo, D, c.x, F32, D, N, D, D);
     g.bias = l.bo;
     g.residual = c.x; g.ldr = D;
+    if (fold) c.norm_out(g, l.fn);
     LL_TRY(run_gemm(g, st));
-    LL_TRY(launch_rmsnorm(c.x, N, D, l.fn, c.xn, adt, st));
+    if (!fold) LL_TRY(launch_rmsnorm(c.x, N, D, l.fn, c.xn, adt, st));
     g = c.G(c.xn, adt, D, l.w1, D, c.hf, adt, F, N, F, D);
     g.bias = l.b1;
     g.act = ACT_SILU;
+    if (fold) c.norm_in(g);
     LL_TRY(run_gemm(g, st));
     g = c.G(c.hf, adt, F, l.w2, F, c.x, F32, D, N, D, F);
     g.bias = l.b2;
     g.residual = c.x; g.ldr = D;
+    // the last layer's output goes to the final norm inside the fusion input instead
+    if (fold && i + 1 < d.n_layers) c.norm_out(g, h->layer[i + 1].an);
     LL_TRY(run_gemm(g, st));
   }
   // fusion u = SiLU(W_f [x; t; x*t] + b_f) with x the final-normed state

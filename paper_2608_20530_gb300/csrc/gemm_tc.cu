@@ -32,6 +32,7 @@ constexpr int TC_THREADS = 320;            // producer, MMA, 8 epilogue warps
 constexpr int EPI_THREADS = 256;
 constexpr uint32_t CHUNK_BYTES = 128 * 128;   // staging chunk: 128 rows x 128 bytes
 constexpr long long WAIT_LIMIT_CYCLES = 4000000000ll;   // about 2 s at the SM clock
+constexpr float TC_RMS_EPS = 1e-6f;                    // the network's RMSNorm epsilon
 
 __device__ __forceinline__ void epi_bar() {   // the 8 epilogue warps only
   asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
@@ -54,6 +55,13 @@ struct TcEpilogue {
   const float* bias_rows; int rows_per_bias;
   int has_residual;
   int act;
+  // RMSNorm of the output rows folded into the next product (fp32 outputs): the output
+  // times `c2_gain` per column, rounded to bf16, into c2 [M, ldc2], and each thread's sum of
+  // squares of its part of the row into ss_out[m * SS_LD + 2 * column tile + half]
+  __nv_bfloat16* c2; int ldc2; const float* c2_gain; float* ss_out;
+  // ...and its use: the accumulator scaled by rsqrt(sum of ss_in[m * SS_LD + 0..ss_slots) *
+  // ss_scale + eps) before the bias
+  const float* ss_in; int ss_slots; float ss_scale;
 };
 
 template <int BN, bool OUT_BF16>
@@ -65,10 +73,12 @@ struct TcCfg {
   static constexpr int NCH = BN / CH;
   static constexpr uint32_t TMEM_COLS = 2 * BN;         // two accumulators
   static constexpr size_t RING = (size_t)STAGES * (A_BYTES + B_BYTES);
-  static constexpr size_t SMEM = 1024 + RING + 4 * (size_t)CHUNK_BYTES + BN * sizeof(float);
+  static constexpr size_t SMEM = 1024 + RING + 4 * (size_t)CHUNK_BYTES + 2 * BN * sizeof(float);
 };
 
-template <int BN, bool OUT_BF16>
+// FOLD: the instantiation with the folded-RMSNorm epilogue (c2 / ss_out, ss_in); the
+// others leave that code out and keep their registers.
+template <int BN, bool OUT_BF16, bool FOLD>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
                    const __grid_constant__ CUtensorMap mapW,
@@ -85,6 +95,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint8_t* s_out = smem + Cfg::RING;                   // 2 staging chunks
   uint8_t* s_res = s_out + 2 * CHUNK_BYTES;            // 2 residual chunks
   float* s_bias = reinterpret_cast<float*>(s_res + 2 * CHUNK_BYTES);
+  float* s_gain = s_bias + BN;                         // c2_gain of the tile's columns
   __shared__ __align__(8) uint64_t full[S], empty[S], acc_full[2], acc_empty[2], res_full[2];
   __shared__ uint32_t tmem_base;
   __shared__ volatile int abort_flag;
@@ -188,12 +199,25 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       tma_load_2d(s_res + (k & 1u) * CHUNK_BYTES, &mapR, bar, n0 + c * CH, m0);
     };
     if (ep.has_residual && leader && (int)blockIdx.x < tiles) issue_res(blockIdx.x, 0, 0);
+    // folded RMSNorm of the input rows: the row's sums of squares, loaded a tile ahead
+    float4 ssn[SS_LD / 4];
+    auto load_ss = [&](int t) {
+      const int mm = (t / tiles_n) * TC_BM + row;
+      const float4* src = reinterpret_cast<const float4*>(ep.ss_in + (size_t)mm * SS_LD);
+#pragma unroll
+      for (int i = 0; i < SS_LD / 4; ++i)
+        ssn[i] = (t < tiles && mm < M && 4 * i < ep.ss_slots) ? src[i]
+                                                              : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    if (FOLD && ep.ss_in) load_ss(blockIdx.x);
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++lt) {
       const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
       const uint32_t acc = lt & 1u;
       epi_bar();                                  // s_bias free again
-      for (int j = threadIdx.x - 64; j < BN; j += EPI_THREADS)
+      for (int j = threadIdx.x - 64; j < BN; j += EPI_THREADS) {
         s_bias[j] = (ep.bias && n0 + j < N) ? ep.bias[n0 + j] : 0.f;
+        if (FOLD && !OUT_BF16 && ep.c2) s_gain[j] = n0 + j < N ? ep.c2_gain[n0 + j] : 0.f;
+      }
       if (!abort_flag && !mbar_wait(&acc_full[acc], (lt >> 1) & 1u, wait_limit))
         abort_flag = 1;
       tc_fence_after();
@@ -201,6 +225,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int m = m0 + row;
       const float* brow = (ep.bias_rows && m < M)
                               ? ep.bias_rows + (size_t)(m / ep.rows_per_bias) * N : nullptr;
+      float rs = 1.f;                             // folded RMSNorm of the input rows
+      if (FOLD && ep.ss_in) {
+        float sum = 0.f;                          // slots past ss_slots hold zeros
+#pragma unroll
+        for (int i = 0; i < SS_LD / 4; ++i) sum += (ssn[i].x + ssn[i].y) + (ssn[i].z + ssn[i].w);
+        rs = rsqrtf(sum * ep.ss_scale + TC_RMS_EPS);
+        load_ss(t + gridDim.x);
+      }
+      float ssq = 0.f;                            // this thread's squares of the output row
 #pragma unroll 1
       for (int c = 0; c < NCH; ++c, ++cc) {
         const uint32_t b = cc & 1u;
@@ -236,9 +269,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           abort_flag = 1;
 #pragma unroll
         for (int j = 0; j < HC; j += 4) {
-          float4 x = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
           const float4 bb = *reinterpret_cast<const float4*>(s_bias + cl + j);
-          x.x += bb.x; x.y += bb.y; x.z += bb.z; x.w += bb.w;
+          // the product (scaled per row by a folded RMSNorm) plus the bias
+          float4 x = make_float4(fmaf(v[j], rs, bb.x), fmaf(v[j + 1], rs, bb.y),
+                                 fmaf(v[j + 2], rs, bb.z), fmaf(v[j + 3], rs, bb.w));
           if (brow && n0 + cl + j < N) {
             const float4 br = *reinterpret_cast<const float4*>(brow + n0 + cl + j);
             x.x += br.x; x.y += br.y; x.z += br.z; x.w += br.w;
@@ -256,6 +290,34 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             x.x += rr.x; x.y += rr.y; x.z += rr.z; x.w += rr.w;
           }
           v[j] = x.x; v[j + 1] = x.y; v[j + 2] = x.z; v[j + 3] = x.w;
+        }
+        if constexpr (FOLD && !OUT_BF16) {
+          if (ep.c2) {                      // the next RMSNorm's input, and its sums
+            uint32_t wv[HC / 2];
+#pragma unroll
+            for (int j = 0; j < HC; j += 2) {
+              ssq = fmaf(v[j], v[j], fmaf(v[j + 1], v[j + 1], ssq));
+              wv[j / 2] = pack_bf16x2(v[j] * s_gain[cl + j], v[j + 1] * s_gain[cl + j + 1]);
+            }
+            // the warp holds 32 rows x 32 bytes: lanes 2i and 2i+1 store the two halves
+            // of row i (then of row 16 + i), one whole 32-byte sector per pair
+            static_assert(HC == 16, "fp32 chunk halves of 16 columns");
+#pragma unroll
+            for (int rd = 0; rd < 2; ++rd) {
+              const int src = 16 * rd + (lane >> 1), piece = lane & 1;
+              uint32_t o[4];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const uint32_t a0 = __shfl_sync(0xffffffffu, wv[k], src);
+                const uint32_t a1 = __shfl_sync(0xffffffffu, wv[4 + k], src);
+                o[k] = piece ? a1 : a0;
+              }
+              const int mr = m0 + q * 32 + src;
+              if (mr < M && n0 + cl < N)
+                *reinterpret_cast<uint4*>(ep.c2 + (size_t)mr * ep.ldc2 + n0 + cl + 8 * piece) =
+                    make_uint4(o[0], o[1], o[2], o[3]);
+            }
+          }
         }
         epi_bar();          // staging buffer b: its store two chunks ago has been read
         uint8_t* stg = s_out + b * CHUNK_BYTES;
@@ -282,6 +344,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           tma_store_wait_read_le1();         // the other buffer is free for the next chunk
         }
       }
+      if (FOLD && !OUT_BF16 && ep.c2 && m < M)
+        ep.ss_out[(size_t)m * SS_LD + 2 * (t % tiles_n) + half] = ssq;
     }
     if (leader) tma_store_wait_all();
   }
@@ -307,11 +371,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   }
 }
 
-template <int BN, bool OUT_BF16>
+template <int BN, bool OUT_BF16, bool FOLD>
 lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   using Cfg = TcCfg<BN, OUT_BF16>;
   static bool configured[64] = {false};
-  LL_TRY(allow_max_dynamic_smem(gemm_tc_kernel<BN, OUT_BF16>, configured));
+  LL_TRY(allow_max_dynamic_smem(gemm_tc_kernel<BN, OUT_BF16, FOLD>, configured));
   CUtensorMap ma, mw, mc, mr;
   const CUtensorMapDataType bf = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const CUtensorMapDataType f32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
@@ -330,22 +394,36 @@ lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   ep.rows_per_bias = g.rows_per_bias;
   ep.has_residual = g.residual != nullptr;
   ep.act = g.act;
+  ep.c2 = static_cast<__nv_bfloat16*>(g.c2);
+  ep.ldc2 = g.ldc2;
+  ep.c2_gain = g.c2_gain;
+  ep.ss_out = g.ss_out;
+  ep.ss_in = g.ss_in;
+  ep.ss_slots = g.ss_slots;
+  ep.ss_scale = 1.0f / (float)g.Kd;
   const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
   const long long wait = g.wait_limit > 0 ? g.wait_limit : WAIT_LIMIT_CYCLES;
-  LL_TRY(launch_k(gemm_tc_kernel<BN, OUT_BF16>, grid, TC_THREADS, Cfg::SMEM, st, ma, mw, mc, mr, ep,
+  LL_TRY(launch_k(gemm_tc_kernel<BN, OUT_BF16, FOLD>, grid, TC_THREADS, Cfg::SMEM, st, ma, mw, mc, mr, ep,
                   g.M, g.N, g.Kd, g.status, wait, g.test_starve));
   return LILICORR_OK;
 }
 
-template <bool OUT_BF16>
-lilicorr_status_t launch_out(const GemmArgs& g, cudaStream_t st) {
-  // column tile: the widest of 256/128/64 that still gives every SM a tile
-  const int mt = ceil_div(g.M, TC_BM);
+// Column tile: the widest of 256/128/64 that still gives every SM a tile.
+int tc_column_tile(int M, int N) {
+  const int mt = ceil_div(M, TC_BM);
   const int sms = num_sms();
-  if (g.N >= 256 && mt * ceil_div(g.N, 256) >= sms) return launch_bn<256, OUT_BF16>(g, st);
-  if (g.N >= 128 && mt * ceil_div(g.N, 128) >= sms / 2) return launch_bn<128, OUT_BF16>(g, st);
-  return launch_bn<64, OUT_BF16>(g, st);
+  if (N >= 256 && mt * ceil_div(N, 256) >= sms) return 256;
+  if (N >= 128 && mt * ceil_div(N, 128) >= sms / 2) return 128;
+  return 64;
+}
+
+template <bool OUT_BF16, bool FOLD>
+lilicorr_status_t launch_out(const GemmArgs& g, cudaStream_t st) {
+  const int bn = tc_column_tile(g.M, g.N);
+  if (bn == 256) return launch_bn<256, OUT_BF16, FOLD>(g, st);
+  if (bn == 128) return launch_bn<128, OUT_BF16, FOLD>(g, st);
+  return launch_bn<64, OUT_BF16, FOLD>(g, st);
 }
 
 }  // namespace
@@ -397,8 +475,15 @@ bool make_map_nd(CUtensorMap* map, const void* base, CUtensorMapDataType type, i
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int gemm_tc_ss_slots(int M, int N) { return 2 * ceil_div(N, tc_column_tile(M, N)); }
+
 bool gemm_tc_supported(const GemmArgs& g) {
   if (g.a_dt != LILICORR_BF16 || g.w_dt != LILICORR_BF16) return false;
+  // folded RMSNorm: fp32 output, whole 32-column groups, 16-byte aligned bf16 copy rows
+  if (g.c2 && (g.c_dt != LILICORR_F32 || !g.c2_gain || !g.ss_out || (g.N % 32) ||
+               !aligned16(g.c2) || (g.ldc2 % 8) || gemm_tc_ss_slots(g.M, g.N) > SS_LD))
+    return false;
+  if (g.ss_in && (g.ss_slots < 1 || g.ss_slots > SS_LD)) return false;
   if (g.M <= 0 || g.N <= 0 || g.Kd <= 0) return false;
   // TMA: 16-byte aligned bases and row strides, outputs in 16-byte column groups
   if (!aligned16(g.A) || !aligned16(g.W) || !aligned16(g.C)) return false;
@@ -410,7 +495,10 @@ bool gemm_tc_supported(const GemmArgs& g) {
 }
 
 lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st) {
-  return g.c_dt == LILICORR_BF16 ? launch_out<true>(g, st) : launch_out<false>(g, st);
+  const bool fold = g.c2 || g.ss_in;
+  if (g.c_dt == LILICORR_BF16)
+    return fold ? launch_out<true, true>(g, st) : launch_out<true, false>(g, st);
+  return fold ? launch_out<false, true>(g, st) : launch_out<false, false>(g, st);
 }
 
 }  // namespace lilicorr

@@ -210,6 +210,7 @@ struct WsLayout {
   size_t hproj, tn, t, anc, cb;
   size_t x, c1, xn, qkv, att, hf, u, oi;
   size_t A, P, choice, pw_counters;
+  size_t ss;           // folded RMSNorm: row sums of squares [N, SS_LD]
   size_t total;
 };
 WsLayout ws_layout(const lilicorr_head_desc& d, int B);
@@ -268,7 +269,15 @@ struct GemmArgs {
   long long wait_limit;    // SM cycles per bounded wait of the tensor-core kernel; 0: ~2 s
   int test_starve;         // test hook only: the tensor-core kernel's producer issues no
                            // copies, so its consumers' waits run out (see the testing header)
+  // RMSNorm folded into the products around it (tensor-core kernel only). Producer (fp32 C):
+  // c2 [M, ldc2] (bf16) receives C times c2_gain per column, ss_out [M, SS_LD] partial sums of
+  // squares of C's rows (gemm_tc_ss_slots(M, N) slots per row). Consumer: the product is
+  // scaled per row by rsqrt(sum of ss_in's first ss_slots slots / Kd + eps) before the bias.
+  void* c2; int ldc2; const float* c2_gain; float* ss_out;
+  const float* ss_in; int ss_slots;
 };
+constexpr int SS_LD = 16;  // floats per row of a folded-RMSNorm sums-of-squares buffer
+int gemm_tc_ss_slots(int M, int N);
 lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
 lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st);   // M <= 64
 bool gemm_tc_supported(const GemmArgs& g);
