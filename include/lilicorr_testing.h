@@ -55,6 +55,14 @@ lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, flo
  * kernel that `mode` names, else 0. */
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode);
 
+/* Switch for the chain's attention core (Sec. 3.2 and App. A: bidirectional attention
+ * with the slot-distance and same-slot biases, bf16 heads): mode 1 runs it on the
+ * tcgen05 tensor cores where the head width is 32 or 64 and a sequence has at most 256
+ * nodes, mode 0 on the mma.sync kernel, mode 2 (the default) on tcgen05 for sequences of
+ * exactly 256 nodes whose slots hold a multiple of 8 candidates and on mma.sync otherwise.
+ * Process-wide, like the switch above. Returns the previous mode. */
+int lilicorr_test_attention_path(int mode);
+
 #ifdef __cplusplus
 }
 #endif

@@ -69,6 +69,7 @@ _SIGS = {
     "lilicorr_get_device_status": (_I, [_P, _P]),
     "lilicorr_launch_count": (ctypes.c_uint64, []),
     "lilicorr_test_fused_path": (_I, [_P, _I]),
+    "lilicorr_test_attention_path": (_I, [_I]),
     "lilicorr_topk_lse_noalloc_max_bytes": (_S, []),
     "lilicorr_topk_partial_bytes": (_S, [_I]),
     "lilicorr_lm_head_topk_workspace_bytes": (_S, [_I, _I, _I, _I]),
@@ -505,6 +506,12 @@ def test_linear_timeout(A: torch.Tensor, W: torch.Tensor, wait_cycles: int,
                                               int(wait_cycles), status.data_ptr(), _stream()),
            "test_linear_timeout")
     return C
+
+
+def test_attention_path(mode: int) -> int:
+    """Test hook: the chain's attention core on tcgen05 where supported (1), on the
+    mma.sync kernel (0), or by shape (2, the default); returns the previous mode."""
+    return int(lib().lilicorr_test_attention_path(int(mode)))
 
 
 def test_fused_path(head: Optional[Head], mode: int) -> bool:

@@ -15,7 +15,7 @@ INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "lib")
 LIB = os.path.join(LIBDIR, "liblilicorr.so")
 SOURCES = ["api.cu", "topk_lse.cu", "head_kernels.cu", "pair_walk.cu", "gemm_tc.cu",
-           "attention_tc.cu", "net_fused.cu",
+           "attention_tc.cu", "attention_umma.cu", "net_fused.cu",
            "diagnostics.cu", "gemm_small.cu", "lm_head.cu",
            "net_cluster.cu", "net_pair.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

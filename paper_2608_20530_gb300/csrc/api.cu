@@ -18,6 +18,11 @@ size_t pair_walk_smem_bytes(int L, int K, int d);
 
 static std::atomic<uint64_t> g_launches{0};
 int g_fused_enabled = 1;
+// The chain's attention core: 0 the mma.sync kernel, 1 the tcgen05 kernel wherever it
+// applies, 2 (the default) the tcgen05 kernel on full 256-node tiles with slots in 8-node
+// groups (where it was measured faster: 104 against 179 us per launch at 256 sequences x
+// 8 heads of 64), the mma.sync kernel elsewhere.
+int g_attn_umma = 2;
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 int num_sms() {
@@ -402,7 +407,11 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
     g.bias = l.bqkv;
     if (fold) c.norm_in(g);
     LL_TRY(run_gemm(g, st));
-    if (c.tc_attn)
+    if (c.tc_attn && attention_umma_supported(d.L, d.K, D, d.n_heads) &&
+        (g_attn_umma == 1 || (g_attn_umma == 2 && d.L * d.K == 256 && d.K % 8 == 0)))
+      LL_TRY(launch_attention_umma(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att,
+                                   c.status, st));
+    else if (c.tc_attn)
       LL_TRY(launch_attention_tc(c.qkv, c.B, d.L, d.K, D, d.n_heads, l.dist, l.same, c.att, st));
     else
       LL_TRY(launch_attention(static_cast<const float*>(c.qkv), c.B, d.L, d.K, D, d.n_heads,
@@ -917,6 +926,12 @@ lilicorr_status_t lilicorr_test_linear_timeout(const void* A, const void* W, flo
   g.wait_limit = wait_cycles;
   g.test_starve = 1;
   return gemm_tc_supported(g) ? launch_gemm_tc(g, stream) : LILICORR_ERR_SHAPE;
+}
+
+int lilicorr_test_attention_path(int mode) {
+  const int prev = g_attn_umma;
+  g_attn_umma = mode < 0 ? 0 : mode > 2 ? 2 : mode;
+  return prev;
 }
 
 int lilicorr_test_fused_path(const lilicorr_head* head, int mode) {

@@ -343,6 +343,13 @@ size_t attention_tc_smem_bytes(int LK, int hd, int L);
 lilicorr_status_t launch_attention_tc(const void* qkv, int B, int L, int K, int D, int n_heads,
                                       const float* dist, const float* same, void* out,
                                       cudaStream_t st);
+// the same core on tcgen05 (attention_umma.cu): 32- or 64-wide heads, up to 256 nodes per
+// sequence; g_attn_umma (api.cu) says where the chain uses it
+bool attention_umma_supported(int L, int K, int D, int n_heads);
+lilicorr_status_t launch_attention_umma(const void* qkv, int B, int L, int K, int D, int n_heads,
+                                        const float* dist, const float* same, void* out,
+                                        uint32_t* status, cudaStream_t st);
+extern int g_attn_umma;
 lilicorr_status_t launch_fusion_input(const float* x, int B, int LK, int D, const float* gain,
                                       const float* t, void* fin, lilicorr_dtype_t dt,
                                       cudaStream_t st);
