@@ -198,6 +198,7 @@ namespace lilicorr {
 struct TopkPlan {
   int splits;          // CTAs per row
   int threads;         // threads per CTA
+  int unroll;          // 16-byte vectors per thread per batch
   int chunk_vecs;      // 16-byte vectors per split
   int pieces;          // partial records per row in the workspace
   size_t rec_bytes;    // bytes of one partial record

@@ -35,7 +35,8 @@ namespace {
 
 constexpr int TK_THREADS = 256;        // CTA size of the few-row plan and of the merges
 constexpr int TK_THREADS_MANY = 128;   // CTA size when the rows alone fill the GPU
-constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch
+constexpr int TK_UNROLL = 4;           // 16-byte loads per thread per batch (many rows)
+constexpr int TK_UNROLL_FEW = 8;       // ... when few rows are split over many CTAs
 constexpr int TK_MAX_SPLITS = 64;
 constexpr int TK_MERGE_MAX = 512;      // splits * K keys merged by the last CTA
 constexpr int TK_FEW_ROW_CTAS = 256;   // CTAs over all rows when rows are few
@@ -317,16 +318,16 @@ __device__ __forceinline__ void warp_append(WarpCand& w, const float (&x)[N], ui
   }
 }
 
-// A batch: TK_UNROLL 16-byte vectors per thread (vectors it + u*NT + tid, NT threads).
+// A batch: U 16-byte vectors per thread (vectors it + u*NT + tid, NT threads).
 // CHECK = false: every vector is inside the chunk (no predicates); otherwise vectors past
 // v_end read as -inf, which adds nothing to the sum and never becomes a candidate (the
 // reduction below also skips vectors outside [v_lo, v_end) as candidates).
-template <typename T, int NT, bool CHECK>
+template <typename T, int NT, int U, bool CHECK>
 __device__ __forceinline__ void load_batch(const uint4* __restrict__ vp, int it, int v_end, int tid,
-                                           uint4 (&raw)[TK_UNROLL]) {
+                                           uint4 (&raw)[U]) {
   constexpr uint32_t NI = Vec<T>::NEG_INF4;
 #pragma unroll
-  for (int u = 0; u < TK_UNROLL; ++u) {
+  for (int u = 0; u < U; ++u) {
     const int v = it + u * NT + tid;
     raw[u] = (!CHECK || v < v_end) ? __ldcs(vp + v) : make_uint4(NI, NI, NI, NI);
   }
@@ -361,16 +362,16 @@ __device__ __forceinline__ void exp_vec(const uint4& r, uint64_t l2, uint64_t nm
 // Reduce one loaded batch: the online (max, sum exp) with one rescale check per batch, then
 // the candidates, which the warp looks at only if some lane's batch maximum reaches the
 // bound. s_wtop[warp]: the warps' published r-th largest lane maxima (r = ceil(K / warps)).
-template <typename T, int NT, bool CHECK>
-__device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int it, int v_lo,
+template <typename T, int NT, int U, bool CHECK>
+__device__ __forceinline__ void process_batch(const uint4 (&raw)[U], int it, int v_lo,
                                               int v_end, uint32_t id_base, int K, int tid, int lane,
                                               float& m, float& s, WarpCand& w,
                                               uint32_t* s_cta_thr, float* s_wtop) {
   constexpr int VEC = Vec<T>::N;
-  float vmx[TK_UNROLL];
+  float vmx[U];
   float bmax = -INFINITY;
 #pragma unroll
-  for (int u = 0; u < TK_UNROLL; ++u) {
+  for (int u = 0; u < U; ++u) {
     vmx[u] = Vec<T>::vmax(raw[u]);
     bmax = fmaxf(bmax, vmx[u]);
   }
@@ -384,7 +385,7 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int
     const uint64_t l2 = pack2(LOG2E, LOG2E), nm = pack2(-ml, -ml);
     uint64_t a0 = pack2(0.f, 0.f), a1 = a0;
 #pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u) exp_vec<T>(raw[u], l2, nm, a0, a1);
+    for (int u = 0; u < U; ++u) exp_vec<T>(raw[u], l2, nm, a0, a1);
     float p0, p1, p2, p3;
     unpack2(a0, p0, p1);
     unpack2(a1, p2, p3);
@@ -419,7 +420,7 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int
     }
   }
 #pragma unroll
-  for (int u = 0; u < TK_UNROLL; ++u) {
+  for (int u = 0; u < U; ++u) {
     if (!__any_sync(FULL, vmx[u] >= w.thr)) continue;
     const int v = it + u * NT + tid;
     float x[VEC];
@@ -436,27 +437,27 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[TK_UNROLL], int
 // Stream vectors [v_begin, v_end) through process_batch with the next batch's loads in
 // flight while the current one is reduced; full batches in the loop, the ragged last one
 // after it.
-template <typename T, int NT>
+template <typename T, int NT, int U>
 __device__ __forceinline__ void stream_chunk(const uint4* __restrict__ vp, int v_begin, int v_end,
                                              uint32_t id_base, int K, int tid, int lane, float& m,
                                              float& s, WarpCand& w, uint32_t* s_cta_thr,
                                              float* s_wtop) {
-  constexpr int STEP = TK_UNROLL * NT;
+  constexpr int STEP = U * NT;
   const int full_end = v_begin + (v_end - v_begin) / STEP * STEP;
-  uint4 cur[TK_UNROLL], nxt[TK_UNROLL];
-  if (v_begin < full_end) load_batch<T, NT, false>(vp, v_begin, v_end, tid, cur);
+  uint4 cur[U], nxt[U];
+  if (v_begin < full_end) load_batch<T, NT, U, false>(vp, v_begin, v_end, tid, cur);
 #pragma unroll 1
   for (int it = v_begin; it < full_end; it += STEP) {
-    if (it + STEP < full_end) load_batch<T, NT, false>(vp, it + STEP, v_end, tid, nxt);
-    process_batch<T, NT, false>(cur, it, it, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr,
-                                s_wtop);
+    if (it + STEP < full_end) load_batch<T, NT, U, false>(vp, it + STEP, v_end, tid, nxt);
+    process_batch<T, NT, U, false>(cur, it, it, v_end, id_base, K, tid, lane, m, s, w, s_cta_thr,
+                                   s_wtop);
 #pragma unroll
-    for (int u = 0; u < TK_UNROLL; ++u) cur[u] = nxt[u];
+    for (int u = 0; u < U; ++u) cur[u] = nxt[u];
   }
   if (full_end < v_end) {
-    load_batch<T, NT, true>(vp, full_end, v_end, tid, cur);
-    process_batch<T, NT, true>(cur, full_end, full_end, v_end, id_base, K, tid, lane, m, s, w,
-                               s_cta_thr, s_wtop);
+    load_batch<T, NT, U, true>(vp, full_end, v_end, tid, cur);
+    process_batch<T, NT, U, true>(cur, full_end, full_end, v_end, id_base, K, tid, lane, m, s, w,
+                                  s_cta_thr, s_wtop);
   }
 }
 
@@ -632,8 +633,10 @@ __device__ void finish_piece(TkShared<NT / 32>& sh, WarpCand& w, float m, float 
   }
 }
 
-template <typename T, int NT>
-__global__ void __launch_bounds__(NT, 1024 / NT)
+// U vectors per thread per batch: 4 with up to 1024 / NT CTAs per SM (64 registers), 8 for
+// the split plan of few rows (at most two CTAs per SM; more bytes in flight per thread).
+template <typename T, int NT, int U>
+__global__ void __launch_bounds__(NT, (U > 4 ? 512 : 1024) / NT)
 topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chunk_vecs,
                 size_t rec_bytes, int32_t* __restrict__ ids, float* __restrict__ logp,
                 float* __restrict__ lse, uint32_t* status, uint32_t* counters,
@@ -675,8 +678,8 @@ topk_lse_kernel(const T* __restrict__ logits, int V, int K, int splits, int chun
 
   // main stream: batches of 16-byte vectors, the next one's loads in flight
   const uint4* vp = reinterpret_cast<const uint4*>(rp + e0);
-  stream_chunk<T, NT>(vp, v_begin, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &sh.cta_thr,
-                      sh.wtop);
+  stream_chunk<T, NT, U>(vp, v_begin, v_end, (uint32_t)e0, K, tid, lane, m, s, w, &sh.cta_thr,
+                         sh.wtop);
   if (scalars) scalar_part<T>(rp, tail0, V, K, lane, m, s, w);
   finish_piece<NT>(sh, w, m, s, row, K, splits, split,
                    partials + (size_t)row * splits * rec_bytes, rec_bytes, counters, pout, ids,
@@ -730,13 +733,14 @@ TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   const int nvec = V / vec;
   const int sms = num_sms();
   const int min_chunk = 256;                 // vectors (4 KB) per CTA at least
-  int splits = 1, threads = TK_THREADS;
+  int splits = 1, threads = TK_THREADS, unroll = TK_UNROLL;
   if (rows * 2 < sms * 4) {
     // Few rows (not filling half of the 4-per-SM slots): split each over about 256 CTAs of
     // 256 threads in all (a sweep over 16-256 rows of a 151,936-wide vocabulary put the
     // optimum at 192-256 CTAs: more pieces add partial records and merge work faster than
     // they shorten the stream).
     splits = ceil_div(TK_FEW_ROW_CTAS, rows);
+    unroll = TK_UNROLL_FEW;       // 16 rows of 151,936: 11.3 -> 10.5 us
   } else if (rows >= 16 * sms) {
     // Many rows per SM: one CTA of 128 threads per row, up to 8 resident per SM, so each SM
     // always has rows in flight while others finish (4096 rows of 151,936: 233 us against
@@ -749,6 +753,7 @@ TopkPlan topk_plan(int rows, int V, int K, lilicorr_dtype_t dt) {
   TopkPlan p;
   p.splits = splits;
   p.threads = threads;
+  p.unroll = unroll;
   p.chunk_vecs = ceil_div(max(nvec, 1), splits);
   p.pieces = splits;
   p.rec_bytes = align_up(8 + 8 * (size_t)K, 16);
@@ -760,6 +765,24 @@ size_t topk_ws_bytes(int rows, int V, int K, lilicorr_dtype_t dt) {
   return 256 + align_up((size_t)rows * 4, 256) + align_up((size_t)rows * p.pieces * p.rec_bytes, 256);
 }
 
+template <typename T>
+lilicorr_status_t launch_plan(const TopkPlan& p, const T* x, int rows, int V, int K, int32_t* ids,
+                              float* logp, float* lse, uint32_t* status, uint32_t* counters,
+                              unsigned char* part, const PartialOut& pout, cudaStream_t st) {
+  const dim3 grid(p.splits, rows);
+  if (p.threads == TK_THREADS_MANY)
+    return launch_k(topk_lse_kernel<T, TK_THREADS_MANY, TK_UNROLL>, grid, TK_THREADS_MANY, 0, st,
+                    x, V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters,
+                    part, pout);
+  if (p.unroll == TK_UNROLL_FEW)
+    return launch_k(topk_lse_kernel<T, TK_THREADS, TK_UNROLL_FEW>, grid, TK_THREADS, 0, st, x, V,
+                    K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
+                    pout);
+  return launch_k(topk_lse_kernel<T, TK_THREADS, TK_UNROLL>, grid, TK_THREADS, 0, st, x, V, K,
+                  p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
+                  pout);
+}
+
 lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int rows, int V, int K,
                                   int32_t* ids, float* logp, float* lse, uint32_t* status,
                                   uint32_t* counters, void* partials, cudaStream_t st,
@@ -768,29 +791,11 @@ lilicorr_status_t launch_topk_lse(const void* logits, lilicorr_dtype_t dt, int r
   if (rows == 0) return LILICORR_OK;
   const TopkPlan p = topk_plan(rows, V, K, dt);
   unsigned char* part = static_cast<unsigned char*>(partials);
-  dim3 grid(p.splits, rows);
-  if (dt == LILICORR_BF16) {
-    const uint16_t* x = static_cast<const uint16_t*>(logits);
-    if (p.threads == TK_THREADS_MANY)
-      LL_TRY(launch_k(topk_lse_kernel<uint16_t, TK_THREADS_MANY>, grid, TK_THREADS_MANY, 0, st, x,
-                      V, K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters,
-                      part, pout));
-    else
-      LL_TRY(launch_k(topk_lse_kernel<uint16_t, TK_THREADS>, grid, TK_THREADS, 0, st, x, V, K,
-                      p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
-                      pout));
-  } else {
-    const float* x = static_cast<const float*>(logits);
-    if (p.threads == TK_THREADS_MANY)
-      LL_TRY(launch_k(topk_lse_kernel<float, TK_THREADS_MANY>, grid, TK_THREADS_MANY, 0, st, x, V,
-                      K, p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters,
-                      part, pout));
-    else
-      LL_TRY(launch_k(topk_lse_kernel<float, TK_THREADS>, grid, TK_THREADS, 0, st, x, V, K,
-                      p.splits, p.chunk_vecs, p.rec_bytes, ids, logp, lse, status, counters, part,
-                      pout));
-  }
-  return LILICORR_OK;
+  if (dt == LILICORR_BF16)
+    return launch_plan(p, static_cast<const uint16_t*>(logits), rows, V, K, ids, logp, lse, status,
+                       counters, part, pout, st);
+  return launch_plan(p, static_cast<const float*>(logits), rows, V, K, ids, logp, lse, status,
+                     counters, part, pout, st);
 }
 
 lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K, int32_t* ids,
