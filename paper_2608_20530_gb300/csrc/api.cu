@@ -276,7 +276,17 @@ struct HeadCall {
     g.c2 = xn; g.ldc2 = D; g.c2_gain = gain; g.ss_out = ss;
   }
   void norm_in(GemmArgs& g) const {
-    g.ss_in = ss; g.ss_slots = gemm_tc_ss_slots(N, D);
+    g.ss_in = ss; g.ss_slots = gemm_tc_ss_slots(N, D); g.ss_dim = D;
+  }
+  // the final norm into the fusion layer's input [x; x*t] (App. A), both blocks at once:
+  // xn [N, 2D] receives bf16(state * gain) and bf16(state * gain * t of the sequence)
+  void final_norm_out(GemmArgs& g, const float* gain) const {
+    norm_out(g, gain);
+    g.C = nullptr;               // nothing reads the last state itself
+    g.ldc2 = 2 * D;
+    g.c3 = static_cast<__nv_bfloat16*>(xn) + D;
+    g.c3_t = t;
+    g.c3_rows_per = LK;
   }
 };
 
@@ -347,16 +357,20 @@ bool fold_norms(const HeadCall& c) {
   const int D = c.D, F = c.F, N = c.N;
   const lilicorr_dtype_t adt = c.adt, F32 = LILICORR_F32;
   if (c.wdt != LILICORR_BF16) return false;
-  GemmArgs p[5] = {c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D),
+  GemmArgs p[7] = {c.G(c.c1, adt, D, h->conf2_w, D, c.x, F32, D, N, D, D),
                    c.G(c.xn, adt, D, h->layer[0].wqkv, D, c.qkv, c.qkv_dt, 3 * D, N, 3 * D, D),
                    c.G(c.att, adt, D, h->layer[0].wo, D, c.x, F32, D, N, D, D),
                    c.G(c.xn, adt, D, h->layer[0].w1, D, c.hf, adt, F, N, F, D),
-                   c.G(c.hf, adt, F, h->layer[0].w2, F, c.x, F32, D, N, D, F)};
-  for (int i : {0, 2, 4}) {
+                   c.G(c.hf, adt, F, h->layer[0].w2, F, c.x, F32, D, N, D, F),
+                   c.G(c.hf, adt, F, h->layer[0].w2, F, c.x, F32, D, N, D, F),
+                   c.G(c.xn, adt, 2 * D, h->fuse_x, 2 * D, c.u, adt, D, N, D, 2 * D)};
+  for (int i : {0, 2, 4, 5}) {
     p[i].residual = c.x; p[i].ldr = D;
     c.norm_out(p[i], h->layer[0].an);
   }
-  for (int i : {1, 3}) c.norm_in(p[i]);
+  c.final_norm_out(p[5], h->final_norm);
+  p[6].bias_rows = c.cb; p[6].rows_per_bias = c.LK; p[6].act = ACT_SILU;
+  for (int i : {1, 3, 6}) c.norm_in(p[i]);
   for (const GemmArgs& g : p)
     if (!takes_gemm_tc(g)) return false;
   return true;
@@ -430,16 +444,21 @@ lilicorr_status_t run_body(const HeadCall& c, const int32_t* ids, const float* l
     g = c.G(c.hf, adt, F, l.w2, F, c.x, F32, D, N, D, F);
     g.bias = l.b2;
     g.residual = c.x; g.ldr = D;
-    // the last layer's output goes to the final norm inside the fusion input instead
-    if (fold && i + 1 < d.n_layers) c.norm_out(g, h->layer[i + 1].an);
+    // the last layer's output feeds the final norm: both blocks of the fusion input
+    if (fold) {
+      if (i + 1 < d.n_layers) c.norm_out(g, h->layer[i + 1].an);
+      else c.final_norm_out(g, h->final_norm);
+    }
     LL_TRY(run_gemm(g, st));
   }
-  // fusion u = SiLU(W_f [x; t; x*t] + b_f) with x the final-normed state
-  LL_TRY(launch_fusion_input(c.x, c.B, c.LK, D, h->final_norm, c.t, c.xn, adt, st));
+  // fusion u = SiLU(W_f [x; t; x*t] + b_f) with x the final-normed state (the t block is
+  // the per-sequence bias cb)
+  if (!fold) LL_TRY(launch_fusion_input(c.x, c.B, c.LK, D, h->final_norm, c.t, c.xn, adt, st));
   g = c.G(c.xn, adt, 2 * D, h->fuse_x, 2 * D, c.u, adt, D, N, D, 2 * D);
   g.bias_rows = c.cb;
   g.rows_per_bias = c.LK;
   g.act = ACT_SILU;
+  if (fold) c.norm_in(g);
   LL_TRY(run_gemm(g, st));
   // out and in heads in one product: oi = [W_o u + b_o | W_i u + b_i]
   g = c.G(c.u, adt, D, h->woi, D, c.oi, F32, 2 * d.d, N, 2 * d.d, D);

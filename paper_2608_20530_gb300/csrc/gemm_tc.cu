@@ -59,6 +59,10 @@ struct TcEpilogue {
   // times `c2_gain` per column, rounded to bf16, into c2 [M, ldc2], and each thread's sum of
   // squares of its part of the row into ss_out[m * SS_LD + 2 * column tile + half]
   __nv_bfloat16* c2; int ldc2; const float* c2_gain; float* ss_out;
+  // ...and optionally a second copy times a per-sequence row vector: c3 [M, ldc2] receives
+  // bf16(output * c2_gain * c3_t[m / c3_rows_per]) (c3_t [*, N])
+  __nv_bfloat16* c3; const float* c3_t; int c3_rows_per;
+  int no_c;              // folded producer whose output C nobody reads: only c2 / c3 written
   // ...and its use: the accumulator scaled by rsqrt(sum of ss_in[m * SS_LD + 0..ss_slots) *
   // ss_scale + eps) before the bias
   const float* ss_in; int ss_slots; float ss_scale;
@@ -73,7 +77,7 @@ struct TcCfg {
   static constexpr int NCH = BN / CH;
   static constexpr uint32_t TMEM_COLS = 2 * BN;         // two accumulators
   static constexpr size_t RING = (size_t)STAGES * (A_BYTES + B_BYTES);
-  static constexpr size_t SMEM = 1024 + RING + 4 * (size_t)CHUNK_BYTES + 2 * BN * sizeof(float);
+  static constexpr size_t SMEM = 1024 + RING + 4 * (size_t)CHUNK_BYTES + 3 * BN * sizeof(float);
 };
 
 // FOLD: the instantiation with the folded-RMSNorm epilogue (c2 / ss_out, ss_in); the
@@ -96,6 +100,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   uint8_t* s_res = s_out + 2 * CHUNK_BYTES;            // 2 residual chunks
   float* s_bias = reinterpret_cast<float*>(s_res + 2 * CHUNK_BYTES);
   float* s_gain = s_bias + BN;                         // c2_gain of the tile's columns
+  float* s_t = s_gain + BN;                            // c3_t of the tile's sequence
   __shared__ __align__(8) uint64_t full[S], empty[S], acc_full[2], acc_empty[2], res_full[2];
   __shared__ uint32_t tmem_base;
   __shared__ volatile int abort_flag;
@@ -214,9 +219,14 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       const int m0 = (t / tiles_n) * TC_BM, n0 = (t % tiles_n) * BN;
       const uint32_t acc = lt & 1u;
       epi_bar();                                  // s_bias free again
+      // c3: when the tile's rows all belong to one sequence, its c3_t row goes to shared
+      // memory with the gains; otherwise every thread reads its own row's
+      const int tb0 = (FOLD && ep.c3) ? min(m0, M - 1) / ep.c3_rows_per : 0;
+      const bool t_shared = (FOLD && ep.c3) && min(m0 + TC_BM - 1, M - 1) / ep.c3_rows_per == tb0;
       for (int j = threadIdx.x - 64; j < BN; j += EPI_THREADS) {
         s_bias[j] = (ep.bias && n0 + j < N) ? ep.bias[n0 + j] : 0.f;
         if (FOLD && !OUT_BF16 && ep.c2) s_gain[j] = n0 + j < N ? ep.c2_gain[n0 + j] : 0.f;
+        if (t_shared) s_t[j] = n0 + j < N ? ep.c3_t[(size_t)tb0 * N + n0 + j] : 0.f;
       }
       if (!abort_flag && !mbar_wait(&acc_full[acc], (lt >> 1) & 1u, wait_limit))
         abort_flag = 1;
@@ -293,29 +303,47 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
         if constexpr (FOLD && !OUT_BF16) {
           if (ep.c2) {                      // the next RMSNorm's input, and its sums
+            // the warp holds 32 rows x 32 bytes: lanes 2i and 2i+1 store the two halves
+            // of row i (then of row 16 + i), one whole 32-byte sector per pair
+            static_assert(HC == 16, "fp32 chunk halves of 16 columns");
+            auto store_rows = [&](const uint32_t (&wv)[HC / 2], __nv_bfloat16* dst) {
+#pragma unroll
+              for (int rd = 0; rd < 2; ++rd) {
+                const int src = 16 * rd + (lane >> 1), piece = lane & 1;
+                uint32_t o[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const uint32_t a0 = __shfl_sync(0xffffffffu, wv[k], src);
+                  const uint32_t a1 = __shfl_sync(0xffffffffu, wv[4 + k], src);
+                  o[k] = piece ? a1 : a0;
+                }
+                const int mr = m0 + q * 32 + src;
+                if (mr < M && n0 + cl < N)
+                  *reinterpret_cast<uint4*>(dst + (size_t)mr * ep.ldc2 + n0 + cl + 8 * piece) =
+                      make_uint4(o[0], o[1], o[2], o[3]);
+              }
+            };
+            float g[HC];
+#pragma unroll
+            for (int j = 0; j < HC; ++j) g[j] = v[j] * s_gain[cl + j];
             uint32_t wv[HC / 2];
 #pragma unroll
             for (int j = 0; j < HC; j += 2) {
               ssq = fmaf(v[j], v[j], fmaf(v[j + 1], v[j + 1], ssq));
-              wv[j / 2] = pack_bf16x2(v[j] * s_gain[cl + j], v[j + 1] * s_gain[cl + j + 1]);
+              wv[j / 2] = pack_bf16x2(g[j], g[j + 1]);
             }
-            // the warp holds 32 rows x 32 bytes: lanes 2i and 2i+1 store the two halves
-            // of row i (then of row 16 + i), one whole 32-byte sector per pair
-            static_assert(HC == 16, "fp32 chunk halves of 16 columns");
+            store_rows(wv, ep.c2);
+            if (ep.c3) {
+              const float4* tr = reinterpret_cast<const float4*>(
+                  t_shared ? s_t + cl
+                           : ep.c3_t + (size_t)(m < M ? m / ep.c3_rows_per : 0) * N + n0 + cl);
 #pragma unroll
-            for (int rd = 0; rd < 2; ++rd) {
-              const int src = 16 * rd + (lane >> 1), piece = lane & 1;
-              uint32_t o[4];
-#pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                const uint32_t a0 = __shfl_sync(0xffffffffu, wv[k], src);
-                const uint32_t a1 = __shfl_sync(0xffffffffu, wv[4 + k], src);
-                o[k] = piece ? a1 : a0;
+              for (int j = 0; j < HC; j += 4) {
+                const float4 tv = tr[j / 4];
+                wv[j / 2] = pack_bf16x2(g[j] * tv.x, g[j + 1] * tv.y);
+                wv[j / 2 + 1] = pack_bf16x2(g[j + 2] * tv.z, g[j + 3] * tv.w);
               }
-              const int mr = m0 + q * 32 + src;
-              if (mr < M && n0 + cl < N)
-                *reinterpret_cast<uint4*>(ep.c2 + (size_t)mr * ep.ldc2 + n0 + cl + 8 * piece) =
-                    make_uint4(o[0], o[1], o[2], o[3]);
+              store_rows(wv, ep.c3);
             }
           }
         }
@@ -339,7 +367,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
         fence_async_shared();
         epi_bar();
-        if (leader && !abort_flag && n0 + c * CH < N) {
+        if (leader && !abort_flag && n0 + c * CH < N && !(FOLD && ep.no_c)) {
           tma_store_2d(&mapC, stg, n0 + c * CH, m0);
           tma_store_wait_read_le1();         // the other buffer is free for the next chunk
         }
@@ -381,13 +409,16 @@ lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   const CUtensorMapDataType f32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
   if (!make_map(&ma, g.A, bf, 2, g.M, g.Kd, g.lda, TC_BM, TC_BK)) return LILICORR_ERR_CUDA;
   if (!make_map(&mw, g.W, bf, 2, g.N, g.Kd, g.ldw, BN, TC_BK)) return LILICORR_ERR_CUDA;
-  if (!make_map(&mc, g.C, OUT_BF16 ? bf : f32, OUT_BF16 ? 2 : 4, g.M, g.N, g.ldc, TC_BM, Cfg::CH))
-    return LILICORR_ERR_CUDA;
   if (g.residual) {
     if (!make_map(&mr, g.residual, f32, 4, g.M, g.N, g.ldr, TC_BM, 32)) return LILICORR_ERR_CUDA;
-  } else {
-    mr = mc;                                   // never read
   }
+  if (g.C) {
+    if (!make_map(&mc, g.C, OUT_BF16 ? bf : f32, OUT_BF16 ? 2 : 4, g.M, g.N, g.ldc, TC_BM, Cfg::CH))
+      return LILICORR_ERR_CUDA;
+  } else {
+    mc = g.residual ? mr : ma;                 // never written (no_c)
+  }
+  if (!g.residual) mr = mc;                    // never read
   TcEpilogue ep;
   ep.bias = g.bias;
   ep.bias_rows = g.bias_rows;
@@ -400,7 +431,11 @@ lilicorr_status_t launch_bn(const GemmArgs& g, cudaStream_t st) {
   ep.ss_out = g.ss_out;
   ep.ss_in = g.ss_in;
   ep.ss_slots = g.ss_slots;
-  ep.ss_scale = 1.0f / (float)g.Kd;
+  ep.c3 = static_cast<__nv_bfloat16*>(g.c3);
+  ep.c3_t = g.c3_t;
+  ep.c3_rows_per = g.c3_rows_per;
+  ep.no_c = g.C == nullptr;
+  ep.ss_scale = 1.0f / (float)(g.ss_dim > 0 ? g.ss_dim : g.Kd);
   const int tiles = ceil_div(g.M, TC_BM) * ceil_div(g.N, BN);
   const int grid = tiles < num_sms() ? tiles : num_sms();
   const long long wait = g.wait_limit > 0 ? g.wait_limit : WAIT_LIMIT_CYCLES;
@@ -483,9 +518,13 @@ bool gemm_tc_supported(const GemmArgs& g) {
   if (g.c2 && (g.c_dt != LILICORR_F32 || !g.c2_gain || !g.ss_out || (g.N % 32) ||
                !aligned16(g.c2) || (g.ldc2 % 8) || gemm_tc_ss_slots(g.M, g.N) > SS_LD))
     return false;
+  if (g.c3 && (!g.c2 || !g.c3_t || g.c3_rows_per < 1 || !aligned16(g.c3) || !aligned16(g.c3_t)))
+    return false;
   if (g.ss_in && (g.ss_slots < 1 || g.ss_slots > SS_LD)) return false;
   if (g.M <= 0 || g.N <= 0 || g.Kd <= 0) return false;
   // TMA: 16-byte aligned bases and row strides, outputs in 16-byte column groups
+  // C may be absent only for a folded producer (its bf16 copies are the output)
+  if (!g.C && !(g.c2 && g.c_dt == LILICORR_F32)) return false;
   if (!aligned16(g.A) || !aligned16(g.W) || !aligned16(g.C)) return false;
   if ((g.lda % 8) || (g.ldw % 8) || (g.Kd % 8) || (g.N % 8) || (g.ldc % 8)) return false;
   if (g.residual && (g.c_dt != LILICORR_F32 || !aligned16(g.residual) || (g.ldr % 4)))

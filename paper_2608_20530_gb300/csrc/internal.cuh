@@ -276,6 +276,10 @@ struct GemmArgs {
   // scaled per row by rsqrt(sum of ss_in's first ss_slots slots / Kd + eps) before the bias.
   void* c2; int ldc2; const float* c2_gain; float* ss_out;
   const float* ss_in; int ss_slots;
+  int ss_dim;              // the norm's row length (0: Kd)
+  // producer, also: c3 [M, ldc2] (bf16) receives C times c2_gain times c3_t's row
+  // m / c3_rows_per (c3_t [*, N], fp32), e.g. the x*t block of the fusion input
+  void* c3; const float* c3_t; int c3_rows_per;
 };
 constexpr int SS_LD = 16;  // floats per row of a folded-RMSNorm sums-of-squares buffer
 int gemm_tc_ss_slots(int M, int N);
