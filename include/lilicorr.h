@@ -213,7 +213,9 @@ lilicorr_status_t lilicorr_lm_head_topk(const void* hidden, const void* w_vocab,
  *     that overlap on the GPU (different streams, or different host threads) race
  *     and give undefined results; order them on one stream.
  *   - A non-finite row is detected as in lilicorr_topk_lse, but the status word lives
- *     in the fixed array and is not reported; that row's outputs are undefined. */
+ *     in the fixed array and is not reported. Such a row's lse comes out non-finite
+ *     (NaN for a row holding NaN or +inf, -inf for a row of only -inf), which the
+ *     caller can test; its ids and logp are undefined. */
 size_t lilicorr_topk_lse_noalloc_max_bytes(void);
 lilicorr_status_t lilicorr_topk_lse_noalloc(const void* logits, lilicorr_dtype_t dtype, int rows,
                                             int V, int K, int32_t* ids, float* logp, float* lse,

@@ -68,12 +68,13 @@ __host__ __device__ constexpr size_t ua_region_a(int LKp) {
 }
 __host__ __device__ constexpr size_t ua_smem(int LKp, int HD, int L) {
   return 1024 + ua_region_a(LKp) + (size_t)LKp * 128 +
-         ((sizeof(float) * (2 * L - 1) + LKp + 15) / 16) * 16 + 16;
+         ((sizeof(float) * (2 * L - 1) + LKp + 15) / 16) * 16 + 32;
 }
 
 template <int HD>
 __global__ void __launch_bounds__(UA_THREADS, 2)
-attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D, int n_heads,
+attention_umma_kernel(const __grid_constant__ CUtensorMap map_qkv, int use_tma,
+                      const __nv_bfloat16* __restrict__ qkv, int L, int K, int D, int n_heads,
                       const float* __restrict__ dist, const float* __restrict__ same,
                       __nv_bfloat16* __restrict__ out, uint32_t* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -92,6 +93,8 @@ attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D
       (reinterpret_cast<uintptr_t>(s_slot + LKp) + 7) & ~static_cast<uintptr_t>(7));
   uint64_t* bar_s = bars;
   uint64_t* bar_o = bars + 1;
+  uint64_t* bar_qk = bars + 2;                        // TMA staging: Q and K, then V
+  uint64_t* bar_v = bars + 3;
 
   const int tid = threadIdx.x, warp = tid >> 5;
   // the query tiles of one (sequence, head) are neighbours in the grid, so the second
@@ -105,34 +108,52 @@ attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D
   if (tid == 0) {
     mbar_init(bar_s, 1);
     mbar_init(bar_o, 1);
+    mbar_init(bar_qk, 1);
+    mbar_init(bar_v, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   pdl_wait();
 
-  // ---- staging: Q, K and V rows by asynchronous copies (zeros past the head width and
-  // past the nodes) in two groups, Q and K first (S needs them), V second (it lands while
-  // the probabilities are formed); the biases and the key slots
-  const uint4 zero = make_uint4(0, 0, 0, 0);
-  for (int i = tid; i < 128 * 8; i += UA_THREADS) {
-    const int r = i >> 3, p = i & 7;
-    uint8_t* dst = sQ + swz(r, p);
-    if (p < HD / 8 && q0 + r < LK) cp16(dst, base + (size_t)(q0 + r) * ld + 8 * p);
-    else *reinterpret_cast<uint4*>(dst) = zero;
+  if (use_tma) {
+    // 64-wide heads of 256-node sequences (no padding anywhere): Q, K and V as five
+    // 128-row TMA boxes of the q|k|v buffer, issued by one thread, in the same swizzled
+    // rows as the copies below
+    if (tid == 0) {
+      const int row0 = b * LK, col = h * HD;
+      mbar_expect_tx(bar_qk, 3 * UA_CHUNK);
+      tma_load_2d(sQ, &map_qkv, bar_qk, col, row0 + q0);
+      tma_load_2d(sK, &map_qkv, bar_qk, D + col, row0);
+      tma_load_2d(sK + UA_CHUNK, &map_qkv, bar_qk, D + col, row0 + 128);
+      mbar_expect_tx(bar_v, 2 * UA_CHUNK);
+      tma_load_2d(sV, &map_qkv, bar_v, 2 * D + col, row0);
+      tma_load_2d(sV + UA_CHUNK, &map_qkv, bar_v, 2 * D + col, row0 + 128);
+    }
+  } else {
+    // ---- staging: Q, K and V rows by asynchronous copies (zeros past the head width and
+    // past the nodes) in two groups, Q and K first (S needs them), V second (it lands while
+    // the probabilities are formed); the biases and the key slots
+    const uint4 zero = make_uint4(0, 0, 0, 0);
+    for (int i = tid; i < 128 * 8; i += UA_THREADS) {
+      const int r = i >> 3, p = i & 7;
+      uint8_t* dst = sQ + swz(r, p);
+      if (p < HD / 8 && q0 + r < LK) cp16(dst, base + (size_t)(q0 + r) * ld + 8 * p);
+      else *reinterpret_cast<uint4*>(dst) = zero;
+    }
+    for (int i = tid; i < LKp * 8; i += UA_THREADS) {
+      const int j = i >> 3, p = i & 7;
+      uint8_t* dk = sK + swz(j, p);
+      if (p < HD / 8 && j < LK) cp16(dk, base + (size_t)j * ld + D + 8 * p);
+      else *reinterpret_cast<uint4*>(dk) = zero;
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    for (int i = tid; i < LKp * 8; i += UA_THREADS) {
+      const int j = i >> 3, p = i & 7;
+      uint8_t* dv = sV + swz(j, p);
+      if (p < HD / 8 && j < LK) cp16(dv, base + (size_t)j * ld + 2 * D + 8 * p);
+      else *reinterpret_cast<uint4*>(dv) = zero;
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
   }
-  for (int i = tid; i < LKp * 8; i += UA_THREADS) {
-    const int j = i >> 3, p = i & 7;
-    uint8_t* dk = sK + swz(j, p);
-    if (p < HD / 8 && j < LK) cp16(dk, base + (size_t)j * ld + D + 8 * p);
-    else *reinterpret_cast<uint4*>(dk) = zero;
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
-  for (int i = tid; i < LKp * 8; i += UA_THREADS) {
-    const int j = i >> 3, p = i & 7;
-    uint8_t* dv = sV + swz(j, p);
-    if (p < HD / 8 && j < LK) cp16(dv, base + (size_t)j * ld + 2 * D + 8 * p);
-    else *reinterpret_cast<uint4*>(dv) = zero;
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
   for (int i = tid; i < 2 * L - 1; i += UA_THREADS) s_dist[i] = dist[(size_t)h * (2 * L - 1) + i] * UA_LOG2E;
   for (int i = tid; i < LKp; i += UA_THREADS) s_slot[i] = (uint8_t)min(i / K, L - 1);
   asm volatile("cp.async.wait_group 1;" ::: "memory");       // Q and K
@@ -145,6 +166,7 @@ attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D
 
   // ---- S = Q K^T
   if (tid == 0) {
+    if (use_tma && !mbar_wait(bar_qk, 0, UA_WAIT)) ok = false;
     const uint64_t qd = smem_desc(sQ), kd = smem_desc(sK);
 #pragma unroll
     for (int k = 0; k < 4; ++k) mma_bf16(tmem, qd + 2ull * k, kd + 2ull * k, instr_desc(128, LKp), k > 0);
@@ -294,6 +316,7 @@ attention_umma_kernel(const __nv_bfloat16* __restrict__ qkv, int L, int K, int D
   // ---- O = P V over S's first 64 columns; V is the MN-major B operand (instruction
   // descriptor bit 16), each K step of 16 keys starting 16 rows (2048 bytes) further on
   if (tid == 0) {
+    if (use_tma && !mbar_wait(bar_v, 0, UA_WAIT)) ok = false;
     constexpr uint32_t idesc_pv = instr_desc(128, 64) | (1u << 16);
     for (int kc = 0; kc < nkc; ++kc) {
       const uint64_t pd = smem_desc(sP + (size_t)kc * UA_CHUNK);
@@ -341,8 +364,15 @@ lilicorr_status_t launch_umma_hd(const __nv_bfloat16* qkv, int B, int L, int K, 
   LL_TRY(allow_max_dynamic_smem(attention_umma_kernel<HD>, configured));
   const int LK = L * K, LKp = (LK + 63) / 64 * 64;
   dim3 grid(ceil_div(LK, 128), B * n_heads);
-  LL_TRY(launch_k(attention_umma_kernel<HD>, grid, UA_THREADS, ua_smem(LKp, HD, L), st, qkv, L,
-                  K, D, n_heads, dist, same, out, status));
+  // TMA staging where no row or column is padded: 64-wide heads, 256-node sequences
+  CUtensorMap map;
+  memset(&map, 0, sizeof(map));
+  const int use_tma = HD == 64 && LK == UA_MAX_KEYS;
+  if (use_tma && !make_map(&map, qkv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, B * LK, 3 * D, 3 * D,
+                           128, 64))
+    return LILICORR_ERR_CUDA;
+  LL_TRY(launch_k(attention_umma_kernel<HD>, grid, UA_THREADS, ua_smem(LKp, HD, L), st, map,
+                  use_tma, qkv, L, K, D, n_heads, dist, same, out, status));
   return LILICORR_OK;
 }
 

@@ -60,3 +60,31 @@ def test_noalloc_rejects_sizes_beyond_its_scratch():
                                        f.data_ptr(), f.data_ptr(),
                                        torch.cuda.current_stream().cuda_stream)
     assert st == 7
+
+
+@pytest.mark.parametrize("bad", ["nan", "plus_inf", "all_minus_inf"])
+def test_noalloc_nonfinite_row_has_nonfinite_lse(bad):
+    """The status word of this entry point is not reported; a non-finite row shows as a
+    non-finite lse instead (the other rows are unaffected)."""
+    ll = _ll()
+    x = np.random.default_rng(3).standard_normal((6, 4000)).astype(np.float32)
+    if bad == "nan":
+        x[2, 17] = np.nan
+    elif bad == "plus_inf":
+        x[2, 17] = np.inf
+    else:
+        x[2] = -np.inf
+    t = torch.from_numpy(x).cuda()
+    ids, logp, lse = ll.topk_lse_noalloc(t, 4)
+    ids_ref, logp_ref, lse_ref = ll.topk_lse(t, 4)
+    torch.cuda.synchronize()
+    lse, lse_ref = lse.cpu().numpy(), lse_ref.cpu().numpy()
+    assert not np.isfinite(lse[2])
+    if bad == "all_minus_inf":
+        assert lse[2] == -np.inf
+    else:
+        assert np.isnan(lse[2])
+    ok = [0, 1, 3, 4, 5]
+    assert np.isfinite(lse[ok]).all()
+    assert np.abs(lse[ok] - lse_ref[ok]).max() <= TOL
+    assert torch.equal(ids[ok], ids_ref[ok])
