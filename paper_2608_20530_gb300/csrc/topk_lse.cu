@@ -209,6 +209,20 @@ __device__ __forceinline__ float warp_kth_largest(float v, int K, int lane) {
   return __shfl_sync(FULL, v, K - 1);
 }
 
+// r-th largest (1 <= r <= 32) of one value per lane, in the order of ord32 (-0 below +0):
+// rounds of a warp-wide maximum over the lanes not yet taken, equal values counted at once
+// (at most r rounds; every float's image is above 0, which marks a lane as taken). Cheaper
+// than the sorting network for small r (4096 rows of 151,936 at K = 16: 237.6 -> 224.0 us).
+__device__ __forceinline__ float warp_rth_largest(float v, int r) {
+  uint32_t in = ord32(v);
+  for (;;) {
+    const uint32_t mx = __reduce_max_sync(FULL, in);
+    r -= __popc(__ballot_sync(FULL, in == mx));
+    if (r <= 0) return unord32(mx);
+    if (in == mx) in = 0u;
+  }
+}
+
 // A warp's candidates: keys appended to a shared-memory buffer, plus a value bound
 // below which no element can be in the CTA's top-K. The bound is the larger of
 //   * the K-th largest running maximum over the warp's lanes (each lane's running maximum
@@ -398,7 +412,7 @@ __device__ __forceinline__ void process_batch(const uint4 (&raw)[U], int it, int
     // the CTA-wide bound from the warps' published lane maxima
     constexpr int NW = NT / 32;
     const int r = (K + NW - 1) / NW;
-    const float mine = r == 1 ? warp_max(m) : warp_kth_largest(m, r, lane);
+    const float mine = warp_rth_largest(m, r);
     volatile float* wtop = s_wtop;
     if (lane == 0) wtop[tid >> 5] = mine;             // lane maxima only grow
     __syncwarp();
