@@ -25,7 +25,9 @@ extern "C" {
  * 1 = tiled CUDA-core kernel, 2 = few-row (split-N) CUDA-core kernel,
  * 3 = tensor cores (bf16 A and W only; LILICORR_ERR_DTYPE otherwise),
  * 4 = tensor cores for one tile of rows (M <= 128, Kd <= 512 a multiple of 64, N a
- *     multiple of 32 (fp32 out) or 64 (bf16 out); LILICORR_ERR_SHAPE otherwise).
+ *     multiple of 32 (fp32 out) or 64 (bf16 out); LILICORR_ERR_SHAPE otherwise),
+ * 5 = row-block CUDA-core kernel for fp32 A (Kd a multiple of 8, lda of 4, ldw of 8, A and
+ *     W 16-byte aligned; LILICORR_ERR_SHAPE otherwise).
  * status: a device uint32 word that receives bounded-wait timeouts (may be NULL). */
 lilicorr_status_t lilicorr_test_linear(const void* A, lilicorr_dtype_t a_dt, int lda, const void* W,
                                        lilicorr_dtype_t w_dt, int ldw, void* C,

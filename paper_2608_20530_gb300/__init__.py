@@ -483,7 +483,8 @@ def select_block(head: Head, logits: torch.Tensor, hidden: torch.Tensor, target:
 def test_linear(A: torch.Tensor, W: torch.Tensor, out_dtype=torch.float32, bias=None,
                 residual=None, act: int = 0, path: int = 0, status: Optional[torch.Tensor] = None):
     """Test hook: one linear layer C = act(A W^T + bias) + residual through kernel `path`
-    (0 auto, 1 tiled CUDA cores, 2 few-row CUDA cores, 3 tensor cores)."""
+    (0 auto, 1 tiled CUDA cores, 2 few-row CUDA cores, 3 tensor cores, 4 tensor cores for one
+    tile of rows, 5 row-block CUDA cores for fp32 A)."""
     M, Kd = A.shape
     N = W.shape[0]
     C = torch.empty((M, N), dtype=out_dtype, device=A.device)

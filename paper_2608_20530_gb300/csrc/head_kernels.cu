@@ -177,6 +177,64 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
   }
 }
 
+// ----------------------------------------------------------------------------- row-block linear
+// Per-sequence products with fp32 activations and more rows than the few-row kernel takes
+// (the target state t of a batch against W_a and the fusion layer's t block: M = B up to
+// 1024, Kd = D). CTA = 16 rows x 32 columns: lane = output column (it streams its weight
+// row in 16-byte pieces), warp = two rows; the 16 rows' activations are staged in shared
+// memory, GR_KC columns at a time, and read as broadcasts. No cross-lane reduction.
+constexpr int GR_M = 16, GR_N = 32, GR_THREADS = 256, GR_KC = 512;
+template <typename TW, typename TC>
+__global__ void __launch_bounds__(GR_THREADS) gemm_rows_kernel(GemmArgs g) {
+  pdl_wait();
+  __shared__ __align__(16) float As[GR_M][GR_KC + 4];
+  const float* A = static_cast<const float*>(g.A);
+  const TW* W = static_cast<const TW*>(g.W);
+  const int m0 = blockIdx.y * GR_M, n0 = blockIdx.x * GR_N;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int n = n0 + lane, r0 = 2 * warp;
+  float acc0 = 0.f, acc1 = 0.f;
+  for (int k0 = 0; k0 < g.Kd; k0 += GR_KC) {
+    const int kc4 = min(GR_KC, g.Kd - k0) >> 2;          // 16-byte pieces per row
+    __syncthreads();                                     // the previous chunk is consumed
+    for (int i = threadIdx.x; i < GR_M * kc4; i += GR_THREADS) {
+      const int r = i / kc4, c = 4 * (i % kc4);
+      *reinterpret_cast<float4*>(&As[r][c]) =
+          m0 + r < g.M ? *reinterpret_cast<const float4*>(A + (size_t)(m0 + r) * g.lda + k0 + c)
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    __syncthreads();
+    if (n < g.N) {
+      const TW* wr = W + (size_t)n * g.ldw + k0;
+#pragma unroll 4
+      for (int k = 0; k < 4 * kc4; k += 8) {
+        float w[8];
+        load8(wr + k, w);
+        const float4 a0 = *reinterpret_cast<const float4*>(&As[r0][k]);
+        const float4 a1 = *reinterpret_cast<const float4*>(&As[r0][k + 4]);
+        const float4 b0 = *reinterpret_cast<const float4*>(&As[r0 + 1][k]);
+        const float4 b1 = *reinterpret_cast<const float4*>(&As[r0 + 1][k + 4]);
+        acc0 = fmaf(a0.x, w[0], fmaf(a0.y, w[1], fmaf(a0.z, w[2], fmaf(a0.w, w[3], acc0))));
+        acc0 = fmaf(a1.x, w[4], fmaf(a1.y, w[5], fmaf(a1.z, w[6], fmaf(a1.w, w[7], acc0))));
+        acc1 = fmaf(b0.x, w[0], fmaf(b0.y, w[1], fmaf(b0.z, w[2], fmaf(b0.w, w[3], acc1))));
+        acc1 = fmaf(b1.x, w[4], fmaf(b1.y, w[5], fmaf(b1.z, w[6], fmaf(b1.w, w[7], acc1))));
+      }
+    }
+  }
+  if (n >= g.N) return;
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int m = m0 + r0 + i;
+    if (m >= g.M) continue;
+    float v = i ? acc1 : acc0;
+    if (g.bias) v += g.bias[n];
+    if (g.bias_rows) v += g.bias_rows[(size_t)(m / g.rows_per_bias) * g.N + n];
+    if (g.act == ACT_SILU) v = silu_f(v);
+    if (g.residual) v += g.residual[(size_t)m * g.ldr + n];
+    st_elem(static_cast<TC*>(g.C), (size_t)m * g.ldc + n, v);
+  }
+}
+
 template <typename TA, typename TW, int MB>
 lilicorr_status_t skinny_dispatch_m(const GemmArgs& g, cudaStream_t st) {
   dim3 grid(ceil_div(g.N, SK_NB), ceil_div(g.M, MB));
@@ -483,6 +541,24 @@ __global__ void attention_kernel(const float* __restrict__ qkv, int L, int K, in
 size_t attention_smem_bytes(int LK, int hd, int warps) {
   return sizeof(float) * ((size_t)LK * (hd + 1) + (size_t)LK * hd + (size_t)warps * hd +
                           (size_t)warps * LK);
+}
+
+bool gemm_rows_supported(const GemmArgs& g) {
+  return g.a_dt == LILICORR_F32 && g.M > 0 && g.N > 0 && g.Kd % 8 == 0 && g.lda % 4 == 0 &&
+         g.ldw % 8 == 0 && (reinterpret_cast<uintptr_t>(g.A) & 15) == 0 &&
+         (reinterpret_cast<uintptr_t>(g.W) & 15) == 0;
+}
+
+lilicorr_status_t launch_gemm_rows(const GemmArgs& g, cudaStream_t st) {
+  if (!gemm_rows_supported(g)) return LILICORR_ERR_SHAPE;
+  const dim3 grid(ceil_div(g.N, GR_N), ceil_div(g.M, GR_M));
+  if (g.w_dt == LILICORR_F32) {
+    if (g.c_dt == LILICORR_F32) return launch_k(gemm_rows_kernel<float, float>, grid, GR_THREADS, 0, st, g);
+    return launch_k(gemm_rows_kernel<float, __nv_bfloat16>, grid, GR_THREADS, 0, st, g);
+  }
+  if (g.c_dt == LILICORR_F32)
+    return launch_k(gemm_rows_kernel<__nv_bfloat16, float>, grid, GR_THREADS, 0, st, g);
+  return launch_k(gemm_rows_kernel<__nv_bfloat16, __nv_bfloat16>, grid, GR_THREADS, 0, st, g);
 }
 
 lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st) {

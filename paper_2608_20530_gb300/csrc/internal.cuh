@@ -285,6 +285,9 @@ constexpr int SS_LD = 16;  // floats per row of a folded-RMSNorm sums-of-squares
 int gemm_tc_ss_slots(int M, int N);
 lilicorr_status_t launch_gemm_simt(const GemmArgs& g, cudaStream_t st);
 lilicorr_status_t launch_gemm_skinny(const GemmArgs& g, cudaStream_t st);   // M <= 64
+// fp32 activations, per-sequence row counts (16 x 32 output blocks, no K split)
+bool gemm_rows_supported(const GemmArgs& g);
+lilicorr_status_t launch_gemm_rows(const GemmArgs& g, cudaStream_t st);
 bool gemm_tc_supported(const GemmArgs& g);
 lilicorr_status_t launch_gemm_tc(const GemmArgs& g, cudaStream_t st);
 // one tile of rows (M <= 128, Kd <= 512, a multiple of 64): whole-K TMA copies (gemm_small.cu)

@@ -106,3 +106,49 @@ def test_linear_one_row_tile_rejects_other_shapes():
     W = torch.randn((256, 1024), device="cuda").to(torch.bfloat16)
     with pytest.raises(ll.LilicorrError):
         ll.test_linear(A, W, path=4)                        # Kd above 512
+
+
+ROW_CASES = [  # M, N, Kd: fp32 activations at per-sequence row counts
+    (256, 512, 512), (65, 40, 1032), (1000, 200, 512), (1024, 512, 256), (17, 8, 8),
+    (300, 96, 2048),
+]
+
+
+@pytest.mark.parametrize("M,N,Kd", ROW_CASES)
+@pytest.mark.parametrize("wdt", [torch.bfloat16, torch.float32])
+def test_linear_fp32_rows(M, N, Kd, wdt):
+    """The row-block kernel (path 5) and the network's own choice for fp32 activations with
+    more than 64 rows, against fp32 PyTorch: bias, SiLU, residual, bf16 output, ragged M and
+    N, Kd over several staged chunks."""
+    ll = _ll()
+    g = torch.Generator(device="cuda").manual_seed(M * 3 + N + Kd)
+    A = torch.randn((M, Kd), generator=g, device="cuda")
+    W = (0.05 * torch.randn((N, Kd), generator=g, device="cuda")).to(wdt)
+    bias = 0.1 * torch.randn(N, generator=g, device="cuda")
+    res = torch.randn((M, N), generator=g, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for path in (5, 0) if M > 64 else (5,):
+        for act, b, r, odt in [(0, None, None, torch.float32), (1, bias, None, torch.float32),
+                               (0, bias, res, torch.float32), (1, bias, None, torch.bfloat16)]:
+            C = ll.test_linear(A, W, odt, bias=b, residual=r, act=act, path=path, status=status)
+            torch.cuda.synchronize()
+            want = _ref(A, W, b, r, act)
+            tol = 2e-2 if odt == torch.bfloat16 else 2e-5 * max(1.0, (Kd / 256) ** 0.5)
+            err = (C.float() - want).abs().max().item()
+            assert err <= tol * max(1.0, want.abs().max().item()), (path, act, odt, err)
+    assert int(status.item()) == 0
+
+
+def test_linear_fp32_rows_rejects_unaligned():
+    ll = _ll()
+    W = torch.randn((32, 96), device="cuda")
+    A = torch.randn((80, 102), device="cuda")[:, :96]     # row stride 102: not 16-byte rows
+    with pytest.raises(ll.LilicorrError):
+        ll.test_linear(A, W, path=5)
+    A = torch.randn((80, 100), device="cuda")
+    with pytest.raises(ll.LilicorrError):
+        ll.test_linear(A, torch.randn((32, 100), device="cuda"), path=5)   # Kd not a multiple of 8
+    A = torch.randn((80, 102), device="cuda")[:, :96]
+    C = ll.test_linear(A, W, path=0)                      # the network's choice falls back
+    torch.cuda.synchronize()
+    assert (C - A @ W.T).abs().max().item() < 1e-4
