@@ -212,12 +212,12 @@ bool takes_gemm_tc(const GemmArgs& g) {
 lilicorr_status_t run_gemm(const GemmArgs& g, cudaStream_t st) {
   // a folded RMSNorm only exists in the persistent tensor-core kernel
   if (g.c2 || g.ss_in) return takes_gemm_tc(g) ? launch_gemm_tc(g, st) : LILICORR_ERR_SHAPE;
-  // few rows: the split-N kernel spreads the weights over many CTAs; fp32 activations
-  // (the tensor-core kernels take bf16) at per-sequence row counts: 16 x 32 output blocks
-  // with the rows staged (256 x 512 x 512: 54 -> ~5 us), else the split-N kernel
-  if (g.M <= 64) return launch_gemm_skinny(g, st);
-  if (g.a_dt == LILICORR_F32 && g.M <= 1024)
-    return gemm_rows_supported(g) ? launch_gemm_rows(g, st) : launch_gemm_skinny(g, st);
+  // fp32 activations (the tensor-core kernels take bf16) at per-sequence row counts above
+  // 16: 16 x 32 output blocks with the rows staged (256 x 512 x 512: 54 -> ~5 us); few rows
+  // otherwise: the split-N kernel spreads the weights over many CTAs
+  if (g.a_dt == LILICORR_F32 && g.M > 16 && g.M <= 1024 && gemm_rows_supported(g))
+    return launch_gemm_rows(g, st);
+  if (g.M <= 64 || (g.a_dt == LILICORR_F32 && g.M <= 1024)) return launch_gemm_skinny(g, st);
   if (gemm_small_supported(g)) return launch_gemm_small(g, st);
   if (gemm_tc_supported(g)) return launch_gemm_tc(g, st);
   return launch_gemm_simt(g, st);

@@ -180,45 +180,69 @@ __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(GemmArgs g) {
 // ----------------------------------------------------------------------------- row-block linear
 // Per-sequence products with fp32 activations and more rows than the few-row kernel takes
 // (the target state t of a batch against W_a and the fusion layer's t block: M = B up to
-// 1024, Kd = D). CTA = 16 rows x 32 columns: lane = output column (it streams its weight
-// row in 16-byte pieces), warp = two rows; the 16 rows' activations are staged in shared
-// memory, GR_KC columns at a time, and read as broadcasts. No cross-lane reduction.
-constexpr int GR_M = 16, GR_N = 32, GR_THREADS = 256, GR_KC = 512;
+// 1024, Kd = D). CTA = 16 rows x 32 columns: lane = output column, warp = two rows. Per
+// chunk of Kd, the 16 activation rows and the 32 weight rows are staged in shared memory by
+// one round of asynchronous 16-byte copies (all in flight at once, coalesced); each lane
+// then reads its weight row and the warp's two activation rows (broadcasts). No
+// cross-lane reduction.
+constexpr int GR_M = 16, GR_N = 32, GR_THREADS = 256;
+__device__ __forceinline__ void cp16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
+               ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src) : "memory");
+}
+template <typename TW>
+struct GrCfg {
+  static constexpr int KC = sizeof(TW) == 2 ? 256 : 128;      // Kd chunk staged at a time
+  static constexpr int AS = KC + 4;                           // row strides (elements), padded
+  static constexpr int WS = KC + 16 / (int)sizeof(TW);        // so 8 lanes' 16-byte reads differ in bank
+};
 template <typename TW, typename TC>
 __global__ void __launch_bounds__(GR_THREADS) gemm_rows_kernel(GemmArgs g) {
   pdl_wait();
-  __shared__ __align__(16) float As[GR_M][GR_KC + 4];
+  using Cfg = GrCfg<TW>;
+  constexpr int KC = Cfg::KC, AS = Cfg::AS, WS = Cfg::WS;
+  constexpr int WV = 16 / (int)sizeof(TW);                    // weights per 16-byte piece
+  __shared__ __align__(16) float As[GR_M * AS];
+  __shared__ __align__(16) TW Ws[GR_N * WS];
   const float* A = static_cast<const float*>(g.A);
   const TW* W = static_cast<const TW*>(g.W);
   const int m0 = blockIdx.y * GR_M, n0 = blockIdx.x * GR_N;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int n = n0 + lane, r0 = 2 * warp;
   float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < g.Kd; k0 += GR_KC) {
-    const int kc4 = min(GR_KC, g.Kd - k0) >> 2;          // 16-byte pieces per row
-    __syncthreads();                                     // the previous chunk is consumed
-    for (int i = threadIdx.x; i < GR_M * kc4; i += GR_THREADS) {
-      const int r = i / kc4, c = 4 * (i % kc4);
-      *reinterpret_cast<float4*>(&As[r][c]) =
-          m0 + r < g.M ? *reinterpret_cast<const float4*>(A + (size_t)(m0 + r) * g.lda + k0 + c)
-                       : make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int k0 = 0; k0 < g.Kd; k0 += KC) {
+    const int kc = min(KC, g.Kd - k0);                          // a multiple of 8
+    __syncthreads();                                            // the previous chunk is consumed
+    for (int i = threadIdx.x; i < GR_M * (kc / 4); i += GR_THREADS) {
+      const int r = i / (kc / 4), c = 4 * (i % (kc / 4));
+      float* dst = &As[r * AS + c];
+      if (m0 + r < g.M) cp16(dst, A + (size_t)(m0 + r) * g.lda + k0 + c);
+      else *reinterpret_cast<float4*>(dst) = make_float4(0.f, 0.f, 0.f, 0.f);
     }
+    for (int i = threadIdx.x; i < GR_N * (kc / WV); i += GR_THREADS) {
+      const int r = i / (kc / WV), c = WV * (i % (kc / WV));
+      TW* dst = &Ws[r * WS + c];
+      if (n0 + r < g.N) cp16(dst, W + (size_t)(n0 + r) * g.ldw + k0 + c);
+      else *reinterpret_cast<uint4*>(dst) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
     __syncthreads();
-    if (n < g.N) {
-      const TW* wr = W + (size_t)n * g.ldw + k0;
+    const TW* wr = &Ws[lane * WS];
+    const float* a0p = &As[r0 * AS];
+    const float* a1p = a0p + AS;
 #pragma unroll 4
-      for (int k = 0; k < 4 * kc4; k += 8) {
-        float w[8];
-        load8(wr + k, w);
-        const float4 a0 = *reinterpret_cast<const float4*>(&As[r0][k]);
-        const float4 a1 = *reinterpret_cast<const float4*>(&As[r0][k + 4]);
-        const float4 b0 = *reinterpret_cast<const float4*>(&As[r0 + 1][k]);
-        const float4 b1 = *reinterpret_cast<const float4*>(&As[r0 + 1][k + 4]);
-        acc0 = fmaf(a0.x, w[0], fmaf(a0.y, w[1], fmaf(a0.z, w[2], fmaf(a0.w, w[3], acc0))));
-        acc0 = fmaf(a1.x, w[4], fmaf(a1.y, w[5], fmaf(a1.z, w[6], fmaf(a1.w, w[7], acc0))));
-        acc1 = fmaf(b0.x, w[0], fmaf(b0.y, w[1], fmaf(b0.z, w[2], fmaf(b0.w, w[3], acc1))));
-        acc1 = fmaf(b1.x, w[4], fmaf(b1.y, w[5], fmaf(b1.z, w[6], fmaf(b1.w, w[7], acc1))));
-      }
+    for (int k = 0; k < kc; k += 8) {
+      float w[8];
+      load8(wr + k, w);
+      const float4 a0 = *reinterpret_cast<const float4*>(a0p + k);
+      const float4 a1 = *reinterpret_cast<const float4*>(a0p + k + 4);
+      const float4 b0 = *reinterpret_cast<const float4*>(a1p + k);
+      const float4 b1 = *reinterpret_cast<const float4*>(a1p + k + 4);
+      acc0 = fmaf(a0.x, w[0], fmaf(a0.y, w[1], fmaf(a0.z, w[2], fmaf(a0.w, w[3], acc0))));
+      acc0 = fmaf(a1.x, w[4], fmaf(a1.y, w[5], fmaf(a1.z, w[6], fmaf(a1.w, w[7], acc0))));
+      acc1 = fmaf(b0.x, w[0], fmaf(b0.y, w[1], fmaf(b0.z, w[2], fmaf(b0.w, w[3], acc1))));
+      acc1 = fmaf(b1.x, w[4], fmaf(b1.y, w[5], fmaf(b1.z, w[6], fmaf(b1.w, w[7], acc1))));
     }
   }
   if (n >= g.N) return;
