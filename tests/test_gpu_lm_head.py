@@ -2,7 +2,8 @@
 (exact where the fp64 logits are not within fp32 rounding of each other; otherwise the
 chosen logits must match rank by rank), log-probabilities and normaliser within 1e-3, on
 one and several row blocks (ragged), ragged vocabulary tiles, K up to 32 and the full
-Qwen3-sized vocabulary."""
+Qwen3-sized vocabulary; up to 16 rows take the kernel with the vocabulary tile as the A
+operand."""
 import numpy as np
 import pytest
 import torch
@@ -36,7 +37,9 @@ def _check(h, W, ids, logp, lse, K, rows_to_check):
 
 
 @pytest.mark.parametrize("rows,H,V,K", [(1, 64, 1000, 4), (16, 256, 33000, 8), (130, 512, 5000, 16),
-                                        (20, 128, 257, 32), (16, 4096, 151936, 8)])
+                                        (20, 128, 257, 32), (16, 4096, 151936, 8),
+                                        (16, 128, 1000, 32), (5, 64, 4097, 16), (13, 192, 20000, 32),
+                                        (2, 64, 100, 8)])
 def test_lm_head_topk_matches_oracle(rows, H, V, K):
     ll = _ll()
     g = torch.Generator(device="cuda").manual_seed(rows * 31 + H + V)
