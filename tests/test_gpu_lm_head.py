@@ -3,7 +3,7 @@
 chosen logits must match rank by rank), log-probabilities and normaliser within 1e-3, on
 one and several row blocks (ragged), ragged vocabulary tiles, K up to 32 and the full
 Qwen3-sized vocabulary; up to 16 rows take the kernel with the vocabulary tile as the A
-operand."""
+operand, more rows the one with the hidden rows as A."""
 import numpy as np
 import pytest
 import torch
@@ -39,7 +39,8 @@ def _check(h, W, ids, logp, lse, K, rows_to_check):
 @pytest.mark.parametrize("rows,H,V,K", [(1, 64, 1000, 4), (16, 256, 33000, 8), (130, 512, 5000, 16),
                                         (20, 128, 257, 32), (16, 4096, 151936, 8),
                                         (16, 128, 1000, 32), (5, 64, 4097, 16), (13, 192, 20000, 32),
-                                        (2, 64, 100, 8)])
+                                        (2, 64, 100, 8), (33, 64, 5000, 8), (64, 256, 33000, 16),
+                                        (64, 4096, 151936, 8), (65, 128, 3000, 8)])
 def test_lm_head_topk_matches_oracle(rows, H, V, K):
     ll = _ll()
     g = torch.Generator(device="cuda").manual_seed(rows * 31 + H + V)
