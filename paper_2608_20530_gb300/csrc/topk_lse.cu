@@ -708,9 +708,10 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
                   int32_t* __restrict__ ids, float* __restrict__ logp, float* __restrict__ lse,
                   uint32_t* status) {
   pdl_wait();
-  extern __shared__ uint64_t s_dyn[];            // [P*K] keys, then [P*K] survivors
+  extern __shared__ uint64_t s_dyn[];   // [P*K] keys, [P*K] survivors, then P (max, sum) pairs
   uint64_t* s_keys = s_dyn;
   uint64_t* s_merge = s_dyn + (size_t)P * K;
+  float2* s_ms = reinterpret_cast<float2*>(s_dyn + 2 * (size_t)P * K);
   __shared__ uint64_t s_top[LILICORR_MAX_K];
   __shared__ int s_count;
   __shared__ uint64_t s_bound;
@@ -722,13 +723,16 @@ topk_merge_kernel(const unsigned char* __restrict__ recs, int P, int rows, int K
     const int32_t id = reinterpret_cast<const int32_t*>(r + 8 + 4 * (size_t)K)[i % K];
     s_keys[i] = id < 0 ? 0ull : make_key(v, (uint32_t)id);
   }
+  for (int p = tid; p < P; p += TK_THREADS) {     // the records' (max, sum), same pass
+    const float* r = reinterpret_cast<const float*>(recs + ((size_t)p * rows + row) * rb);
+    s_ms[p] = make_float2(r[0], r[1]);
+  }
   __syncthreads();
   cta_select<TK_THREADS>(s_keys, P, K, K, s_merge, &s_count, &s_bound, s_top);
   if (warp == 0) {
     float pm = -INFINITY, ps = 0.f;
     for (int p = lane; p < P; p += 32) {
-      const float* r = reinterpret_cast<const float*>(recs + ((size_t)p * rows + row) * rb);
-      const float rm = r[0], rs = r[1];
+      const float rm = s_ms[p].x, rs = s_ms[p].y;
       if (rm == -INFINITY) continue;
       if (rm > pm) { ps = ps * ex2((pm - rm) * LOG2E) + rs; pm = rm; }
       else ps += rs * ex2((rm - pm) * LOG2E);
@@ -818,7 +822,8 @@ lilicorr_status_t launch_topk_merge(const void* partials, int P, int rows, int K
   if (P < 1 || K < 1 || P * K > TOPK_MERGE_KEYS_MAX) return LILICORR_ERR_SHAPE;
   static bool configured[64] = {false};
   LL_TRY(allow_max_dynamic_smem(topk_merge_kernel, configured));
-  LL_TRY(launch_k(topk_merge_kernel, rows, TK_THREADS, 2 * (size_t)P * K * sizeof(uint64_t), st,
+  LL_TRY(launch_k(topk_merge_kernel, rows, TK_THREADS,
+                  2 * (size_t)P * K * sizeof(uint64_t) + (size_t)P * sizeof(float2), st,
                   static_cast<const unsigned char*>(partials), P, rows, K, ids, logp, lse, status));
   return LILICORR_OK;
 }
