@@ -3,9 +3,9 @@
  * selection path; they expose internal building blocks so tests can check them
  * one at a time.
  *
- * The path switch below (lilicorr_test_fused_path) changes process-global dispatch state
- * that every head and every host thread reads when it enqueues a call. It is not
- * synchronised: set it only while no other thread is enqueueing work through the library,
+ * The path switches below (lilicorr_test_fused_path, lilicorr_test_attention_path) change
+ * process-global dispatch state that every head and every host thread reads when it
+ * enqueues a call. They are not synchronised: set it only while no other thread is enqueueing work through the library,
  * and put the default back afterwards.
  */
 #ifndef LILICORR_TESTING_H_
